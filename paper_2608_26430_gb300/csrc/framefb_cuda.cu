@@ -1,0 +1,315 @@
+// Launchers of libframefb: argument validation, tiling, workspace sizing and
+// the launches of the tile, dC-reduction and merge kernels.
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstring>
+#include <vector>
+
+#include "framefb.h"
+#include "framefb_kernels.cuh"
+#include "plan_internal.h"
+#include "plan_layout.h"
+
+namespace {
+
+using ffb::kMaxMats;
+using ffb::kThreads;
+using ffb::kTmax;
+
+constexpr int kSmemBudget = 227 * 1024;  // dynamic shared memory per CTA on sm_103a
+
+inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+const FfbPlanHeader* plan_header(const framefb_plan* p) {
+  if (!p || p->image.size() < sizeof(FfbPlanHeader)) return nullptr;
+  const FfbPlanHeader* h = reinterpret_cast<const FfbPlanHeader*>(p->image.data());
+  if (h->magic != FFB_PLAN_MAGIC || h->version != FFB_PLAN_VERSION || h->P != kThreads) return nullptr;
+  if (static_cast<size_t>(h->total_bytes) != p->image.size()) return nullptr;
+  return h;
+}
+
+bool frame_ok(const framefb_dev_frame* f, int32_t d) {
+  return f && f->dft_groups && f->k == 16 && f->d == d && f->ncols == d && f->rho * 16 == d && f->val &&
+         f->colptr && f->rowidx;
+}
+
+// Group-0 block of column rho (subspace 1, Spectral Tetris row 0, part 0):
+// every column of a k = 16 DFT-group frame stores 32 entries, so the block
+// starts at entry 32 * rho.
+const float* twiddle_source(const framefb_dev_frame* f) { return f->val + static_cast<size_t>(32) * f->rho; }
+
+struct Prepared {
+  ffb::LaunchK* args;  // heap: too large for the stack of some callers
+  ffb::ReduceK* red;
+  int grid;
+  size_t smem;
+  size_t ws_bytes;
+  bool reg;
+};
+
+void* tile_kernel_ptr(framefb_dtype dt, int mode, bool reg) {
+#define FFB_CASE(E, M)                                                      \
+  case M:                                                                   \
+    return reg ? reinterpret_cast<void*>(ffb::tile_kernel<E, M, true>)      \
+               : reinterpret_cast<void*>(ffb::tile_kernel<E, M, false>);
+  if (dt == FRAMEFB_BF16) {
+    switch (mode) {
+      FFB_CASE(__nv_bfloat16, 1)
+      FFB_CASE(__nv_bfloat16, 2)
+      FFB_CASE(__nv_bfloat16, 4)
+      FFB_CASE(__nv_bfloat16, 6)
+      FFB_CASE(__nv_bfloat16, 7)
+      default: return nullptr;
+    }
+  }
+  switch (mode) {
+    FFB_CASE(float, 1)
+    FFB_CASE(float, 2)
+    FFB_CASE(float, 4)
+    FFB_CASE(float, 6)
+    FFB_CASE(float, 7)
+    default: return nullptr;
+  }
+#undef FFB_CASE
+}
+
+// Validate one chunk of matrices and fill the launch parameters.
+framefb_status prepare(const framefb_mat* mats, int32_t nmats, int32_t ops, framefb_dtype dt, Prepared& P) {
+  const size_t esz = dt == FRAMEFB_BF16 ? 2 : 4;
+  const bool F = ops & FRAMEFB_OP_FORWARD, D = ops & FRAMEFB_OP_BACKWARD_DX, C = ops & FRAMEFB_OP_GRAD_COEFF;
+  std::memset(P.args, 0, sizeof(ffb::LaunchK));
+  std::memset(P.red, 0, sizeof(ffb::ReduceK));
+  bool reg = true;
+  int32_t nnz_max = 0;
+  for (int32_t j = 0; j < nmats; ++j) {
+    const FfbPlanHeader* h = plan_header(mats[j].plan);
+    if (!h) return FRAMEFB_EINVAL;
+    if (h->EZ > ffb::kEreg || h->EG > ffb::kEreg) reg = false;
+    nnz_max = std::max(nnz_max, h->nnz);
+  }
+  int64_t units = 0;
+  size_t smem = 0;
+  for (int32_t j = 0; j < nmats; ++j) {
+    const framefb_mat& M = mats[j];
+    const FfbPlanHeader* h = plan_header(M.plan);
+    if (M.N < 0 || M.n <= 0 || M.m <= 0) return FRAMEFB_EINVAL;
+    if (!frame_ok(M.fin, M.n) || !frame_ok(M.fout, M.m)) return FRAMEFB_EINVAL;
+    if (h->n != M.n || h->m != M.m) return FRAMEFB_EINVAL;
+    if (!M.plan_dev || !aligned16(M.plan_dev)) return FRAMEFB_EINVAL;
+    if (!std::isfinite(M.scale)) return FRAMEFB_EINVAL;
+    if ((F || D) && h->nnz > 0 && !M.c_val) return FRAMEFB_EINVAL;
+    const bool needX = F || C, needdY = D || C;
+    if (M.N > 0) {
+      if ((needX || D) && (M.ldx < M.n || (M.ldx * esz) % 16)) return FRAMEFB_EINVAL;
+      if ((needdY || F) && (M.ldy < M.m || (M.ldy * esz) % 16)) return FRAMEFB_EINVAL;
+      if (needX && (!M.X || !aligned16(M.X))) return FRAMEFB_EINVAL;
+      if (needdY && (!M.dY || !aligned16(M.dY))) return FRAMEFB_EINVAL;
+      if (F && (!M.Y || !aligned16(M.Y))) return FRAMEFB_EINVAL;
+      if (D && (!M.dX || !aligned16(M.dX))) return FRAMEFB_EINVAL;
+    }
+    if (C && h->nnz > 0 && !M.dC) return FRAMEFB_EINVAL;
+    // tokens per tile: as many as fit in shared memory, at most kTmax
+    int T = kTmax;
+    while (T > 1 && ffb_tile_layout(*h, ops, T, C && !reg).total * 4 > kSmemBudget) --T;
+    const size_t bytes = static_cast<size_t>(ffb_tile_layout(*h, ops, T, C && !reg).total) * 4;
+    if (bytes > static_cast<size_t>(kSmemBudget)) return FRAMEFB_EUNSUPPORTED;
+    smem = std::max(smem, bytes);
+    const int32_t ntiles = (M.N + T - 1) / T;
+    ffb::MatK& K = P.args->m[j];
+    K.X = M.X;
+    K.dX = M.dX;
+    K.dY = M.dY;
+    K.Y = M.Y;
+    K.plan = static_cast<const uint8_t*>(M.plan_dev);
+    K.c_val = M.c_val;
+    K.tw_in = twiddle_source(M.fin);
+    K.tw_out = twiddle_source(M.fout);
+    K.ldx = M.ldx;
+    K.ldy = M.ldy;
+    K.N = M.N;
+    K.T = T;
+    K.ubeg = static_cast<int32_t>(units);
+    K.ntiles = ntiles;
+    K.seff = M.scale / 16.f;
+    ffb::ReduceMat& R = P.red->m[j];
+    R.dC = M.dC;
+    R.ubeg = K.ubeg;
+    R.ntiles = ntiles;
+    R.nnz = h->nnz;
+    R.seff = K.seff;
+    units += ntiles;
+    if (units > INT32_MAX / 2) return FRAMEFB_EUNSUPPORTED;
+  }
+  P.args->nmats = nmats;
+  P.args->total_units = static_cast<int32_t>(units);
+  P.args->stride = (nnz_max + 63) & ~63;
+  P.red->nmats = nmats;
+  P.red->total_units = static_cast<int32_t>(units);
+  P.red->stride = P.args->stride;
+  P.reg = reg;
+  P.smem = std::max<size_t>(smem, 16);
+  P.grid = 0;
+  P.ws_bytes = 0;
+  if (units == 0) return FRAMEFB_OK;
+  void* fn = tile_kernel_ptr(dt, ops, reg);
+  if (!fn) return FRAMEFB_EINVAL;
+  int dev = 0, sms = 0, per_sm = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return FRAMEFB_ECUDA;
+  if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return FRAMEFB_ECUDA;
+  if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(P.smem)) !=
+      cudaSuccess)
+    return FRAMEFB_ECUDA;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, kThreads, P.smem) != cudaSuccess)
+    return FRAMEFB_ECUDA;
+  if (per_sm < 1) return FRAMEFB_EUNSUPPORTED;
+  P.grid = static_cast<int>(std::min<int64_t>(static_cast<int64_t>(sms) * per_sm, units));
+  P.red->grid = P.grid;
+  if (C) P.ws_bytes = static_cast<size_t>(P.grid + nmats) * P.args->stride * sizeof(float) + 256;
+  return FRAMEFB_OK;
+}
+
+struct Buffers {
+  std::vector<uint8_t> a, r;
+  Buffers() : a(sizeof(ffb::LaunchK)), r(sizeof(ffb::ReduceK)) {}
+  Prepared prep() {
+    Prepared p{};
+    p.args = reinterpret_cast<ffb::LaunchK*>(a.data());
+    p.red = reinterpret_cast<ffb::ReduceK*>(r.data());
+    return p;
+  }
+};
+
+bool ops_ok(int32_t ops) { return ops == 1 || ops == 2 || ops == 4 || ops == 6 || ops == 7; }
+
+}  // namespace
+
+extern "C" size_t framefb_workspace_size(const framefb_mat* mats, int32_t nmats, int32_t ops) {
+  if (!mats || nmats <= 0 || !ops_ok(ops)) return 0;
+  Buffers b;
+  size_t need = 0;
+  for (int32_t j0 = 0; j0 < nmats; j0 += kMaxMats) {
+    Prepared P = b.prep();
+    // dtype does not change the workspace; bf16 is used for the occupancy query
+    if (prepare(mats + j0, std::min(kMaxMats, nmats - j0), ops, FRAMEFB_BF16, P) != FRAMEFB_OK) return 0;
+    need = std::max(need, P.ws_bytes);
+  }
+  return need;
+}
+
+extern "C" framefb_status framefb_run(const framefb_mat* mats, int32_t nmats, int32_t ops, framefb_dtype dtype,
+                                      void* ws, size_t ws_bytes, void* stream) {
+  if (nmats < 0 || (nmats > 0 && !mats) || !ops_ok(ops)) return FRAMEFB_EINVAL;
+  if (dtype != FRAMEFB_F32 && dtype != FRAMEFB_BF16) return FRAMEFB_EINVAL;
+  if (nmats == 0) return FRAMEFB_OK;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  Buffers b;
+  // validate every chunk before queueing anything
+  for (int32_t j0 = 0; j0 < nmats; j0 += kMaxMats) {
+    Prepared P = b.prep();
+    const framefb_status s = prepare(mats + j0, std::min(kMaxMats, nmats - j0), ops, dtype, P);
+    if (s != FRAMEFB_OK) return s;
+    if (P.ws_bytes > 0) {
+      if (!ws || ws_bytes < P.ws_bytes) return FRAMEFB_EWORKSPACE;
+      if (reinterpret_cast<uintptr_t>(ws) & 255u) return FRAMEFB_EINVAL;
+    }
+  }
+  for (int32_t j0 = 0; j0 < nmats; j0 += kMaxMats) {
+    const int32_t nm = std::min(kMaxMats, nmats - j0);
+    Prepared P = b.prep();
+    const framefb_status s = prepare(mats + j0, nm, ops, dtype, P);
+    if (s != FRAMEFB_OK) return s;
+    if (P.grid == 0) {
+      if (ops & FRAMEFB_OP_GRAD_COEFF) {  // no tokens: the gradient is zero
+        for (int32_t j = 0; j < nm; ++j)
+          if (P.red->m[j].nnz > 0 &&
+              cudaMemsetAsync(P.red->m[j].dC, 0, sizeof(float) * P.red->m[j].nnz, st) != cudaSuccess)
+            return FRAMEFB_ECUDA;
+      }
+      continue;
+    }
+    P.args->partial = static_cast<float*>(ws);
+    P.red->partial = static_cast<const float*>(ws);
+    void* fn = tile_kernel_ptr(dtype, ops, P.reg);
+    void* kargs[] = {P.args};
+    if (cudaLaunchKernel(fn, dim3(P.grid), dim3(kThreads), kargs, P.smem, st) != cudaSuccess)
+      return FRAMEFB_ECUDA;
+    if (ops & FRAMEFB_OP_GRAD_COEFF) {
+      int nnz_max = 0;
+      for (int32_t j = 0; j < nm; ++j) nnz_max = std::max(nnz_max, P.red->m[j].nnz);
+      if (nnz_max > 0) {
+        void* rargs[] = {P.red};
+        const dim3 rg((nnz_max + 255) / 256, nm);
+        if (cudaLaunchKernel(reinterpret_cast<void*>(ffb::dc_reduce_kernel), rg, dim3(256), rargs, 0, st) !=
+            cudaSuccess)
+          return FRAMEFB_ECUDA;
+      }
+    }
+  }
+  return FRAMEFB_OK;
+}
+
+extern "C" framefb_status framefb_forward(const framefb_mat* mats, int32_t nmats, framefb_dtype dtype, void* ws,
+                                          size_t ws_bytes, void* stream) {
+  return framefb_run(mats, nmats, FRAMEFB_OP_FORWARD, dtype, ws, ws_bytes, stream);
+}
+extern "C" framefb_status framefb_backward_dx(const framefb_mat* mats, int32_t nmats, framefb_dtype dtype,
+                                              void* ws, size_t ws_bytes, void* stream) {
+  return framefb_run(mats, nmats, FRAMEFB_OP_BACKWARD_DX, dtype, ws, ws_bytes, stream);
+}
+extern "C" framefb_status framefb_grad_coeff(const framefb_mat* mats, int32_t nmats, framefb_dtype dtype, void* ws,
+                                             size_t ws_bytes, void* stream) {
+  return framefb_run(mats, nmats, FRAMEFB_OP_GRAD_COEFF, dtype, ws, ws_bytes, stream);
+}
+extern "C" framefb_status framefb_backward(const framefb_mat* mats, int32_t nmats, framefb_dtype dtype, void* ws,
+                                           size_t ws_bytes, void* stream) {
+  return framefb_run(mats, nmats, FRAMEFB_OP_BACKWARD_DX | FRAMEFB_OP_GRAD_COEFF, dtype, ws, ws_bytes, stream);
+}
+extern "C" framefb_status framefb_fused_fwd_bwd(const framefb_mat* mats, int32_t nmats, framefb_dtype dtype,
+                                                void* ws, size_t ws_bytes, void* stream) {
+  return framefb_run(mats, nmats, FRAMEFB_OP_FORWARD | FRAMEFB_OP_BACKWARD_DX | FRAMEFB_OP_GRAD_COEFF, dtype, ws,
+                     ws_bytes, stream);
+}
+
+extern "C" framefb_status framefb_merge(const void* W0, framefb_dtype dtype, int32_t m, int32_t n, int64_t ldw,
+                                        const framefb_dev_frame* fin, const framefb_dev_frame* fout,
+                                        const framefb_plan* plan, const void* plan_dev, const float* c_vals,
+                                        int32_t T, float scale, void* Wout, void* stream) {
+  if (dtype != FRAMEFB_F32 && dtype != FRAMEFB_BF16) return FRAMEFB_EINVAL;
+  const FfbPlanHeader* h = plan_header(plan);
+  if (!h || m <= 0 || n <= 0 || T < 0 || h->m != m || h->n != n) return FRAMEFB_EINVAL;
+  if (!frame_ok(fin, n) || !frame_ok(fout, m)) return FRAMEFB_EINVAL;
+  const size_t esz = dtype == FRAMEFB_BF16 ? 2 : 4;
+  if (ldw < n || (ldw * esz) % 16 || !std::isfinite(scale)) return FRAMEFB_EINVAL;
+  if (T == 0) return FRAMEFB_OK;
+  if (!W0 || !Wout || !plan_dev || !aligned16(W0) || !aligned16(Wout) || !aligned16(plan_dev)) return FRAMEFB_EINVAL;
+  if (h->nnz > 0 && !c_vals) return FRAMEFB_EINVAL;
+  {  // Wout must not overlap W0
+    const uintptr_t w0 = reinterpret_cast<uintptr_t>(W0), w1 = w0 + static_cast<size_t>(m) * ldw * esz;
+    const uintptr_t o0 = reinterpret_cast<uintptr_t>(Wout), o1 = o0 + static_cast<size_t>(T) * m * ldw * esz;
+    if (o0 < w1 && w0 < o1) return FRAMEFB_EINVAL;
+  }
+  ffb::MergeK a{};
+  a.W0 = W0;
+  a.Wout = Wout;
+  a.plan = static_cast<const uint8_t*>(plan_dev);
+  a.c_vals = c_vals;
+  a.fin_val = fin->val;
+  a.fout_val = fout->val;
+  a.ldw = ldw;
+  a.m = m;
+  a.n = n;
+  a.rho_in = fin->rho;
+  a.rho_out = fout->rho;
+  a.nnz = h->nnz;
+  a.T = T;
+  a.seff = scale / 16.f;
+  void* kargs[] = {&a};
+  void* fn = dtype == FRAMEFB_BF16 ? reinterpret_cast<void*>(ffb::merge_kernel<__nv_bfloat16>)
+                                   : reinterpret_cast<void*>(ffb::merge_kernel<float>);
+  if (cudaLaunchKernel(fn, dim3(h->Gm, T), dim3(256), kargs, 0, static_cast<cudaStream_t>(stream)) != cudaSuccess)
+    return FRAMEFB_ECUDA;
+  return FRAMEFB_OK;
+}

@@ -1,0 +1,491 @@
+// Host side of libframefb: frame construction (S1), support sampling (S2),
+// plan building and status strings.  Plain C++17, no CUDA calls.
+#include "framefb.h"
+#include "plan_layout.h"
+#include "plan_internal.h"
+
+#include <algorithm>
+#include <cmath>
+#include <cstdlib>
+#include <cstring>
+#include <new>
+#include <unordered_set>
+#include <vector>
+
+extern "C" const char* framefb_status_string(int32_t status) {
+  switch (status) {
+    case FRAMEFB_OK: return "ok";
+    case FRAMEFB_EINVAL: return "invalid argument";
+    case FRAMEFB_EUNSUPPORTED: return "unsupported parameters";
+    case FRAMEFB_ENOMEM: return "out of host memory";
+    case FRAMEFB_ECUDA: return "CUDA runtime error";
+    case FRAMEFB_EWORKSPACE: return "workspace missing or too small";
+    default: return "unknown status";
+  }
+}
+
+extern "C" int32_t framefb_abi_version(void) { return FRAMEFB_ABI_VERSION; }
+
+namespace {
+
+// ---------------------------------------------------------------------------
+// S1: Spectral Tetris (Sec. 3.2 step 1; appendix "Spectral Tetris").
+// F is rho_c x d_c; every row must receive squared norm d_c/rho_c and every
+// column unit norm.  Norms are tracked exactly in units of 1/rho_c: a row
+// needs d_c units and a full entry 1 contributes rho_c units.  Ones are placed
+// while at least rho_c units remain; a remainder 0 < x < 1 closes the row with
+// T(x) = (1/sqrt2)[[sqrt x, sqrt x], [sqrt(2-x), -sqrt(2-x)]] in the next two
+// columns, whose lower row hands 2 - x to the next row.
+// ---------------------------------------------------------------------------
+struct StRow { int32_t first, last; };
+
+bool spectral_tetris(int32_t rho_c, int32_t d_c, std::vector<double>& F, std::vector<StRow>& sup) {
+  if (rho_c < 1 || d_c < 2 * rho_c) return false;
+  F.assign(static_cast<size_t>(rho_c) * d_c, 0.0);
+  int64_t col = 0, handed = 0;
+  for (int32_t r = 0; r < rho_c; ++r) {
+    int64_t rem = static_cast<int64_t>(d_c) - handed;
+    if (rem < 0) return false;
+    while (rem >= rho_c) {
+      if (col >= d_c) return false;
+      F[static_cast<size_t>(r) * d_c + col] = 1.0;
+      ++col;
+      rem -= rho_c;
+    }
+    if (rem > 0) {
+      if (r + 1 >= rho_c || col + 1 >= d_c) return false;
+      const double top = std::sqrt(static_cast<double>(rem) / (2.0 * rho_c));
+      const double bot = std::sqrt(static_cast<double>(2 * rho_c - rem) / (2.0 * rho_c));
+      F[static_cast<size_t>(r) * d_c + col] = top;
+      F[static_cast<size_t>(r) * d_c + col + 1] = top;
+      F[static_cast<size_t>(r + 1) * d_c + col] = bot;
+      F[static_cast<size_t>(r + 1) * d_c + col + 1] = -bot;
+      col += 2;
+      handed = 2 * static_cast<int64_t>(rho_c) - rem;
+    } else {
+      handed = 0;
+    }
+  }
+  if (col != d_c) return false;
+  sup.assign(rho_c, StRow{-1, -1});
+  for (int32_t r = 0; r < rho_c; ++r) {
+    for (int32_t j = 0; j < d_c; ++j) {
+      if (F[static_cast<size_t>(r) * d_c + j] != 0.0) {
+        if (sup[r].first < 0) sup[r].first = j;
+        sup[r].last = j;
+      }
+    }
+    if (sup[r].first < 0) return false;
+  }
+  return true;
+}
+
+template <typename T>
+T* alloc_array(size_t n) {
+  return static_cast<T*>(std::malloc(std::max<size_t>(n, 1) * sizeof(T)));
+}
+
+}  // namespace
+
+extern "C" void framefb_frame_free(framefb_frame* f) {
+  if (!f) return;
+  std::free(f->csc_colptr);
+  std::free(f->csc_rowidx);
+  std::free(f->csc_val);
+  std::free(f->csr_rowptr);
+  std::free(f->csr_colidx);
+  std::free(f->csr_val);
+  std::free(f->grp_row0);
+  std::free(f->grp_nrows);
+  std::memset(f, 0, sizeof(*f));
+}
+
+// S1: (k, rho, d) tight fusion frame -- Sec. 3.2 steps (1)-(3), appendix example.
+extern "C" framefb_status framefb_frame_build(int32_t d, const framefb_frame_params* params,
+                                              framefb_frame* out) {
+  if (!out) return FRAMEFB_EINVAL;
+  std::memset(out, 0, sizeof(*out));
+  if (!params) return FRAMEFB_EINVAL;
+  const int32_t k = params->k, rho = params->rho;
+  if (d <= 0 || (d & 1) || k < 1 || rho < 2 || (rho & 1)) return FRAMEFB_EINVAL;
+  if (static_cast<int64_t>(k) * rho > (int64_t{1} << 30) || d > (1 << 30)) return FRAMEFB_EINVAL;
+  const int32_t rho_c = rho / 2, d_c = d / 2;
+
+  std::vector<double> F;
+  std::vector<StRow> sup;
+  try {
+    if (!spectral_tetris(rho_c, d_c, F, sup)) return FRAMEFB_EUNSUPPORTED;
+  } catch (const std::bad_alloc&) {
+    return FRAMEFB_ENOMEM;
+  }
+  // Modulation is tight when no two columns of F sharing a row are congruent
+  // mod k (the k-th-root sums cancel every other pair): k >= widest row support.
+  for (const StRow& s : sup)
+    if (s.last - s.first + 1 > k) return FRAMEFB_EUNSUPPORTED;
+
+  const int32_t ncols = k * rho;
+  int64_t nnz = 0;
+  for (const StRow& s : sup) nnz += static_cast<int64_t>(k) * 2 * 2 * (s.last - s.first + 1);
+  out->d = d;
+  out->k = k;
+  out->rho = rho;
+  out->ncols = ncols;
+  out->nnz = nnz;
+  out->A = static_cast<double>(k) * rho / d;
+  out->scale = params->parseval ? 1.0 / std::sqrt(out->A) : 1.0;
+  out->ngroups = rho_c;
+  out->dft_groups = (static_cast<int64_t>(k) * rho == d) ? 1 : 0;
+
+  out->csc_colptr = alloc_array<int64_t>(ncols + 1);
+  out->csc_rowidx = alloc_array<int32_t>(nnz);
+  out->csc_val = alloc_array<double>(nnz);
+  out->csr_rowptr = alloc_array<int64_t>(static_cast<size_t>(d) + 1);
+  out->csr_colidx = alloc_array<int32_t>(nnz);
+  out->csr_val = alloc_array<double>(nnz);
+  out->grp_row0 = alloc_array<int32_t>(rho_c);
+  out->grp_nrows = alloc_array<int32_t>(rho_c);
+  if (!out->csc_colptr || !out->csc_rowidx || !out->csc_val || !out->csr_rowptr || !out->csr_colidx ||
+      !out->csr_val || !out->grp_row0 || !out->grp_nrows) {
+    framefb_frame_free(out);
+    return FRAMEFB_ENOMEM;
+  }
+  for (int32_t r = 0; r < rho_c; ++r) {
+    out->grp_row0[r] = 2 * sup[r].first;
+    out->grp_nrows[r] = 2 * (sup[r].last - sup[r].first + 1);
+  }
+
+  // Modulation by omega^{(i j) mod k} (appendix "Modulation"), unit-norm
+  // scaling by sqrt(rho_c/d_c), optional Parseval scaling, and realification
+  // x + iy -> [[x, -y], [y, x]] applied to the frame-vector rows.
+  const double two_pi = 6.283185307179586476925286766559;
+  const double unit = std::sqrt(static_cast<double>(rho_c) / d_c) * out->scale;
+  int64_t pos = 0;
+  out->csc_colptr[0] = 0;
+  for (int32_t c = 0; c < ncols; ++c) {
+    const int32_t i = c / rho, r = (c % rho) / 2, s = c % 2;
+    for (int32_t j = sup[r].first; j <= sup[r].last; ++j) {
+      const double f = F[static_cast<size_t>(r) * d_c + j] * unit;
+      const int64_t e = (static_cast<int64_t>(i) * j) % k;
+      const double ang = two_pi * static_cast<double>(e) / k;
+      const double zr = f * std::cos(ang), zi = f * std::sin(ang);
+      out->csc_rowidx[pos] = 2 * j;
+      out->csc_val[pos] = (s == 0) ? zr : zi;
+      ++pos;
+      out->csc_rowidx[pos] = 2 * j + 1;
+      out->csc_val[pos] = (s == 0) ? -zi : zr;
+      ++pos;
+    }
+    out->csc_colptr[c + 1] = pos;
+  }
+  // CSR by counting transpose (columns come out ascending within each row).
+  std::vector<int64_t> fill(static_cast<size_t>(d) + 1, 0);
+  for (int64_t q = 0; q < nnz; ++q) fill[out->csc_rowidx[q] + 1]++;
+  for (int32_t j = 0; j < d; ++j) fill[j + 1] += fill[j];
+  std::memcpy(out->csr_rowptr, fill.data(), (static_cast<size_t>(d) + 1) * sizeof(int64_t));
+  for (int32_t c = 0; c < ncols; ++c) {
+    for (int64_t q = out->csc_colptr[c]; q < out->csc_colptr[c + 1]; ++q) {
+      const int64_t dst = fill[out->csc_rowidx[q]]++;
+      out->csr_colidx[dst] = c;
+      out->csr_val[dst] = out->csc_val[q];
+    }
+  }
+  return FRAMEFB_OK;
+}
+
+// ---------------------------------------------------------------------------
+// S2: support sampling (Sec. 3.3: random positions shared across layers).
+// splitmix64 stream; uniform_int(R) = ((x >> 11) * R) >> 53 with a 128-bit
+// product; uniform_01 = (x >> 11) * 2^-53; duplicates are discarded.
+// ---------------------------------------------------------------------------
+namespace {
+struct SplitMix64 {
+  uint64_t state;
+  uint64_t next() {
+    state += 0x9E3779B97F4A7C15ull;
+    uint64_t z = state;
+    z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+    z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+    return z ^ (z >> 31);
+  }
+  uint64_t uniform_int(uint64_t r) {
+    const unsigned __int128 p = static_cast<unsigned __int128>(next() >> 11) * r;
+    return static_cast<uint64_t>(p >> 53);
+  }
+  double uniform_01() { return static_cast<double>(next() >> 11) * (1.0 / 9007199254740992.0); }
+};
+}  // namespace
+
+extern "C" framefb_status framefb_support_build(int32_t rows, int32_t cols, int64_t nnz, uint64_t seed,
+                                                int32_t mode, double zipf_s, int32_t k, int32_t* row,
+                                                int32_t* col, int64_t* csr_rowptr, int32_t* csc_perm) {
+  if (rows <= 0 || cols <= 0 || nnz < 0) return FRAMEFB_EINVAL;
+  const int64_t total = static_cast<int64_t>(rows) * cols;
+  if (nnz > total || nnz > (int64_t{1} << 31) - 1) return FRAMEFB_EINVAL;
+  if (nnz > 0 && (!row || !col)) return FRAMEFB_EINVAL;
+  if (mode == FRAMEFB_SUPPORT_BLOCKDIAG) {
+    if (k < 1 || rows % k || cols % k) return FRAMEFB_EINVAL;
+    if (nnz > static_cast<int64_t>(k) * (rows / k) * (cols / k)) return FRAMEFB_EINVAL;
+  } else if (mode == FRAMEFB_SUPPORT_ZIPF_ROWS) {
+    if (!(zipf_s > 0.0) || !std::isfinite(zipf_s)) return FRAMEFB_EINVAL;
+  } else if (mode != FRAMEFB_SUPPORT_UNIFORM) {
+    return FRAMEFB_EINVAL;
+  }
+  try {
+    SplitMix64 rng{seed};
+    std::vector<double> cdf;
+    if (mode == FRAMEFB_SUPPORT_ZIPF_ROWS) {
+      cdf.resize(rows);
+      double acc = 0.0;
+      for (int32_t r = 1; r <= rows; ++r) {
+        acc += std::pow(static_cast<double>(r), -zipf_s);
+        cdf[r - 1] = acc;
+      }
+    }
+    std::unordered_set<uint64_t> seen;
+    seen.reserve(static_cast<size_t>(nnz) * 2 + 1);
+    std::vector<uint64_t> keys;
+    keys.reserve(static_cast<size_t>(nnz));
+    while (static_cast<int64_t>(keys.size()) < nnz) {
+      uint64_t a, b;
+      if (mode == FRAMEFB_SUPPORT_UNIFORM) {
+        const uint64_t p = rng.uniform_int(static_cast<uint64_t>(total));
+        a = p / cols;
+        b = p % cols;
+      } else if (mode == FRAMEFB_SUPPORT_ZIPF_ROWS) {
+        const double u = rng.uniform_01() * cdf.back();
+        a = static_cast<uint64_t>(std::upper_bound(cdf.begin(), cdf.end(), u) - cdf.begin());
+        if (a >= static_cast<uint64_t>(rows)) a = rows - 1;
+        b = rng.uniform_int(static_cast<uint64_t>(cols));
+      } else {
+        const uint64_t i = rng.uniform_int(static_cast<uint64_t>(k));
+        const uint64_t rb = rows / k, cb = cols / k;
+        a = i * rb + rng.uniform_int(rb);
+        b = i * cb + rng.uniform_int(cb);
+      }
+      const uint64_t key = a * static_cast<uint64_t>(cols) + b;
+      if (seen.insert(key).second) keys.push_back(key);
+    }
+    std::sort(keys.begin(), keys.end());
+    for (int64_t q = 0; q < nnz; ++q) {
+      row[q] = static_cast<int32_t>(keys[q] / cols);
+      col[q] = static_cast<int32_t>(keys[q] % cols);
+    }
+    if (csr_rowptr) {
+      std::fill(csr_rowptr, csr_rowptr + rows + 1, 0);
+      for (int64_t q = 0; q < nnz; ++q) csr_rowptr[row[q] + 1]++;
+      for (int32_t a = 0; a < rows; ++a) csr_rowptr[a + 1] += csr_rowptr[a];
+    }
+    if (csc_perm) {
+      std::vector<int32_t> perm(static_cast<size_t>(nnz));
+      for (int64_t q = 0; q < nnz; ++q) perm[q] = static_cast<int32_t>(q);
+      std::sort(perm.begin(), perm.end(), [&](int32_t x, int32_t y) {
+        return col[x] != col[y] ? col[x] < col[y] : row[x] < row[y];
+      });
+      std::memcpy(csc_perm, perm.data(), static_cast<size_t>(nnz) * sizeof(int32_t));
+    }
+  } catch (const std::bad_alloc&) {
+    return FRAMEFB_ENOMEM;
+  }
+  return FRAMEFB_OK;
+}
+
+// ---------------------------------------------------------------------------
+// Plan: the support re-indexed group-major and cut into per-thread chunks.
+// ---------------------------------------------------------------------------
+namespace {
+
+// Paper column c = i*rho + 2r + s  ->  group-major x = 32 r + 2 i + s (k = 16).
+inline int32_t group_major(int32_t c, int32_t rho) {
+  const int32_t i = c / rho, rr = c % rho;
+  return FFB_GROUP * (rr / 2) + 2 * i + (rr & 1);
+}
+
+struct Entry { int32_t key0, key1, q; };
+
+// Cut `ent` (sorted by key0, key1) into P chunks of E entries.  Each run of
+// equal key0 inside a chunk stores its partial sum once, at its last entry:
+// the first run of a key goes to that key's own slot phys(key0); later runs
+// (the key continues from an earlier chunk) go to overflow slots base + o.
+// Returns per-entry store targets and the fix-up list.
+void cut_chunks(const std::vector<Entry>& ent, int32_t P, int32_t E, int32_t base, int32_t nkeys,
+                std::vector<int32_t>& store, std::vector<int32_t>& fix, int32_t& novf) {
+  const int32_t nnz = static_cast<int32_t>(ent.size());
+  store.assign(nnz, FFB_NO_STORE);
+  std::vector<uint8_t> seen(nkeys, 0);
+  std::vector<int32_t> first_ovf(nkeys, -1), n_ovf(nkeys, 0);
+  novf = 0;
+  for (int32_t p = 0; p < P; ++p) {
+    const int32_t lo = p * E, hi = std::min(nnz, (p + 1) * E);
+    for (int32_t e = lo; e < hi; ++e) {
+      const bool run_end = (e + 1 == hi) || ent[e + 1].key0 != ent[e].key0;
+      if (!run_end) continue;
+      const int32_t key = ent[e].key0;
+      if (!seen[key]) {
+        seen[key] = 1;
+        store[e] = ffb_phys(key);
+      } else {
+        if (first_ovf[key] < 0) first_ovf[key] = novf;
+        n_ovf[key]++;
+        store[e] = base + novf;
+        ++novf;
+      }
+    }
+  }
+  fix.clear();
+  for (int32_t key = 0; key < nkeys; ++key) {
+    if (n_ovf[key] == 0) continue;
+    fix.push_back(ffb_phys(key));
+    fix.push_back(base + first_ovf[key]);
+    fix.push_back(n_ovf[key]);
+    fix.push_back(0);
+  }
+}
+
+inline int32_t align16(size_t x) { return static_cast<int32_t>((x + 15) & ~size_t{15}); }
+
+}  // namespace
+
+extern "C" framefb_status framefb_plan_build(const framefb_frame* fin, const framefb_frame* fout,
+                                             const int32_t* row, const int32_t* col, int64_t nnz,
+                                             framefb_plan** out) {
+  if (!out) return FRAMEFB_EINVAL;
+  *out = nullptr;
+  if (!fin || !fout || nnz < 0 || (nnz > 0 && (!row || !col))) return FRAMEFB_EINVAL;
+  if (!fin->dft_groups || !fout->dft_groups || fin->k != 16 || fout->k != 16) return FRAMEFB_EUNSUPPORTED;
+  const int32_t n = fin->d, m = fout->d;
+  if (n % FFB_GROUP || m % FFB_GROUP || fin->ncols != n || fout->ncols != m) return FRAMEFB_EUNSUPPORTED;
+  if (n > 32768 || m > 32768) return FRAMEFB_EUNSUPPORTED;  // 16-bit shared-memory offsets
+  if (nnz > static_cast<int64_t>(m) * n || nnz > (1 << 24)) return FRAMEFB_EINVAL;
+  const int32_t nz = static_cast<int32_t>(nnz);
+  for (int32_t q = 0; q < nz; ++q) {
+    if (row[q] < 0 || row[q] >= m || col[q] < 0 || col[q] >= n) return FRAMEFB_EINVAL;
+    if (q > 0) {
+      const int64_t prev = static_cast<int64_t>(row[q - 1]) * n + col[q - 1];
+      const int64_t cur = static_cast<int64_t>(row[q]) * n + col[q];
+      if (cur <= prev) return FRAMEFB_EINVAL;  // not sorted row-major or duplicated
+    }
+  }
+  try {
+    const int32_t P = FRAMEFB_THREADS;
+    const int32_t Gn = n / FFB_GROUP, Gm = m / FFB_GROUP;
+    std::vector<Entry> byrow(nz), bycol(nz);
+    for (int32_t q = 0; q < nz; ++q) {
+      const int32_t a = group_major(row[q], fout->rho), b = group_major(col[q], fin->rho);
+      byrow[q] = Entry{a, b, q};
+      bycol[q] = Entry{b, a, q};
+    }
+    auto lt = [](const Entry& x, const Entry& y) { return x.key0 != y.key0 ? x.key0 < y.key0 : x.key1 < y.key1; };
+    std::sort(byrow.begin(), byrow.end(), lt);
+    std::sort(bycol.begin(), bycol.end(), lt);
+    const int32_t EZ = (nz + P - 1) / P, EG = EZ;
+
+    std::vector<int32_t> storeZ, fixZ, storeG, fixG;
+    int32_t novfZ = 0, novfG = 0;
+    cut_chunks(byrow, P, EZ, m, m, storeZ, fixZ, novfZ);
+    cut_chunks(bycol, P, EG, n, n, storeG, fixG, novfG);
+
+    FfbPlanHeader h;
+    std::memset(&h, 0, sizeof(h));
+    h.magic = FFB_PLAN_MAGIC;
+    h.version = FFB_PLAN_VERSION;
+    h.n = n;
+    h.m = m;
+    h.Gn = Gn;
+    h.Gm = Gm;
+    h.nnz = nz;
+    h.P = P;
+    h.EZ = EZ;
+    h.EG = EG;
+    h.ovfZ = (novfZ + 3) & ~3;
+    h.ovfG = (novfG + 3) & ~3;
+    h.nfixZ = static_cast<int32_t>(fixZ.size() / 4);
+    h.nfixG = static_cast<int32_t>(fixG.size() / 4);
+
+    size_t off = align16(sizeof(FfbPlanHeader));
+    auto take = [&](size_t bytes) { const int32_t o = static_cast<int32_t>(off); off = align16(off + bytes); return o; };
+    const size_t ezp = static_cast<size_t>(EZ) * P, egp = static_cast<size_t>(EG) * P;
+    h.off_zb = take(ezp * 4);
+    h.off_zq = take(ezp * 4);
+    h.off_ga = take(egp * 4);
+    h.off_gb = take(egp * 4);
+    h.off_gq = take(egp * 4);
+    h.off_fixZ = take(fixZ.size() * 4);
+    h.off_fixG = take(fixG.size() * 4);
+    h.off_zmask = take(static_cast<size_t>(Gm) * 4);
+    h.off_gmask = take(static_cast<size_t>(Gn) * 4);
+    const size_t nblk = static_cast<size_t>(Gm) * Gn;
+    h.off_blkptr = take((nblk + 1) * 4);
+    h.off_blkent = take(static_cast<size_t>(nz) * 8);
+    if (off > static_cast<size_t>(INT32_MAX)) return FRAMEFB_EUNSUPPORTED;
+    h.total_bytes = static_cast<int32_t>(off);
+
+    framefb_plan* plan = new framefb_plan;
+    plan->image.assign(off, 0);
+    uint8_t* base = plan->image.data();
+    auto arr = [&](int32_t o) { return reinterpret_cast<int32_t*>(base + o); };
+    std::memcpy(base, &h, sizeof(h));
+
+    // Per-thread chunk tables, entry-major ([e][p]) so that a warp reading
+    // entry e of its 32 threads touches 128 contiguous bytes.
+    int32_t* zb = arr(h.off_zb);
+    int32_t* zq = arr(h.off_zq);
+    int32_t* ga = arr(h.off_ga);
+    int32_t* gb = arr(h.off_gb);
+    int32_t* gq = arr(h.off_gq);
+    for (int32_t p = 0; p < P; ++p) {
+      for (int32_t e = 0; e < EZ; ++e) {
+        const int32_t idx = p * EZ + e;
+        const size_t slot = static_cast<size_t>(e) * P + p;
+        if (idx < nz) {
+          zb[slot] = ffb_phys(byrow[idx].key1) | (storeZ[idx] << 16);
+          zq[slot] = byrow[idx].q;
+        } else {
+          zb[slot] = (FFB_NO_STORE << 16);
+          zq[slot] = -1;
+        }
+      }
+      for (int32_t e = 0; e < EG; ++e) {
+        const int32_t idx = p * EG + e;
+        const size_t slot = static_cast<size_t>(e) * P + p;
+        if (idx < nz) {
+          ga[slot] = ffb_phys(bycol[idx].key1) | (storeG[idx] << 16);
+          gb[slot] = ffb_phys(bycol[idx].key0);
+          gq[slot] = bycol[idx].q;
+        } else {
+          ga[slot] = (FFB_NO_STORE << 16);
+          gb[slot] = 0;
+          gq[slot] = -1;
+        }
+      }
+    }
+    if (!fixZ.empty()) std::memcpy(arr(h.off_fixZ), fixZ.data(), fixZ.size() * 4);
+    if (!fixG.empty()) std::memcpy(arr(h.off_fixG), fixG.data(), fixG.size() * 4);
+    uint32_t* zmask = reinterpret_cast<uint32_t*>(arr(h.off_zmask));
+    uint32_t* gmask = reinterpret_cast<uint32_t*>(arr(h.off_gmask));
+    for (int32_t q = 0; q < nz; ++q) {
+      zmask[byrow[q].key0 >> 5] |= 1u << (byrow[q].key0 & 31);
+      gmask[bycol[q].key0 >> 5] |= 1u << (bycol[q].key0 & 31);
+    }
+    // Merge: entries grouped by 32 x 32 block (out group g, in group h).
+    int32_t* blkptr = arr(h.off_blkptr);
+    int32_t* blkent = arr(h.off_blkent);
+    std::vector<int32_t> cnt(nblk + 1, 0);
+    for (int32_t q = 0; q < nz; ++q) cnt[static_cast<size_t>(byrow[q].key0 >> 5) * Gn + (byrow[q].key1 >> 5) + 1]++;
+    for (size_t b = 0; b < nblk; ++b) cnt[b + 1] += cnt[b];
+    std::memcpy(blkptr, cnt.data(), (nblk + 1) * 4);
+    for (int32_t q = 0; q < nz; ++q) {  // byrow is sorted by (a, b): entries stay ordered inside a block
+      const size_t b = static_cast<size_t>(byrow[q].key0 >> 5) * Gn + (byrow[q].key1 >> 5);
+      const int32_t dst = cnt[b]++;
+      blkent[2 * dst] = (byrow[q].key0 & 31) | ((byrow[q].key1 & 31) << 8);
+      blkent[2 * dst + 1] = byrow[q].q;
+    }
+    *out = plan;
+  } catch (const std::bad_alloc&) {
+    return FRAMEFB_ENOMEM;
+  }
+  return FRAMEFB_OK;
+}
+
+extern "C" size_t framefb_plan_bytes(const framefb_plan* plan) { return plan ? plan->image.size() : 0; }
+extern "C" const void* framefb_plan_data(const framefb_plan* plan) { return plan ? plan->image.data() : nullptr; }
+extern "C" void framefb_plan_free(framefb_plan* plan) { delete plan; }

@@ -1,0 +1,83 @@
+// Device image of a framefb plan: a header followed by int32 tables, all
+// offsets in bytes from the start of the image, every table 16-byte aligned.
+// Shared by the host builder (framefb_host.cpp) and the kernels (framefb_cuda.cu).
+//
+// Index spaces.  A frame column in the paper's order c = i*rho + 2r + s
+// (subspace i, Spectral Tetris row r, realified part s) is re-indexed
+// group-major as x = 32 r + 2 i + s, so that group r (coordinates
+// [32 r, 32 r + 32) of a k = 16, k*rho = d frame) owns the 32 contiguous
+// columns [32 r, 32 r + 32): its coefficient vector is the 16 complex values
+// (Re, Im interleaved) of the DFT_16 of that coordinate block.
+//
+// Inside shared memory a token row of frame coefficients is stored with its
+// 16-byte chunks XOR-swizzled inside each 128-byte group, so that a warp
+// writing or reading 32 consecutive groups hits 32 distinct banks:
+//     phys(x) = 32 g + 4 ((x/4 mod 8) xor (g mod 8)) + x mod 4,   g = x / 32.
+#pragma once
+#include <stdint.h>
+
+#ifndef __CUDACC__
+#ifndef __host__
+#define __host__
+#endif
+#ifndef __device__
+#define __device__
+#endif
+#endif
+
+#define FFB_PLAN_MAGIC 0x50424646  /* "FFBP" */
+#define FFB_PLAN_VERSION 1
+#define FFB_GROUP 32               /* real coordinates (and frame columns) per group */
+#define FFB_NO_STORE 0xFFFFu
+
+struct FfbPlanHeader {
+  int32_t magic, version;
+  int32_t n, m;            // in / out features (= K_n, K_m: k*rho = d)
+  int32_t Gn, Gm;          // groups of 32 on the input / output side
+  int32_t nnz;
+  int32_t P;               // threads the chunks were cut for
+  int32_t EZ, EG;          // chunk length (entries per thread) by row / by column
+  int32_t ovfZ, ovfG;      // overflow slots after the m (resp. n) row slots, multiple of 4
+  int32_t nfixZ, nfixG;    // fix-up items (rows / columns split between chunks)
+  int32_t off_zb, off_zq;  // [EZ][P]: packed (phys b | store << 16), c index (-1 = padding)
+  int32_t off_ga, off_gb, off_gq;  // [EG][P]: packed (phys a | store << 16), phys b, c index
+  int32_t off_fixZ, off_fixG;      // int4 {dst phys, first overflow slot, count, 0}
+  int32_t off_zmask, off_gmask;    // uint32 per group: bit w = row (col) 32g+w is in the support
+  int32_t off_blkptr;              // merge: [Gm*Gn + 1] entry ranges of each 32x32 block (g, h)
+  int32_t off_blkent;              // merge: int2 {a_local | b_local << 8, c index}
+  int32_t total_bytes;
+  int32_t reserved[6];
+};
+
+static inline __host__ __device__ int32_t ffb_phys(int32_t x) {
+  const int32_t g = x >> 5;
+  return (g << 5) | ((((x >> 2) & 7) ^ (g & 7)) << 2) | (x & 3);
+}
+
+// Shared-memory layout of one tile of T tokens (floats).  MODE bits:
+// 1 = forward (Y), 2 = backward dX, 4 = coefficient gradient.  V = X Phi_in
+// rows (n), U = dY Phi_out rows (m), RZ = coefficient-SpMM row sums for Y
+// (m + ovfZ), RG = the same for dX (n + ovfG); DC = per-thread dC
+// accumulators when the chunks do not fit in registers.
+struct FfbTileLayout {
+  int32_t sV, sU, sRZ, sRG;      // token-row strides
+  int32_t oV, oU, oRZ, oRG, oDC; // region offsets
+  int32_t total;                 // floats
+};
+
+static inline __host__ __device__ FfbTileLayout ffb_tile_layout(const FfbPlanHeader& h, int mode, int T,
+                                                                bool dc_in_smem) {
+  FfbTileLayout L;
+  const bool fwd = mode & 1, bdx = mode & 2, gc = mode & 4;
+  L.sV = h.n;
+  L.sU = h.m;
+  L.sRZ = h.m + h.ovfZ;
+  L.sRG = h.n + h.ovfG;
+  L.oV = 0;
+  L.oU = L.oV + ((fwd || gc) ? T * L.sV : 0);
+  L.oRZ = L.oU + ((bdx || gc) ? T * L.sU : 0);
+  L.oRG = L.oRZ + (fwd ? T * L.sRZ : 0);
+  L.oDC = L.oRG + (bdx ? T * L.sRG : 0);
+  L.total = L.oDC + ((gc && dc_in_smem) ? h.EG * h.P : 0);
+  return L;
+}

@@ -1,0 +1,240 @@
+"""GPU parity of the CUDA path (through the C ABI) against the fp64 oracle.
+
+Tolerances (stated for the adapter path): fp32 activations -- max |g - r| /
+max |r| <= 1e-5; bf16 activations with fp32 accumulation -- per element
+|g - r| <= 2e-2 max(|r|, rms(r)) and ||g - r||_F / ||r||_F <= 5e-3.
+Deltas are checked with Y_in = dX_in = 0; accumulation is checked in fp32.
+"""
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+
+from paper_2608_26430_gb300 import framefb as ffb
+from paper_2608_26430_gb300 import workloads as wl
+from paper_2608_26430_gb300.batch import AdapterBatch
+from tests.oracle_side import Expect, assert_bf16, assert_f32, host64
+
+pytestmark = pytest.mark.gpu
+
+DEV = "cuda:0"
+ALL = ffb.OP_FORWARD | ffb.OP_BACKWARD_DX | ffb.OP_GRAD_COEFF
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2608_26430_gb300.build import build
+    build()
+    ffb.lib()
+
+
+def check_batch(batch, ops, js=None, unit=None, rows=None):
+    w = batch.w
+    close = assert_f32 if w.dtype == "f32" else assert_bf16
+    torch.cuda.synchronize()
+    for j in (range(len(batch.bufs)) if js is None else js):
+        b = batch.bufs[j]
+        e = Expect(batch, j)
+        X, dY = host64(b.X), host64(b.dY)
+        sel = slice(None) if rows is None else rows
+        if ops & ffb.OP_FORWARD:
+            r = e.y(X[sel], np.zeros((X[sel].shape[0], b.spec.m)))
+            close(host64(b.Y)[sel], r, what=f"Y[{j}]")
+        if ops & ffb.OP_BACKWARD_DX:
+            r = e.dx(dY[sel], np.zeros((dY[sel].shape[0], b.spec.n)))
+            close(host64(b.dX)[sel], r, what=f"dX[{j}]")
+        if ops & ffb.OP_GRAD_COEFF:
+            r = e.dc(X, dY)
+            close(host64(b.dC), r, what=f"dC[{j}]")
+
+
+def run(batch, ops):
+    ws = batch.workspace(ops)
+    batch.run(ops, ws)
+    torch.cuda.synchronize()
+
+
+# ---------------------------------------------------------------------------
+# the five workloads at oracle-friendly sizes (several tiles and a ragged tail)
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("ops", [ffb.OP_FORWARD, ffb.OP_BACKWARD_DX, ffb.OP_GRAD_COEFF,
+                                 ffb.OP_BACKWARD_DX | ffb.OP_GRAD_COEFF, ALL])
+@pytest.mark.parametrize("unit", [True, False])
+def test_single_256_fp32(ops, unit):
+    b = AdapterBatch(wl.WORKLOADS["single_256_fp32"], DEV, unit_scale=unit, ops=ops)
+    run(b, ops)
+    check_batch(b, ops)
+
+
+@pytest.mark.parametrize("N", [37, 1, 4])
+def test_roberta_base_all_matrices(N):
+    b = AdapterBatch(wl.WORKLOADS["roberta_base_qv"], DEV, N=N, ops=ALL)
+    run(b, ALL)
+    check_batch(b, ALL)
+
+
+def test_vit_b16_mixed_shapes():
+    w = wl.WORKLOADS["vit_b16_merge"]
+    b = AdapterBatch(w, DEV, N=23, ops=ALL)
+    run(b, ALL)
+    check_batch(b, ALL, js=[0, 3, 4, 5, 10, 11, 70, 71])
+
+
+def test_llama2_shape_small_n():
+    w = wl.WORKLOADS["llama2_7b_qkvo"]
+    b = AdapterBatch(w, DEV, N=13, indices=[0, 5, 127], ops=ALL)
+    run(b, ALL)
+    check_batch(b, ALL)
+
+
+def test_llama3_zipf_nonsquare():
+    # nnz = 8192 exceeds the register-resident chunk: exercises the streamed-plan path
+    w = wl.WORKLOADS["llama3_8b_all"]
+    b = AdapterBatch(w, DEV, N=9, indices=list(range(7)), alias_inputs=True, ops=ALL)
+    run(b, ALL)
+    check_batch(b, ALL)
+
+
+# ---------------------------------------------------------------------------
+# semantics and edge cases
+# ---------------------------------------------------------------------------
+def test_entry_points_agree_with_fused():
+    w = wl.WORKLOADS["roberta_base_qv"]
+    fused = AdapterBatch(w, DEV, N=29, indices=[0, 1, 2], ops=ALL)
+    run(fused, ALL)
+    sep = AdapterBatch(w, DEV, N=29, indices=[0, 1, 2], ops=ALL)
+    ws = sep.workspace(ALL)
+    ffb.framefb_forward(sep.mats, sep.dtype_code, ws)
+    ffb.framefb_backward_dx(sep.mats, sep.dtype_code, ws)
+    ffb.framefb_grad_coeff(sep.mats, sep.dtype_code, ws)
+    torch.cuda.synchronize()
+    for a, c in zip(fused.bufs, sep.bufs):
+        assert torch.equal(a.Y, c.Y) and torch.equal(a.dX, c.dX)
+        assert torch.equal(a.dC, c.dC)        # deterministic reduction order
+
+
+def test_accumulates_into_y_and_dx_fp32():
+    w = wl.WORKLOADS["single_256_fp32"]
+    b = AdapterBatch(w, DEV, N=11, y_init="random", ops=ALL)
+    Y0, dX0 = host64(b.bufs[0].Y), host64(b.bufs[0].dX)
+    run(b, ALL)
+    e = Expect(b, 0)
+    assert_f32(host64(b.bufs[0].Y), e.y(host64(b.bufs[0].X), Y0), what="Y")
+    assert_f32(host64(b.bufs[0].dX), e.dx(host64(b.bufs[0].dY), dX0), what="dX")
+    run(b, ffb.OP_FORWARD)             # a second call adds the delta again
+    assert_f32(host64(b.bufs[0].Y), Y0 + 2 * (e.y(host64(b.bufs[0].X), Y0) - Y0), what="Y twice")
+
+
+def test_deterministic_dc():
+    w = wl.WORKLOADS["roberta_base_qv"]
+    b = AdapterBatch(w, DEV, N=300, indices=[0, 1], ops=ffb.OP_GRAD_COEFF)
+    run(b, ffb.OP_GRAD_COEFF)
+    first = [x.dC.clone() for x in b.bufs]
+    run(b, ffb.OP_GRAD_COEFF)
+    for f, x in zip(first, b.bufs):
+        assert torch.equal(f, x.dC)
+
+
+def test_zero_tokens_gives_zero_dc_and_no_writes():
+    w = wl.WORKLOADS["roberta_base_qv"]
+    b = AdapterBatch(w, DEV, N=0, indices=[0], ops=ALL)
+    run(b, ALL)
+    assert torch.count_nonzero(b.bufs[0].dC) == 0
+
+
+def test_empty_support_is_a_no_op():
+    fin = ffb.Frame(256, 16, 16)
+    dfin = fin.to_device(DEV)
+    plan = ffb.Plan(fin, fin, np.zeros(0, np.int32), np.zeros(0, np.int32))
+    pd = plan.to_device(DEV)
+    X = torch.randn(10, 256, device=DEV, dtype=torch.bfloat16)
+    Y = torch.randn(10, 256, device=DEV, dtype=torch.bfloat16)
+    Y0 = Y.clone()
+    m = ffb.make_mat(dfin, dfin, plan, pd, None, 1.0, 10, X=X, Y=Y)
+    ffb.framefb_forward([m], ffb.FRAMEFB_BF16)
+    torch.cuda.synchronize()
+    assert torch.equal(Y, Y0)
+
+
+def test_strided_rows_and_untouched_padding():
+    w = wl.WORKLOADS["roberta_base_qv"]
+    N, n, m = 19, 768, 768
+    src = AdapterBatch(w, DEV, N=N, indices=[0], ops=ALL)
+    bb = src.bufs[0]
+    pad = 64
+    Xp = torch.zeros(N, n + pad, device=DEV, dtype=torch.bfloat16)
+    Xp[:, :n] = bb.X
+    dYp = torch.zeros(N + 2, m + pad, device=DEV, dtype=torch.bfloat16)
+    dYp[:N, :m] = bb.dY
+    Yp = torch.full((N + 2, m + pad), 3.0, device=DEV, dtype=torch.bfloat16)
+    dXp = torch.full((N, n + pad), 5.0, device=DEV, dtype=torch.bfloat16)
+    dC = torch.zeros(w.nnz, device=DEV)
+    mat = ffb.make_mat(src.dev_frames[n], src.dev_frames[m], src.plans[(m, n)], src.plan_dev[(m, n)], bb.c_val,
+                       bb.scale, N, X=Xp, dX=dXp, dY=dYp, Y=Yp, dC=dC, ldx=n + pad, ldy=m + pad)
+    ws = ffb.workspace([mat], ALL, DEV)
+    ffb.framefb_run([mat], ALL, ffb.FRAMEFB_BF16, ws)
+    torch.cuda.synchronize()
+    assert torch.all(Yp[:, m:] == 3.0) and torch.all(Yp[N:, :] == 3.0) and torch.all(dXp[:, n:] == 5.0)
+    e = Expect(src, 0)
+    assert_bf16(host64(Yp[:N, :m]) - 3.0, e.y(host64(bb.X), np.zeros((N, m))), what="Y strided")
+    assert_bf16(host64(dXp[:, :n]) - 5.0, e.dx(host64(bb.dY), np.zeros((N, n))), what="dX strided")
+    assert_bf16(host64(dC), e.dc(host64(bb.X), host64(bb.dY)), what="dC strided")
+
+
+def test_invalid_arguments_return_status():
+    w = wl.WORKLOADS["roberta_base_qv"]
+    b = AdapterBatch(w, DEV, N=8, indices=[0], ops=ALL)
+    good = b.mats[0]
+    bad = ffb.framefb_mat.from_buffer_copy(good)
+    bad.X = good.X + 2                         # misaligned
+    with pytest.raises(ffb.FramefbError) as e:
+        ffb.framefb_run([bad], ALL, ffb.FRAMEFB_BF16, b.workspace(ALL))
+    assert e.value.status == ffb.FRAMEFB_EINVAL
+    with pytest.raises(ffb.FramefbError) as e:         # no workspace for dC
+        ffb.framefb_run([good], ALL, ffb.FRAMEFB_BF16, None)
+    assert e.value.status == ffb.FRAMEFB_EWORKSPACE
+    bad = ffb.framefb_mat.from_buffer_copy(good)
+    bad.n = 1024                               # frame / plan mismatch
+    with pytest.raises(ffb.FramefbError) as e:
+        ffb.framefb_run([bad], ffb.OP_FORWARD, ffb.FRAMEFB_BF16)
+    assert e.value.status == ffb.FRAMEFB_EINVAL
+    with pytest.raises(ffb.FramefbError) as e:
+        ffb.framefb_run([good], 3 | 8, ffb.FRAMEFB_BF16)
+    assert e.value.status == ffb.FRAMEFB_EINVAL
+
+
+# ---------------------------------------------------------------------------
+# merge
+# ---------------------------------------------------------------------------
+def _merge_case(wname, T=None):
+    w = wl.WORKLOADS[wname]
+    m, n = w.merge_shape
+    T = w.merge_tenants if T is None else T
+    fin, fout = ffb.Frame(n, w.k, n // w.k), ffb.Frame(m, w.k, m // w.k)
+    row, col, _, _ = ffb.framefb_support_build(m, n, w.nnz, w.support_seed, w.support_mode, w.zipf_s, w.k)
+    plan = ffb.Plan(fin, fout, row, col)
+    W0 = wl.w0_input(w, DEV)
+    cv = wl.merge_c_values(w, DEV)[:T].contiguous()
+    Wout = torch.full((T, m, n), float("nan"), device=DEV, dtype=W0.dtype)
+    s = 200.0 / (m * n) ** 0.5
+    ffb.framefb_merge(W0, fin.to_device(DEV), fout.to_device(DEV), plan, plan.to_device(DEV), cv, T, s, Wout)
+    torch.cuda.synchronize()
+    from oracle import adapter
+    from tests.oracle_side import frame, oracle_support
+    orow, ocol, _, _ = oracle_support(m, n, w.nnz, w.support_seed, w.support_mode, w.zipf_s, w.k)
+    Cs = [adapter.dense_C(m, n, orow, ocol, host64(cv[t])) for t in range(T)]
+    ref = adapter.merge(host64(W0), Cs, frame(n, w.k), frame(m, w.k), s)
+    return host64(W0), host64(Wout), ref
+
+
+def test_merge_fp32_delta_precision():
+    W0, got, ref = _merge_case("single_256_fp32")
+    for t in range(got.shape[0]):
+        assert_f32(got[t] - W0, ref[t] - W0, what=f"dW[{t}]")
+
+
+def test_merge_vit_64_tenants_bf16():
+    W0, got, ref = _merge_case("vit_b16_merge")
+    assert_bf16(got, ref, what="W_t")

@@ -1,0 +1,237 @@
+"""CPU tests of libframefb's host side: exports, frame construction, support
+sampling and plans, checked bit for bit (indices) against the oracle."""
+import os
+import re
+
+import numpy as np
+import pytest
+
+from oracle import adapter, frames, support
+from paper_2608_26430_gb300 import framefb as ffb
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built_library():
+    from paper_2608_26430_gb300.build import build
+    build()
+
+
+def header_functions():
+    txt = open(os.path.join(ROOT, "include", "framefb.h")).read()
+    txt = re.sub(r"/\*.*?\*/", "", txt, flags=re.S)
+    return sorted(set(re.findall(r"\b(framefb_[a-z_0-9]+)\s*\(", txt)))
+
+
+def test_library_exports_every_declared_function():
+    names = header_functions()
+    assert len(names) >= 17
+    got = ffb.exported_symbols(names)
+    assert all(got.values()), [n for n, ok in got.items() if not ok]
+    assert ffb.lib().framefb_abi_version() == 1
+
+
+@pytest.mark.parametrize("d,k,rho,parseval", [(256, 16, 16, True), (768, 16, 48, True), (22, 6, 6, False),
+                                              (22, 6, 6, True), (40, 7, 8, True), (64, 8, 8, False),
+                                              (1024, 16, 64, True), (46, 10, 10, True)])
+def test_frame_build_matches_oracle(d, k, rho, parseval):
+    fr = ffb.Frame(d, k, rho, parseval)
+    P = frames.real_frame(d, k, rho, parseval)
+    pat = frames.structural_pattern(d, k, rho)
+    colptr, rowidx, val = frames.csc_from_dense(P, pat)
+    rowptr, colidx, rval = frames.csr_from_dense(P, pat)
+    g_colptr, g_rowidx, g_val = fr.csc()
+    g_rowptr, g_colidx, g_rval = fr.csr()
+    assert np.array_equal(g_colptr, colptr) and np.array_equal(g_rowidx, rowidx)
+    assert np.array_equal(g_rowptr, rowptr) and np.array_equal(g_colidx, colidx)
+    np.testing.assert_allclose(g_val, val, rtol=0, atol=2e-15)
+    np.testing.assert_allclose(g_rval, rval, rtol=0, atol=2e-15)
+    row0, nrows = frames.group_table(d, k, rho)
+    g0, gn = fr.groups()
+    assert np.array_equal(g0, row0) and np.array_equal(gn, nrows)
+    assert fr.nnz == pat.sum() and fr.ncols == k * rho
+    assert fr.A == pytest.approx(frames.frame_bound(d, k, rho), rel=1e-15)
+    assert fr.dft_groups == int(k * rho == d)
+
+
+@pytest.mark.parametrize("d", [4096, 14336, 3072])
+def test_frame_build_large_dims_indices(d):
+    fr = ffb.Frame(d, 16, d // 16)
+    colptr, rowidx, val = fr.csc()
+    assert np.array_equal(colptr, 32 * np.arange(d + 1))
+    # column c = i*rho + 2r + s covers the coordinates of group r
+    rho = d // 16
+    c = np.arange(d)
+    r = (c % rho) // 2
+    np.testing.assert_array_equal(rowidx.reshape(d, 32), 32 * r[:, None] + np.arange(32)[None, :])
+    np.testing.assert_allclose(np.abs(val).max(), 0.25, rtol=1e-15)
+
+
+@pytest.mark.parametrize("d,k,rho,status", [(22, 5, 6, ffb.FRAMEFB_EUNSUPPORTED), (14, 4, 8, ffb.FRAMEFB_EUNSUPPORTED),
+                                            (21, 4, 6, ffb.FRAMEFB_EINVAL), (24, 4, 3, ffb.FRAMEFB_EINVAL),
+                                            (0, 4, 2, ffb.FRAMEFB_EINVAL), (24, 0, 2, ffb.FRAMEFB_EINVAL)])
+def test_frame_build_rejects(d, k, rho, status):
+    with pytest.raises(ffb.FramefbError) as e:
+        ffb.Frame(d, k, rho)
+    assert e.value.status == status
+
+
+SUPPORT_CASES = [(256, 256, 128, 1, 0, 1), (768, 768, 1000, 1, 0, 1), (4096, 4096, 4096, 1, 0, 1),
+                 (4096, 14336, 8192, 1, 1, 1), (1024, 4096, 8192, 1, 1, 1), (14336, 4096, 8192, 1, 1, 1),
+                 (768, 768, 2000, 1, 0, 1), (96, 96, 500, 3, 2, 16), (64, 32, 2048, 9, 0, 1), (10, 10, 0, 1, 0, 1)]
+
+
+@pytest.mark.parametrize("rows,cols,nnz,seed,mode,k", SUPPORT_CASES)
+def test_support_build_bit_exact(rows, cols, nnz, seed, mode, k):
+    row, col, rowptr, perm = ffb.framefb_support_build(rows, cols, nnz, seed, mode, 1.1, k)
+    orow, ocol, orowptr, operm = support.sample_support(rows, cols, nnz, seed, mode, 1.1, k)
+    assert np.array_equal(row, orow) and np.array_equal(col, ocol)
+    assert np.array_equal(rowptr, orowptr) and np.array_equal(perm, operm)
+
+
+def test_support_build_rejects():
+    for args in [(10, 10, 101, 1, 0, 1.1, 1), (10, 10, 5, 1, 7, 1.1, 1), (10, 12, 5, 1, 2, 1.1, 3),
+                 (10, 10, 5, 1, 1, -1.0, 1), (0, 10, 0, 1, 0, 1.1, 1)]:
+        with pytest.raises(ffb.FramefbError) as e:
+            ffb.framefb_support_build(*args)
+        assert e.value.status == ffb.FRAMEFB_EINVAL
+
+
+# ---------------------------------------------------------------------------
+# plans: decode the image and replay the kernels' sparse steps on the CPU
+# ---------------------------------------------------------------------------
+HDR = ["magic", "version", "n", "m", "Gn", "Gm", "nnz", "P", "EZ", "EG", "ovfZ", "ovfG", "nfixZ", "nfixG",
+       "off_zb", "off_zq", "off_ga", "off_gb", "off_gq", "off_fixZ", "off_fixG", "off_zmask", "off_gmask",
+       "off_blkptr", "off_blkent", "total_bytes"]
+
+
+def decode(img):
+    h = dict(zip(HDR, np.frombuffer(img[:4 * len(HDR)].tobytes(), dtype=np.int32).tolist()))
+    def arr(off, count, dt=np.int32):
+        return np.frombuffer(img[off:off + count * np.dtype(dt).itemsize].tobytes(), dtype=dt)
+    P = h["P"]
+    t = dict(h=h)
+    t["zb"] = arr(h["off_zb"], h["EZ"] * P, np.uint32).reshape(h["EZ"], P)
+    t["zq"] = arr(h["off_zq"], h["EZ"] * P).reshape(h["EZ"], P)
+    t["ga"] = arr(h["off_ga"], h["EG"] * P, np.uint32).reshape(h["EG"], P)
+    t["gb"] = arr(h["off_gb"], h["EG"] * P, np.uint32).reshape(h["EG"], P)
+    t["gq"] = arr(h["off_gq"], h["EG"] * P).reshape(h["EG"], P)
+    t["fixZ"] = arr(h["off_fixZ"], 4 * h["nfixZ"]).reshape(-1, 4)
+    t["fixG"] = arr(h["off_fixG"], 4 * h["nfixG"]).reshape(-1, 4)
+    t["zmask"] = arr(h["off_zmask"], h["Gm"], np.uint32)
+    t["gmask"] = arr(h["off_gmask"], h["Gn"], np.uint32)
+    nblk = h["Gm"] * h["Gn"]
+    t["blkptr"] = arr(h["off_blkptr"], nblk + 1)
+    t["blkent"] = arr(h["off_blkent"], 2 * h["nnz"]).reshape(-1, 2)
+    return t
+
+
+def group_major(c, rho):
+    """paper column c = i*rho + 2r + s  ->  x = 32 r + 2 i + s (k = 16)."""
+    c = np.asarray(c)
+    i, rr = c // rho, c % rho
+    return 32 * (rr // 2) + 2 * i + (rr & 1)
+
+
+def phys(x):
+    x = np.asarray(x)
+    g = x >> 5
+    return (g << 5) | ((((x >> 2) & 7) ^ (g & 7)) << 2) | (x & 3)
+
+
+PLAN_CASES = [(256, 256, 128, 0), (768, 768, 1000, 0), (768, 3072, 2000, 0), (4096, 1024, 8192, 1),
+              (1024, 256, 6000, 1), (256, 768, 4000, 0), (512, 512, 7, 0), (256, 256, 256 * 17, 0)]
+
+
+@pytest.mark.parametrize("n,m,nnz,mode", PLAN_CASES)
+def test_plan_replays_coefficient_products(n, m, nnz, mode):
+    fin, fout = ffb.Frame(n, 16, n // 16), ffb.Frame(m, 16, m // 16)
+    row, col, _, _ = support.sample_support(m, n, nnz, 1, mode, 1.1)
+    t = decode(ffb.Plan(fin, fout, row, col).image())
+    h = t["h"]
+    assert h["magic"] == 0x50424646 and h["P"] == ffb.THREADS and h["nnz"] == nnz
+    # every entry appears once in each chunk table
+    assert sorted(t["zq"][t["zq"] >= 0].tolist()) == list(range(nnz))
+    assert sorted(t["gq"][t["gq"] >= 0].tolist()) == list(range(nnz))
+    a_int, b_int = group_major(row, m // 16), group_major(col, n // 16)
+    assert len(set(a_int.tolist())) == len(set(row.tolist()))
+    # masks
+    zm = np.zeros(h["Gm"], np.uint32)
+    gm = np.zeros(h["Gn"], np.uint32)
+    for a in a_int:
+        zm[a >> 5] |= np.uint32(1) << np.uint32(a & 31)
+    for b in b_int:
+        gm[b >> 5] |= np.uint32(1) << np.uint32(b & 31)
+    assert np.array_equal(zm, t["zmask"]) and np.array_equal(gm, t["gmask"])
+
+    # replay with random V (input side) and U (output side) rows, 3 tokens
+    rng = np.random.default_rng(0)
+    Tn = 3
+    c = rng.standard_normal(nnz)
+    Vint = rng.standard_normal((Tn, n))
+    Uint = rng.standard_normal((Tn, m))
+    Vs = np.zeros((Tn, n)); Vs[:, phys(np.arange(n))] = Vint
+    Us = np.zeros((Tn, m)); Us[:, phys(np.arange(m))] = Uint
+    RZ = np.zeros((Tn, m + h["ovfZ"]))
+    RG = np.zeros((Tn, n + h["ovfG"]))
+    dC = np.zeros(nnz)
+    for p in range(h["P"]):
+        acc = np.zeros(Tn)
+        for e in range(h["EZ"]):
+            pk, q = int(t["zb"][e, p]), int(t["zq"][e, p])
+            cv = c[q] if q >= 0 else 0.0
+            acc += cv * Vs[:, pk & 0xFFFF]
+            if (pk >> 16) != 0xFFFF:
+                RZ[:, pk >> 16] = acc
+                acc = np.zeros(Tn)
+        acc = np.zeros(Tn)
+        for e in range(h["EG"]):
+            pa, pb, q = int(t["ga"][e, p]), int(t["gb"][e, p]), int(t["gq"][e, p])
+            cv = c[q] if q >= 0 else 0.0
+            uv = Us[:, pa & 0xFFFF]
+            acc += cv * uv
+            if q >= 0:
+                dC[q] += np.dot(uv, Vs[:, pb])
+            if (pa >> 16) != 0xFFFF:
+                RG[:, pa >> 16] = acc
+                acc = np.zeros(Tn)
+    for dst, src, cnt, _ in t["fixZ"]:
+        RZ[:, dst] += RZ[:, src:src + cnt].sum(axis=1)
+    for dst, src, cnt, _ in t["fixG"]:
+        RG[:, dst] += RG[:, src:src + cnt].sum(axis=1)
+    Z = RZ[:, phys(np.arange(m))]
+    G = RG[:, phys(np.arange(n))]
+    Cint = adapter.dense_C(m, n, a_int, b_int, c)
+    np.testing.assert_allclose(Z, Vint @ Cint.T, atol=1e-12)
+    np.testing.assert_allclose(G, Uint @ Cint, atol=1e-12)
+    np.testing.assert_allclose(dC, np.einsum("ta,tb->ab", Uint, Vint)[a_int, b_int], atol=1e-12)
+    # merge blocks list every entry once with its local indices
+    seen = []
+    Gn = h["Gn"]
+    for blk in range(h["Gm"] * Gn):
+        for e in range(t["blkptr"][blk], t["blkptr"][blk + 1]):
+            pk, q = t["blkent"][e]
+            g, hh = divmod(blk, Gn)
+            assert 32 * g + (pk & 31) == a_int[q] and 32 * hh + ((pk >> 8) & 31) == b_int[q]
+            seen.append(int(q))
+    assert sorted(seen) == list(range(nnz))
+
+
+def test_plan_rejects_unsorted_and_unsupported():
+    f256 = ffb.Frame(256, 16, 16)
+    with pytest.raises(ffb.FramefbError) as e:
+        ffb.Plan(f256, f256, np.array([3, 1], np.int32), np.array([0, 0], np.int32))
+    assert e.value.status == ffb.FRAMEFB_EINVAL
+    with pytest.raises(ffb.FramefbError) as e:
+        ffb.Plan(f256, f256, np.array([1, 1], np.int32), np.array([2, 2], np.int32))
+    assert e.value.status == ffb.FRAMEFB_EINVAL
+    with pytest.raises(ffb.FramefbError) as e:
+        ffb.Plan(f256, f256, np.array([256], np.int32), np.array([0], np.int32))
+    assert e.value.status == ffb.FRAMEFB_EINVAL
+    red = ffb.Frame(22, 6, 6)
+    with pytest.raises(ffb.FramefbError) as e:
+        ffb.Plan(red, red, np.array([0], np.int32), np.array([0], np.int32))
+    assert e.value.status == ffb.FRAMEFB_EUNSUPPORTED
+    p = ffb.Plan(f256, f256, np.zeros(0, np.int32), np.zeros(0, np.int32))
+    assert decode(p.image())["h"]["nnz"] == 0
