@@ -36,6 +36,7 @@ def parse():
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu", action="store_true")
     p.add_argument("--cpu-tokens", type=int, default=1024, help="token sample of the CPU oracle baseline")
+    p.add_argument("--mats", type=int, default=None, help="first MATS matrices only (small profiling cases)")
     return p.parse_args()
 
 
@@ -118,6 +119,18 @@ def algorithmic_bytes(batch) -> int:
         r_out, r_in = 32 * int(np.count_nonzero(zmask)), 32 * int(np.count_nonzero(gmask))
         total += 3 * esz * batch.N * (r_in + r_out) + nnz * (4 + 4 + 8)
     return total
+
+
+def measured_traffic():
+    """ncu DRAM bytes per launch of the dominant kernel, if taken on the current kernel source."""
+    import hashlib
+    try:
+        src = os.path.join(ROOT, "paper_2608_26430_gb300", "csrc", "framefb_kernels.cuh")
+        h = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+        with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
+            return json.load(f).get(h, {}).get("bytes_per_launch")
+    except Exception:
+        return None
 
 
 def cpu_oracle_sample(w, tokens: int):
@@ -204,7 +217,7 @@ def main():
     from paper_2608_26430_gb300.batch import AdapterBatch
 
     ops = ffb.OP_FORWARD | ffb.OP_BACKWARD_DX | ffb.OP_GRAD_COEFF
-    batch = AdapterBatch(w, dev, ops=ops)
+    batch = AdapterBatch(w, dev, ops=ops, indices=None if args.mats is None else range(args.mats))
     ws = batch.workspace(ops)
     stream = torch.cuda.current_stream()
     alg = algorithmic_bytes(batch)
@@ -286,11 +299,12 @@ def main():
         out = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
                "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
                "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
-               "config": {"workload": w.name, "matrices": len(w.mats), "tokens": w.N, "nnz": w.nnz,
+               "config": {"workload": w.name, "matrices": len(batch.bufs), "tokens": w.N, "nnz": w.nnz,
                           "shape": f"{w.mats[0].m}x{w.mats[0].n}", "k": w.k, "parallelism": "replicas" if world > 1 else "single",
                           "l2": "inputs larger than L2 (32 GB per step)"},
                "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                            "frac": achieved / peak, "traffic": None, "peak_kind": peak_kind,
+                            "frac": achieved / peak,
+                            "traffic": measured_traffic() if args.mats is None and args.workload is None else None, "peak_kind": peak_kind,
                             "kernel": "tile_kernel<bf16, fwd|dx|dc> + dc_reduce", "kernel_ms": kernel_ms,
                             "algorithmic_bytes": alg, "frac_of_8tbs": achieved / 8000.0},
                "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": 2 * args.steps,

@@ -168,8 +168,12 @@ def test_strided_rows_and_untouched_padding():
     Xp[:, :n] = bb.X
     dYp = torch.zeros(N + 2, m + pad, device=DEV, dtype=torch.bfloat16)
     dYp[:N, :m] = bb.dY
+    # padding holds sentinels; the active region starts at zero so that the
+    # bf16 result is the delta itself
     Yp = torch.full((N + 2, m + pad), 3.0, device=DEV, dtype=torch.bfloat16)
+    Yp[:N, :m] = 0
     dXp = torch.full((N, n + pad), 5.0, device=DEV, dtype=torch.bfloat16)
+    dXp[:, :n] = 0
     dC = torch.zeros(w.nnz, device=DEV)
     mat = ffb.make_mat(src.dev_frames[n], src.dev_frames[m], src.plans[(m, n)], src.plan_dev[(m, n)], bb.c_val,
                        bb.scale, N, X=Xp, dX=dXp, dY=dYp, Y=Yp, dC=dC, ldx=n + pad, ldy=m + pad)
@@ -178,8 +182,8 @@ def test_strided_rows_and_untouched_padding():
     torch.cuda.synchronize()
     assert torch.all(Yp[:, m:] == 3.0) and torch.all(Yp[N:, :] == 3.0) and torch.all(dXp[:, n:] == 5.0)
     e = Expect(src, 0)
-    assert_bf16(host64(Yp[:N, :m]) - 3.0, e.y(host64(bb.X), np.zeros((N, m))), what="Y strided")
-    assert_bf16(host64(dXp[:, :n]) - 5.0, e.dx(host64(bb.dY), np.zeros((N, n))), what="dX strided")
+    assert_bf16(host64(Yp[:N, :m]), e.y(host64(bb.X), np.zeros((N, m))), what="Y strided")
+    assert_bf16(host64(dXp[:, :n]), e.dx(host64(bb.dY), np.zeros((N, n))), what="dX strided")
     assert_bf16(host64(dC), e.dc(host64(bb.X), host64(bb.dY)), what="dC strided")
 
 
@@ -238,3 +242,29 @@ def test_merge_fp32_delta_precision():
 def test_merge_vit_64_tenants_bf16():
     W0, got, ref = _merge_case("vit_b16_merge")
     assert_bf16(got, ref, what="W_t")
+
+
+# ---------------------------------------------------------------------------
+# full size, in the launch configuration bench.py times
+# ---------------------------------------------------------------------------
+def test_llama2_full_size_bench_launch_sampled():
+    """All 128 matrices x 8192 tokens in one fused launch; Y and dX checked on
+    96 sampled token rows (rows are independent) and dC in full, for matrices
+    of the first, a middle and the last layer."""
+    w = wl.WORKLOADS["llama2_7b_qkvo"]
+    b = AdapterBatch(w, DEV, ops=ALL)
+    run(b, ALL)
+    rng = np.random.default_rng(1)
+    rows = np.unique(np.concatenate([[0, 1, w.N - 1], rng.choice(w.N, 93, replace=False)]))
+    for j in (0, 66, 127):
+        buf = b.bufs[j]
+        e = Expect(b, j)
+        X = host64(buf.X)
+        dY = host64(buf.dY)
+        assert_bf16(host64(buf.Y[torch.from_numpy(rows).to(DEV)]), e.y(X[rows], np.zeros((rows.size, 4096))),
+                    what=f"Y[{j}] rows")
+        assert_bf16(host64(buf.dX[torch.from_numpy(rows).to(DEV)]), e.dx(dY[rows], np.zeros((rows.size, 4096))),
+                    what=f"dX[{j}] rows")
+        assert_bf16(host64(buf.dC), e.dc(X, dY), what=f"dC[{j}]")
+    del b
+    torch.cuda.empty_cache()
