@@ -230,6 +230,28 @@ size_t framefb_workspace_size(const framefb_mat* mats, int32_t nmats, int32_t op
 framefb_status framefb_run(const framefb_mat* mats, int32_t nmats, int32_t ops, framefb_dtype dtype,
                            void* ws, size_t ws_bytes, void* stream);
 
+/*
+ * framefb_run without a caller-provided workspace.  The paper has no
+ * counterpart: this entry point is for callers that cannot allocate device
+ * memory where they call the library -- code that runs inside a fixed device
+ * memory budget handed out by a host framework, or a latency-critical path
+ * that must not call cudaMalloc because it can synchronise the device.
+ * The dC partial sums go to a library-owned static device array of
+ * FRAMEFB_STATIC_WS_BYTES (8 MiB) that every GPU which loads the library
+ * holds until the process exits; nothing is allocated per call.  A call whose
+ * workspace need (framefb_workspace_size) exceeds that size returns
+ * FRAMEFB_EWORKSPACE and queues nothing.  The first call on a device looks up
+ * the array's device address with cudaGetSymbolAddress and caches it: make
+ * that first call outside any stream capture.  All calls on one device share
+ * the array: calls whose kernels can overlap on the GPU (e.g. on unordered
+ * streams) race on it and must be ordered by the caller.  Each call writes
+ * every partial sum it reads, so no state carries over between calls.
+ * Arguments and results are those of framefb_run.
+ */
+#define FRAMEFB_STATIC_WS_BYTES (8u << 20)
+framefb_status framefb_run_static_ws(const framefb_mat* mats, int32_t nmats, int32_t ops, framefb_dtype dtype,
+                                     void* stream);
+
 /* S3 -> S4 -> S5: Y += ((X Phi_in) C^T) Phi_out^T * s  (forward of Y = X W'^T). */
 framefb_status framefb_forward(const framefb_mat* mats, int32_t nmats, framefb_dtype dtype,
                                void* ws, size_t ws_bytes, void* stream);

@@ -6,6 +6,7 @@
 #include <algorithm>
 #include <cmath>
 #include <cstring>
+#include <mutex>
 #include <vector>
 
 #include "framefb.h"
@@ -312,4 +313,43 @@ extern "C" framefb_status framefb_merge(const void* W0, framefb_dtype dtype, int
   if (cudaLaunchKernel(fn, dim3(h->Gm, T), dim3(256), kargs, 0, static_cast<cudaStream_t>(stream)) != cudaSuccess)
     return FRAMEFB_ECUDA;
   return FRAMEFB_OK;
+}
+
+// ---------------------------------------------------------------------------
+// Workspace-free variant of framefb_run for callers that cannot allocate
+// device memory: the dC partial sums live in this file-scope device array.
+// Host code must not use `g_static_ws` as an address (it names a host-side
+// stand-in); the device address is looked up once per device below.
+// ---------------------------------------------------------------------------
+static __device__ __align__(256) unsigned char g_static_ws[FRAMEFB_STATIC_WS_BYTES];
+
+namespace {
+constexpr int kMaxDevices = 64;
+std::mutex g_static_ws_mu;
+void* g_static_ws_ptr[kMaxDevices] = {};
+
+// Device address of g_static_ws on the current device (looked up on first use).
+framefb_status static_ws_address(void** out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return FRAMEFB_ECUDA;
+  std::lock_guard<std::mutex> lock(g_static_ws_mu);
+  if (!g_static_ws_ptr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_static_ws) != cudaSuccess || !p) return FRAMEFB_ECUDA;
+    g_static_ws_ptr[dev] = p;
+  }
+  *out = g_static_ws_ptr[dev];
+  return FRAMEFB_OK;
+}
+}  // namespace
+
+extern "C" framefb_status framefb_run_static_ws(const framefb_mat* mats, int32_t nmats, int32_t ops,
+                                                framefb_dtype dtype, void* stream) {
+  if (nmats < 0 || (nmats > 0 && !mats) || !ops_ok(ops)) return FRAMEFB_EINVAL;
+  if (dtype != FRAMEFB_F32 && dtype != FRAMEFB_BF16) return FRAMEFB_EINVAL;
+  void* ws = nullptr;
+  const framefb_status s = static_ws_address(&ws);
+  if (s != FRAMEFB_OK) return s;
+  // framefb_run rejects a need above FRAMEFB_STATIC_WS_BYTES with FRAMEFB_EWORKSPACE
+  return framefb_run(mats, nmats, ops, dtype, ws, FRAMEFB_STATIC_WS_BYTES, stream);
 }

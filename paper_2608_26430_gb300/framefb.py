@@ -26,8 +26,9 @@ EXPORTED = [
     "framefb_status_string", "framefb_abi_version", "framefb_frame_build", "framefb_frame_free",
     "framefb_support_build", "framefb_plan_build", "framefb_plan_bytes", "framefb_plan_data", "framefb_plan_free",
     "framefb_workspace_size", "framefb_run", "framefb_forward", "framefb_backward_dx", "framefb_grad_coeff",
-    "framefb_backward", "framefb_fused_fwd_bwd", "framefb_merge",
+    "framefb_backward", "framefb_fused_fwd_bwd", "framefb_merge", "framefb_run_static_ws",
 ]
+STATIC_WS_BYTES = 8 << 20
 
 
 class FramefbError(RuntimeError):
@@ -104,6 +105,8 @@ def lib() -> ct.CDLL:
             f = getattr(L, name)
             f.restype = i32
             f.argtypes = [ct.POINTER(framefb_mat), i32, i32, vp, sz, vp]
+        L.framefb_run_static_ws.restype = i32
+        L.framefb_run_static_ws.argtypes = [ct.POINTER(framefb_mat), i32, i32, i32, vp]
         L.framefb_merge.restype = i32
         L.framefb_merge.argtypes = [vp, i32, i32, i32, i64, ct.POINTER(framefb_dev_frame),
                                     ct.POINTER(framefb_dev_frame), vp, vp, vp, i32, ct.c_float, vp, vp]
@@ -286,6 +289,12 @@ def framefb_run(mats: Sequence[framefb_mat], ops: int, dtype: int, ws=None, stre
     wsp = _ptr(ws)
     wsb = 0 if ws is None else ws.numel() * ws.element_size()
     _check(lib().framefb_run(arr, len(mats), ops, dtype, wsp, wsb, _stream(stream)), "framefb_run")
+
+
+def framefb_run_static_ws(mats: Sequence[framefb_mat], ops: int, dtype: int, stream=None) -> None:
+    """framefb_run on the library's static device workspace (no allocation by anyone)."""
+    arr = _mats_array(mats)
+    _check(lib().framefb_run_static_ws(arr, len(mats), ops, dtype, _stream(stream)), "framefb_run_static_ws")
 
 
 def framefb_forward(mats, dtype, ws=None, stream=None):
