@@ -125,8 +125,11 @@ def measured_traffic():
     """ncu DRAM bytes per launch of the dominant kernel, if taken on the current kernel source."""
     import hashlib
     try:
-        src = os.path.join(ROOT, "paper_2608_26430_gb300", "csrc", "framefb_kernels.cuh")
-        h = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+        csrc = os.path.join(ROOT, "paper_2608_26430_gb300", "csrc")
+        hh = hashlib.sha256()
+        for name in ("framefb_kernels.cuh", "framefb_mma.cuh", "plan_layout.h"):
+            hh.update(open(os.path.join(csrc, name), "rb").read())
+        h = hh.hexdigest()[:16]
         with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
             return json.load(f).get(h, {}).get("bytes_per_launch")
     except Exception:
@@ -305,7 +308,7 @@ def main():
                "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                             "frac": achieved / peak,
                             "traffic": measured_traffic() if args.mats is None and args.workload is None else None, "peak_kind": peak_kind,
-                            "kernel": "tile_kernel<bf16, fwd|dx|dc> + dc_reduce", "kernel_ms": kernel_ms,
+                            "kernel": "mma_tile_kernel<fwd|dx|dc> + dc_reduce", "kernel_ms": kernel_ms,
                             "algorithmic_bytes": alg, "frac_of_8tbs": achieved / 8000.0},
                "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": 2 * args.steps,
                "clocks": clk.summary()}

@@ -268,6 +268,13 @@ framefb_status framefb_backward(const framefb_mat* mats, int32_t nmats, framefb_
 framefb_status framefb_fused_fwd_bwd(const framefb_mat* mats, int32_t nmats, framefb_dtype dtype,
                                      void* ws, size_t ws_bytes, void* stream);
 
+/* Number of waits on asynchronous row copies, since the library was loaded
+ * on the current device, that gave up after their time limit (about one
+ * second) instead of hanging; the CTA concerned stopped without finishing its
+ * tiles, so the results of that call are incomplete.  0 in normal operation.
+ * Synchronises with the device. */
+framefb_status framefb_wait_timeouts(uint32_t* count);
+
 /* ------------------------------------------------------------------------ */
 /* S7  multi-tenant merge (device)                                           */
 /* ------------------------------------------------------------------------ */

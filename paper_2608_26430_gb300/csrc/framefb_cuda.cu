@@ -11,6 +11,7 @@
 
 #include "framefb.h"
 #include "framefb_kernels.cuh"
+#include "framefb_mma.cuh"
 #include "plan_internal.h"
 #include "plan_layout.h"
 
@@ -37,11 +38,6 @@ bool frame_ok(const framefb_dev_frame* f, int32_t d) {
          f->colptr && f->rowidx;
 }
 
-// Group-0 block of column rho (subspace 1, Spectral Tetris row 0, part 0):
-// every column of a k = 16 DFT-group frame stores 32 entries, so the block
-// starts at entry 32 * rho.
-const float* twiddle_source(const framefb_dev_frame* f) { return f->val + static_cast<size_t>(32) * f->rho; }
-
 struct Prepared {
   ffb::LaunchK* args;  // heap: too large for the stack of some callers
   ffb::ReduceK* red;
@@ -49,32 +45,72 @@ struct Prepared {
   size_t smem;
   size_t ws_bytes;
   bool reg;
+  int T;  // tile tokens of the bf16 kernel
 };
 
-void* tile_kernel_ptr(framefb_dtype dt, int mode, bool reg) {
-#define FFB_CASE(E, M)                                                      \
-  case M:                                                                   \
-    return reg ? reinterpret_cast<void*>(ffb::tile_kernel<E, M, true>)      \
-               : reinterpret_cast<void*>(ffb::tile_kernel<E, M, false>);
+// bf16 activations: tensor-core kernel with staged rows (tile of T = 1 or 2
+// tokens); fp32: exact FFT kernel.
+void* tile_kernel_ptr(framefb_dtype dt, int mode, bool reg, int T) {
+#define FFB_MMA(M) \
+  case M:          \
+    return reg ? (T == 2 ? reinterpret_cast<void*>(ffb::mma_tile_kernel<M, true, 2>)            \
+                         : reinterpret_cast<void*>(ffb::mma_tile_kernel<M, true, 1>))           \
+               : (T == 2 ? reinterpret_cast<void*>(ffb::mma_tile_kernel<M, false, 2>)           \
+                         : reinterpret_cast<void*>(ffb::mma_tile_kernel<M, false, 1>));
+#define FFB_FFT(M) \
+  case M:          \
+    return reg ? reinterpret_cast<void*>(ffb::fft_tile_kernel<M, true>) : reinterpret_cast<void*>(ffb::fft_tile_kernel<M, false>);
   if (dt == FRAMEFB_BF16) {
+    if (T != 1 && T != 2) return nullptr;
     switch (mode) {
-      FFB_CASE(__nv_bfloat16, 1)
-      FFB_CASE(__nv_bfloat16, 2)
-      FFB_CASE(__nv_bfloat16, 4)
-      FFB_CASE(__nv_bfloat16, 6)
-      FFB_CASE(__nv_bfloat16, 7)
+      FFB_MMA(1)
+      FFB_MMA(2)
+      FFB_MMA(4)
+      FFB_MMA(6)
+      FFB_MMA(7)
       default: return nullptr;
     }
   }
   switch (mode) {
-    FFB_CASE(float, 1)
-    FFB_CASE(float, 2)
-    FFB_CASE(float, 4)
-    FFB_CASE(float, 6)
-    FFB_CASE(float, 7)
+    FFB_FFT(1)
+    FFB_FFT(2)
+    FFB_FFT(4)
+    FFB_FFT(6)
+    FFB_FFT(7)
     default: return nullptr;
   }
-#undef FFB_CASE
+#undef FFB_MMA
+#undef FFB_FFT
+}
+
+inline size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// Shared-memory map of the bf16 kernel for a uniform tile of T tokens: the
+// input rows (X, dY), the output rows (Y, dX) when stage_out, the fp32 tile
+// layout (largest over the matrices), two mbarriers.  Each region is sized
+// for the largest matrix; a matrix packs its rows from the region's start.
+// Returns the total bytes.
+size_t mma_smem_map(const framefb_mat* mats, int32_t nmats, int32_t ops, bool reg, int T, bool stage_out,
+                    ffb::LaunchK* a) {
+  const bool F = ops & FRAMEFB_OP_FORWARD, D = ops & FRAMEFB_OP_BACKWARD_DX, C = ops & FRAMEFB_OP_GRAD_COEFF;
+  size_t in = 0, out = 0, fp32 = 0;
+  for (int32_t j = 0; j < nmats; ++j) {
+    const FfbPlanHeader* h = plan_header(mats[j].plan);
+    const size_t rx = round_up(2 * static_cast<size_t>(h->n), 128), ry = round_up(2 * static_cast<size_t>(h->m), 128);
+    in = std::max(in, T * (((F || C) ? rx : 0) + ((D || C) ? ry : 0)));
+    if (stage_out) out = std::max(out, T * ((F ? ry : 0) + (D ? rx : 0)));
+    fp32 = std::max<size_t>(fp32, static_cast<size_t>(ffb_tile_layout(*h, ops, T, C).total) * 4);
+  }
+  const size_t fbase = round_up(in + out, 128);
+  const size_t mbar = round_up(fbase + fp32, 16);
+  if (a) {
+    a->stg_in = 0;
+    a->stg_out = static_cast<int32_t>(in);
+    a->stage_out = stage_out ? 1 : 0;
+    a->fbase = static_cast<int32_t>(fbase);
+    a->mbar = static_cast<int32_t>(mbar);
+  }
+  return mbar + 16;
 }
 
 // Validate one chunk of matrices and fill the launch parameters.
@@ -93,6 +129,22 @@ framefb_status prepare(const framefb_mat* mats, int32_t nmats, int32_t ops, fram
   }
   int64_t units = 0;
   size_t smem = 0;
+  int T_mma = 0;
+  if (dt == FRAMEFB_BF16) {
+    // one tile size for the launch; stage the output rows too when they fit,
+    // else the synthesis reads them from global memory
+    bool staged = false;
+    for (int pass = 0; pass < 2 && !T_mma; ++pass) {
+      const bool stage_out = pass == 0;
+      for (int T = 2; T >= 1 && !T_mma; --T)
+        if (mma_smem_map(mats, nmats, ops, reg, T, stage_out, nullptr) <= static_cast<size_t>(kSmemBudget)) {
+          T_mma = T;
+          staged = stage_out;
+        }
+    }
+    if (!T_mma) return FRAMEFB_EUNSUPPORTED;
+    smem = mma_smem_map(mats, nmats, ops, reg, T_mma, staged, P.args);
+  }
   for (int32_t j = 0; j < nmats; ++j) {
     const framefb_mat& M = mats[j];
     const FfbPlanHeader* h = plan_header(M.plan);
@@ -113,11 +165,14 @@ framefb_status prepare(const framefb_mat* mats, int32_t nmats, int32_t ops, fram
     }
     if (C && h->nnz > 0 && !M.dC) return FRAMEFB_EINVAL;
     // tokens per tile: as many as fit in shared memory, at most kTmax
-    int T = kTmax;
-    while (T > 1 && ffb_tile_layout(*h, ops, T, C && !reg).total * 4 > kSmemBudget) --T;
-    const size_t bytes = static_cast<size_t>(ffb_tile_layout(*h, ops, T, C && !reg).total) * 4;
-    if (bytes > static_cast<size_t>(kSmemBudget)) return FRAMEFB_EUNSUPPORTED;
-    smem = std::max(smem, bytes);
+    int T = T_mma;
+    if (dt != FRAMEFB_BF16) {
+      T = kTmax;
+      while (T > 1 && ffb_tile_layout(*h, ops, T, C).total * 4 > kSmemBudget) --T;
+      const size_t bytes = static_cast<size_t>(ffb_tile_layout(*h, ops, T, C).total) * 4;
+      if (bytes > static_cast<size_t>(kSmemBudget)) return FRAMEFB_EUNSUPPORTED;
+      smem = std::max(smem, bytes);
+    }
     const int32_t ntiles = (M.N + T - 1) / T;
     ffb::MatK& K = P.args->m[j];
     K.X = M.X;
@@ -126,8 +181,12 @@ framefb_status prepare(const framefb_mat* mats, int32_t nmats, int32_t ops, fram
     K.Y = M.Y;
     K.plan = static_cast<const uint8_t*>(M.plan_dev);
     K.c_val = M.c_val;
-    K.tw_in = twiddle_source(M.fin);
-    K.tw_out = twiddle_source(M.fout);
+    K.fval_in = M.fin->val;
+    K.fval_out = M.fout->val;
+    K.rho_in = M.fin->rho;
+    K.rho_out = M.fout->rho;
+    K.n = M.n;
+    K.m = M.m;
     K.ldx = M.ldx;
     K.ldy = M.ldy;
     K.N = M.N;
@@ -151,11 +210,12 @@ framefb_status prepare(const framefb_mat* mats, int32_t nmats, int32_t ops, fram
   P.red->total_units = static_cast<int32_t>(units);
   P.red->stride = P.args->stride;
   P.reg = reg;
+  P.T = T_mma;
   P.smem = std::max<size_t>(smem, 16);
   P.grid = 0;
   P.ws_bytes = 0;
   if (units == 0) return FRAMEFB_OK;
-  void* fn = tile_kernel_ptr(dt, ops, reg);
+  void* fn = tile_kernel_ptr(dt, ops, reg, T_mma);
   if (!fn) return FRAMEFB_EINVAL;
   int dev = 0, sms = 0, per_sm = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return FRAMEFB_ECUDA;
@@ -233,7 +293,7 @@ extern "C" framefb_status framefb_run(const framefb_mat* mats, int32_t nmats, in
     }
     P.args->partial = static_cast<float*>(ws);
     P.red->partial = static_cast<const float*>(ws);
-    void* fn = tile_kernel_ptr(dtype, ops, P.reg);
+    void* fn = tile_kernel_ptr(dtype, ops, P.reg, P.T);
     void* kargs[] = {P.args};
     if (cudaLaunchKernel(fn, dim3(P.grid), dim3(kThreads), kargs, P.smem, st) != cudaSuccess)
       return FRAMEFB_ECUDA;
@@ -352,4 +412,10 @@ extern "C" framefb_status framefb_run_static_ws(const framefb_mat* mats, int32_t
   if (s != FRAMEFB_OK) return s;
   // framefb_run rejects a need above FRAMEFB_STATIC_WS_BYTES with FRAMEFB_EWORKSPACE
   return framefb_run(mats, nmats, ops, dtype, ws, FRAMEFB_STATIC_WS_BYTES, stream);
+}
+
+extern "C" framefb_status framefb_wait_timeouts(uint32_t* count) {
+  if (!count) return FRAMEFB_EINVAL;
+  if (cudaMemcpyFromSymbol(count, ffb::g_wait_timeouts, sizeof(uint32_t)) != cudaSuccess) return FRAMEFB_ECUDA;
+  return FRAMEFB_OK;
 }

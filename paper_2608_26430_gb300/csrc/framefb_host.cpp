@@ -304,8 +304,9 @@ struct Entry { int32_t key0, key1, q; };
 
 // Cut `ent` (sorted by key0, key1) into P chunks of E entries.  Each run of
 // equal key0 inside a chunk stores its partial sum once, at its last entry:
-// the first run of a key goes to that key's own slot phys(key0); later runs
-// (the key continues from an earlier chunk) go to overflow slots base + o.
+// the first run of a key goes to that key's own slot (target = key0); later
+// runs (the key continues from an earlier chunk) go to overflow slots
+// base + o (targets >= base).
 // Returns per-entry store targets and the fix-up list.
 void cut_chunks(const std::vector<Entry>& ent, int32_t P, int32_t E, int32_t base, int32_t nkeys,
                 std::vector<int32_t>& store, std::vector<int32_t>& fix, int32_t& novf) {
@@ -322,7 +323,7 @@ void cut_chunks(const std::vector<Entry>& ent, int32_t P, int32_t E, int32_t bas
       const int32_t key = ent[e].key0;
       if (!seen[key]) {
         seen[key] = 1;
-        store[e] = ffb_phys(key);
+        store[e] = key;
       } else {
         if (first_ovf[key] < 0) first_ovf[key] = novf;
         n_ovf[key]++;
@@ -334,7 +335,7 @@ void cut_chunks(const std::vector<Entry>& ent, int32_t P, int32_t E, int32_t bas
   fix.clear();
   for (int32_t key = 0; key < nkeys; ++key) {
     if (n_ovf[key] == 0) continue;
-    fix.push_back(ffb_phys(key));
+    fix.push_back(key);
     fix.push_back(base + first_ovf[key]);
     fix.push_back(n_ovf[key]);
     fix.push_back(0);
@@ -437,7 +438,7 @@ extern "C" framefb_status framefb_plan_build(const framefb_frame* fin, const fra
         const int32_t idx = p * EZ + e;
         const size_t slot = static_cast<size_t>(e) * P + p;
         if (idx < nz) {
-          zb[slot] = ffb_phys(byrow[idx].key1) | (storeZ[idx] << 16);
+          zb[slot] = byrow[idx].key1 | (storeZ[idx] << 16);
           zq[slot] = byrow[idx].q;
         } else {
           zb[slot] = (FFB_NO_STORE << 16);
@@ -448,8 +449,8 @@ extern "C" framefb_status framefb_plan_build(const framefb_frame* fin, const fra
         const int32_t idx = p * EG + e;
         const size_t slot = static_cast<size_t>(e) * P + p;
         if (idx < nz) {
-          ga[slot] = ffb_phys(bycol[idx].key1) | (storeG[idx] << 16);
-          gb[slot] = ffb_phys(bycol[idx].key0);
+          ga[slot] = bycol[idx].key1 | (storeG[idx] << 16);
+          gb[slot] = bycol[idx].key0;
           gq[slot] = bycol[idx].q;
         } else {
           ga[slot] = (FFB_NO_STORE << 16);

@@ -11,7 +11,9 @@
 // forward DFT_16; both run here as an exact radix-4 FFT in fp32 registers.
 // The 1/4 of each side is folded into one scale s/16 applied at the end.
 // The twiddles are read from the caller's device frame (column rho: subspace
-// 1 of group 0 holds omega^j / 4 on coordinates 2j, 2j+1).
+// 1 of group 0 holds omega^j / 4 on coordinates 2j, 2j+1).  This exact FFT
+// serves fp32 activations; bf16 activations use the tensor-core kernel of
+// framefb_mma.cuh.
 #pragma once
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -36,17 +38,23 @@ struct MatK {
   void* Y;
   const uint8_t* plan;
   const float* c_val;
-  const float* tw_in;   // 32 floats: group-0 block of column rho of Phi_in
-  const float* tw_out;  // same for Phi_out
+  const float* fval_in;   // device fp32 CSC values of Phi_in (every column holds 32 entries)
+  const float* fval_out;  // same for Phi_out
   int64_t ldx, ldy;
   int32_t N, T, ubeg, ntiles;
-  float seff;           // s / 16
-  int32_t pad;
+  float seff;             // s / 16
+  int32_t rho_in, rho_out;
+  int32_t n, m;           // in / out features
 };
 
 struct LaunchK {
   int32_t nmats, total_units, stride, pad;
   float* partial;       // [(grid + nmats) * stride] dC partial sums, slot = cta + matrix
+  // shared-memory map of the bf16 tensor-core kernel (bytes): the staged
+  // input rows (X then dY of the tile) at stg_in, the staged output rows (Y
+  // then dX) at stg_out when stage_out is set (else read from global
+  // memory), the fp32 region of the tile layout at fbase, two mbarriers
+  int32_t stg_in, stg_out, stage_out, fbase, mbar, pad2;
   MatK m[kMaxMats];
 };
 
@@ -155,53 +163,11 @@ __device__ __forceinline__ void fft16(float (&xr)[16], float (&xi)[16], const Tw
 __device__ __forceinline__ constexpr int slot_of(int k) { return 4 * (k & 3) + (k >> 2); }
 
 // ---------------------------------------------------------------------------
-// 32-element row segments of activations: load as 16 complex values
+// 32-element fp32 row segments of activations: load as 16 complex values
 // (x_{2j}, x_{2j+1}), and read-modify-write y += seff * delta.
 // ---------------------------------------------------------------------------
 template <typename Elem>
 struct Seg;
-
-template <>
-struct Seg<__nv_bfloat16> {
-  uint4 q[4];
-  __device__ __forceinline__ void load_stream(const void* p) {
-    const uint4* s = reinterpret_cast<const uint4*>(p);
-#pragma unroll
-    for (int i = 0; i < 4; ++i) q[i] = __ldcs(s + i);
-  }
-  __device__ __forceinline__ void load(const void* p) {
-    const uint4* s = reinterpret_cast<const uint4*>(p);
-#pragma unroll
-    for (int i = 0; i < 4; ++i) q[i] = s[i];
-  }
-  __device__ __forceinline__ uint32_t word(int j) const {
-    const uint4& v = q[j >> 2];
-    return (j & 3) == 0 ? v.x : (j & 3) == 1 ? v.y : (j & 3) == 2 ? v.z : v.w;
-  }
-  __device__ __forceinline__ void unpack(float (&xr)[16], float (&xi)[16]) const {
-#pragma unroll
-    for (int j = 0; j < 16; ++j) {
-      const uint32_t w = word(j);
-      xr[j] = __uint_as_float(w << 16);
-      xi[j] = __uint_as_float(w & 0xFFFF0000u);
-    }
-  }
-  // y_{2j} += seff * dr[slot_of(j)], y_{2j+1} += seff * di[slot_of(j)], stored to p
-  __device__ __forceinline__ void add_store(void* p, const float (&dr)[16], const float (&di)[16], float seff) {
-    uint32_t out[16];
-#pragma unroll
-    for (int j = 0; j < 16; ++j) {
-      const uint32_t w = word(j);
-      const float lo = fmaf(seff, dr[slot_of(j)], __uint_as_float(w << 16));
-      const float hi = fmaf(seff, di[slot_of(j)], __uint_as_float(w & 0xFFFF0000u));
-      const __nv_bfloat162 b = __floats2bfloat162_rn(lo, hi);
-      out[j] = *reinterpret_cast<const uint32_t*>(&b);
-    }
-    uint4* d = reinterpret_cast<uint4*>(p);
-#pragma unroll
-    for (int i = 0; i < 4; ++i) d[i] = make_uint4(out[4 * i], out[4 * i + 1], out[4 * i + 2], out[4 * i + 3]);
-  }
-};
 
 template <>
 struct Seg<float> {
@@ -237,13 +203,15 @@ struct Seg<float> {
 };
 
 // Store the 32 coefficients of one group (analysis output, slot order) into a
-// swizzled shared-memory token row: chunk c = (V_{2c}, V_{2c+1}) complex.
+// token row laid out by ffb_slot: float4 chunk j (pairs 2j, 2j + 1) goes to
+// chunk j ^ ((j >> 2) & 1), its two pairs swapped when the group is odd.
 __device__ __forceinline__ void store_group(float* row, int g, const float (&xr)[16], const float (&xi)[16]) {
   float* base = row + 32 * g;
 #pragma unroll
   for (int c = 0; c < 8; ++c) {
     const int p0 = slot_of(2 * c), p1 = slot_of(2 * c + 1);
-    *reinterpret_cast<float4*>(base + 4 * (c ^ (g & 7))) = make_float4(xr[p0], xi[p0], xr[p1], xi[p1]);
+    const float4 v = (g & 1) ? make_float4(xr[p1], xi[p1], xr[p0], xi[p0]) : make_float4(xr[p0], xi[p0], xr[p1], xi[p1]);
+    *reinterpret_cast<float4*>(base + 4 * (c ^ ((c >> 2) & 1))) = v;
   }
 }
 
@@ -252,11 +220,12 @@ __device__ __forceinline__ void load_group(const float* row, int g, float (&xr)[
   const float* base = row + 32 * g;
 #pragma unroll
   for (int c = 0; c < 8; ++c) {
-    const float4 v = *reinterpret_cast<const float4*>(base + 4 * (c ^ (g & 7)));
-    xr[2 * c] = v.x;
-    xi[2 * c] = v.y;
-    xr[2 * c + 1] = v.z;
-    xi[2 * c + 1] = v.w;
+    const float4 v = *reinterpret_cast<const float4*>(base + 4 * (c ^ ((c >> 2) & 1)));
+    const bool sw = g & 1;
+    xr[2 * c] = sw ? v.z : v.x;
+    xi[2 * c] = sw ? v.w : v.y;
+    xr[2 * c + 1] = sw ? v.x : v.z;
+    xi[2 * c + 1] = sw ? v.y : v.w;
   }
 }
 
@@ -272,49 +241,356 @@ __device__ __forceinline__ int32_t cta_of_unit(int64_t u, int64_t grid, int64_t 
   return static_cast<int32_t>(((u + 1) * grid - 1) / units);
 }
 
-// Write this thread's dC partial sums of one matrix to its workspace slot.
-template <bool C, bool REG, int E>
-__device__ __forceinline__ void flush_dc(const uint8_t* plan, int EG, float* dst, const float (&dc)[E],
-                                         const float* dcs, int tid) {
-  if constexpr (C) {
-    const int32_t* gq = table<int32_t>(plan, hdr(plan).off_gq);
+// ---------------------------------------------------------------------------
+// Sparse phase shared by both tile kernels.  A thread owns one chunk of the
+// support ordered by row (for Y) and one ordered by column (for dX and dC).
+// REG: the chunk (at most kEreg entries) lives in registers for the whole
+// matrix; otherwise it is streamed from the plan on every tile and the dC
+// accumulators live in shared memory.
+// ---------------------------------------------------------------------------
+// Per-slot token vectors of the sparse phase: TT tokens of one slot.
+// MINOR (token-minor) with TT = 2 uses one 8-byte access; otherwise TT
+// scalar accesses at stride `stride` (token-major) or 1 (token-minor, TT = 1).
+template <int TT, bool MINOR>
+struct Vecs {
+  struct type {
+    float v[TT];
+  };
+  static __device__ __forceinline__ type zero() {
+    type r;
+#pragma unroll
+    for (int t = 0; t < TT; ++t) r.v[t] = 0.f;
+    return r;
+  }
+  static __device__ __forceinline__ type load(const type* base, uint32_t slot, int stride) {
+    const float* b = reinterpret_cast<const float*>(base);
+    type r;
+#pragma unroll
+    for (int t = 0; t < TT; ++t) r.v[t] = MINOR ? b[slot * TT + t] : b[t * stride + slot];
+    return r;
+  }
+  static __device__ __forceinline__ void store(type* base, uint32_t slot, int stride, const type& x) {
+    float* b = reinterpret_cast<float*>(base);
+#pragma unroll
+    for (int t = 0; t < TT; ++t) {
+      if (MINOR)
+        b[slot * TT + t] = x.v[t];
+      else
+        b[t * stride + slot] = x.v[t];
+    }
+  }
+  static __device__ __forceinline__ void fma(type& acc, float c, const type& x) {
+#pragma unroll
+    for (int t = 0; t < TT; ++t) acc.v[t] = fmaf(c, x.v[t], acc.v[t]);
+  }
+  static __device__ __forceinline__ float dot(const type& a, const type& b) {
+    float s = 0.f;
+#pragma unroll
+    for (int t = 0; t < TT; ++t) s = fmaf(a.v[t], b.v[t], s);
+    return s;
+  }
+};
+
+template <>
+struct Vecs<2, true> {
+  using type = float2;
+  static __device__ __forceinline__ float2 zero() { return make_float2(0.f, 0.f); }
+  static __device__ __forceinline__ float2 load(const float2* base, uint32_t slot, int) { return base[slot]; }
+  static __device__ __forceinline__ void store(float2* base, uint32_t slot, int, const float2& x) { base[slot] = x; }
+  static __device__ __forceinline__ void fma(float2& acc, float c, const float2& x) {
+    acc.x = fmaf(c, x.x, acc.x);
+    acc.y = fmaf(c, x.y, acc.y);
+  }
+  static __device__ __forceinline__ float dot(const float2& a, const float2& b) { return fmaf(a.x, b.x, a.y * b.y); }
+};
+
+template <int MODE, bool REG>
+struct Chunk {
+  static constexpr bool F = MODE & MODE_F, D = MODE & MODE_D, C = MODE & MODE_C;
+  static constexpr int E = REG ? kEreg : 1;
+  // zb: V slot of b | RZ slot of the store target << 16 (FFB_NO_STORE: none)
+  // ga: U slot of a | RG slot of the store target << 16;  gb: V slot of b
+  uint32_t zb[E], ga[E], gb[E];
+  float zc[E], gc[E];
+  int EZ, EG, n, m;
+
+  // plan word (index | target << 16) -> (slot | slot << 16)
+  static __device__ __forceinline__ uint32_t slots(uint32_t w, int Klo, int Khi) {
+    const uint32_t lo = w & 0xFFFFu, hi = w >> 16;
+    const uint32_t slo = static_cast<uint32_t>(ffb_slot(static_cast<int32_t>(lo), Klo));
+    const uint32_t shi = hi == FFB_NO_STORE ? FFB_NO_STORE : static_cast<uint32_t>(ffb_slot(static_cast<int32_t>(hi), Khi));
+    return slo | (shi << 16);
+  }
+
+  __device__ __forceinline__ void load(const uint8_t* plan, const float* c_val, int tid) {
+    const FfbPlanHeader& h = hdr(plan);
+    EZ = h.EZ;
+    EG = h.EG;
+    n = h.n;
+    m = h.m;
+#pragma unroll
+    for (int e = 0; e < E; ++e) {
+      zb[e] = FFB_NO_STORE << 16;
+      ga[e] = FFB_NO_STORE << 16;
+      gb[e] = 0;
+      zc[e] = gc[e] = 0.f;
+    }
     if constexpr (REG) {
+      const int32_t* tzb = table<int32_t>(plan, h.off_zb);
+      const int32_t* tzq = table<int32_t>(plan, h.off_zq);
+      const int32_t* tga = table<int32_t>(plan, h.off_ga);
+      const int32_t* tgb = table<int32_t>(plan, h.off_gb);
+      const int32_t* tgq = table<int32_t>(plan, h.off_gq);
 #pragma unroll
       for (int e = 0; e < E; ++e) {
-        if (e < EG) {
-          const int32_t q = __ldg(gq + e * kThreads + tid);
-          if (q >= 0) dst[q] = dc[e];
+        if (F && e < EZ) {
+          zb[e] = slots(static_cast<uint32_t>(__ldg(tzb + e * kThreads + tid)), n, m);
+          const int32_t q = __ldg(tzq + e * kThreads + tid);
+          zc[e] = q >= 0 ? __ldg(c_val + q) : 0.f;
+        }
+        if ((D || C) && e < EG) {
+          ga[e] = slots(static_cast<uint32_t>(__ldg(tga + e * kThreads + tid)), m, n);
+          gb[e] = static_cast<uint32_t>(ffb_slot(__ldg(tgb + e * kThreads + tid), n));
+          const int32_t q = __ldg(tgq + e * kThreads + tid);
+          gc[e] = (D && q >= 0) ? __ldg(c_val + q) : 0.f;
         }
       }
+    }
+  }
+
+  // One block of B entries of the row side from the register chunk or the
+  // streamed tables: (plan word as slots, c).
+  __device__ __forceinline__ void z_entry(const uint8_t* plan, const float* c_val, int tid, int e, uint32_t& w,
+                                          float& c) const {
+    if constexpr (REG) {
+      (void)plan;
+      (void)c_val;
+      (void)tid;
+      w = zb[e];
+      c = zc[e];
     } else {
+      w = slots(static_cast<uint32_t>(__ldg(table<int32_t>(plan, hdr(plan).off_zb) + e * kThreads + tid)), n, m);
+      const int32_t q = __ldg(table<int32_t>(plan, hdr(plan).off_zq) + e * kThreads + tid);
+      c = q >= 0 ? __ldg(c_val + q) : 0.f;
+    }
+  }
+  __device__ __forceinline__ void g_entry(const uint8_t* plan, const float* c_val, int tid, int e, uint32_t& wa,
+                                          uint32_t& wb, float& c) const {
+    if constexpr (REG) {
+      (void)plan;
+      (void)c_val;
+      (void)tid;
+      wa = ga[e];
+      wb = gb[e];
+      c = gc[e];
+    } else {
+      wa = slots(static_cast<uint32_t>(__ldg(table<int32_t>(plan, hdr(plan).off_ga) + e * kThreads + tid)), m, n);
+      wb = static_cast<uint32_t>(ffb_slot(__ldg(table<int32_t>(plan, hdr(plan).off_gb) + e * kThreads + tid), n));
+      c = 0.f;
+      if constexpr (D) {
+        const int32_t q = __ldg(table<int32_t>(plan, hdr(plan).off_gq) + e * kThreads + tid);
+        c = q >= 0 ? __ldg(c_val + q) : 0.f;
+      }
+    }
+  }
+
+  // Y side (by row): RZ[st] = sum over a run of equal rows of c V[b].
+  // dX side (by column): RG[st] = sum over a run of equal columns of c U[a].
+  // dC: dc += sum over the tile's tokens of U[a] V[b].
+  // TT tokens in the tile.  Element (token t, slot s) lives at s * TT + t
+  // (MINOR: token-minor, one vector access per slot) or t * stride + s.
+  // V / U (read) and RZ / RG (written) are disjoint regions: the restrict
+  // pointers let the loads of a block of entries issue ahead of the stores
+  // of the previous block.
+  template <int TT, bool MINOR>
+  __device__ __forceinline__ void z_block(const uint8_t* plan, const float* c_val, int tid, int e0,
+                                          const typename Vecs<TT, MINOR>::type* __restrict__ V,
+                                          typename Vecs<TT, MINOR>::type* __restrict__ RZ, int sV, int sRZ,
+                                          typename Vecs<TT, MINOR>::type& acc) const {
+    using Vec = typename Vecs<TT, MINOR>::type;
+    constexpr int B = FFB_ENTRY_BLOCK;
+    uint32_t w[B];
+    float c[B];
+    Vec v[B];
+#pragma unroll
+    for (int e = 0; e < B; ++e) {
+      if (REG || e0 + e < EZ) {
+        z_entry(plan, c_val, tid, e0 + e, w[e], c[e]);
+      } else {
+        w[e] = FFB_NO_STORE << 16;
+        c[e] = 0.f;
+      }
+      v[e] = Vecs<TT, MINOR>::load(V, w[e] & 0xFFFFu, sV);
+    }
+#pragma unroll
+    for (int e = 0; e < B; ++e) {
+      Vecs<TT, MINOR>::fma(acc, c[e], v[e]);
+      const uint32_t st = w[e] >> 16;
+      if (st != FFB_NO_STORE) {
+        Vecs<TT, MINOR>::store(RZ, st, sRZ, acc);
+        acc = Vecs<TT, MINOR>::zero();
+      }
+    }
+  }
+
+  template <int TT, bool MINOR>
+  __device__ __forceinline__ void g_block(const uint8_t* plan, const float* c_val, int tid, int e0,
+                                          const typename Vecs<TT, MINOR>::type* __restrict__ U,
+                                          const typename Vecs<TT, MINOR>::type* __restrict__ V,
+                                          typename Vecs<TT, MINOR>::type* __restrict__ RG, float* __restrict__ dcs,
+                                          int sU, int sV, int sRG, typename Vecs<TT, MINOR>::type& acc) const {
+    using Vec = typename Vecs<TT, MINOR>::type;
+    constexpr int B = FFB_ENTRY_BLOCK;
+    uint32_t wa[B], wb[B];
+    float c[B];
+    Vec uu[B], vv[B];
+#pragma unroll
+    for (int e = 0; e < B; ++e) {
+      if (REG || e0 + e < EG) {
+        g_entry(plan, c_val, tid, e0 + e, wa[e], wb[e], c[e]);
+      } else {
+        wa[e] = FFB_NO_STORE << 16;
+        wb[e] = 0;
+        c[e] = 0.f;
+      }
+      uu[e] = Vecs<TT, MINOR>::load(U, wa[e] & 0xFFFFu, sU);
+      if constexpr (C) vv[e] = Vecs<TT, MINOR>::load(V, wb[e], sV);
+    }
+    float dsum[B];
+#pragma unroll
+    for (int e = 0; e < B; ++e) {
+      if constexpr (C) dsum[e] = Vecs<TT, MINOR>::dot(uu[e], vv[e]);
+      if constexpr (D) {
+        Vecs<TT, MINOR>::fma(acc, c[e], uu[e]);
+        const uint32_t st = wa[e] >> 16;
+        if (st != FFB_NO_STORE) {
+          Vecs<TT, MINOR>::store(RG, st, sRG, acc);
+          acc = Vecs<TT, MINOR>::zero();
+        }
+      }
+    }
+    if constexpr (C) {
+#pragma unroll
+      for (int e = 0; e < B; ++e) dcs[(e0 + e) * kThreads + tid] += dsum[e];
+    }
+  }
+
+  // Y side (by row): RZ[st] = sum over a run of equal rows of c V[b].
+  // dX side (by column): RG[st] = sum over a run of equal columns of c U[a].
+  // dC: dc += sum over the tile's tokens of U[a] V[b].
+  // TT tokens in the tile.  Element (token t, slot s) lives at s * TT + t
+  // (MINOR: token-minor, one vector access per slot) or t * stride + s.
+  // V / U (read) and RZ / RG (written) are disjoint regions: the restrict
+  // pointers let the loads of a block of entries issue ahead of the stores
+  // of the previous block.
+  template <int TT, bool MINOR>
+  __device__ __forceinline__ void sparse_tt(const uint8_t* plan, const float* c_val, int tid, const FfbTileLayout& L,
+                                            float* fsm) {
+    using Vec = typename Vecs<TT, MINOR>::type;
+    const Vec* V = reinterpret_cast<const Vec*>(fsm + L.oV);
+    const Vec* U = reinterpret_cast<const Vec*>(fsm + L.oU);
+    Vec* RZ = reinterpret_cast<Vec*>(fsm + L.oRZ);
+    Vec* RG = reinterpret_cast<Vec*>(fsm + L.oRG);
+    float* dcs = fsm + L.oDC;
+    constexpr int B = FFB_ENTRY_BLOCK;
+    static_assert(kEreg % B == 0, "register chunk must hold whole blocks");
+    if constexpr (F) {
+      Vec acc = Vecs<TT, MINOR>::zero();
+      if constexpr (REG) {
+#pragma unroll
+        for (int e0 = 0; e0 < E; e0 += B)
+          if (e0 < EZ) z_block<TT, MINOR>(plan, c_val, tid, e0, V, RZ, L.sV, L.sRZ, acc);
+      } else {
+        for (int e0 = 0; e0 < EZ; e0 += B) z_block<TT, MINOR>(plan, c_val, tid, e0, V, RZ, L.sV, L.sRZ, acc);
+      }
+    }
+    if constexpr (D || C) {
+      Vec acc = Vecs<TT, MINOR>::zero();
+      if constexpr (REG) {
+#pragma unroll
+        for (int e0 = 0; e0 < E; e0 += B)
+          if (e0 < EG) g_block<TT, MINOR>(plan, c_val, tid, e0, U, V, RG, dcs, L.sU, L.sV, L.sRG, acc);
+      } else {
+        for (int e0 = 0; e0 < EG; e0 += B)
+          g_block<TT, MINOR>(plan, c_val, tid, e0, U, V, RG, dcs, L.sU, L.sV, L.sRG, acc);
+      }
+    }
+  }
+
+  template <bool MINOR>
+  __device__ __forceinline__ void sparse(const uint8_t* plan, const float* c_val, int tid, const FfbTileLayout& L,
+                                         float* fsm, int Tc) {
+    switch (Tc) {
+      case 1: sparse_tt<1, MINOR>(plan, c_val, tid, L, fsm); break;
+      case 2: sparse_tt<2, MINOR>(plan, c_val, tid, L, fsm); break;
+      case 3: sparse_tt<3, MINOR>(plan, c_val, tid, L, fsm); break;
+      default: sparse_tt<4, MINOR>(plan, c_val, tid, L, fsm); break;
+    }
+  }
+
+  // Write this thread's dC partial sums of one matrix to its workspace slot
+  // (the accumulators live in shared memory, one column per thread).
+  __device__ __forceinline__ void flush(const uint8_t* plan, float* dst, const FfbTileLayout& L, const float* fsm,
+                                        int tid) {
+    if constexpr (C) {
+      const int32_t* gq = table<int32_t>(plan, hdr(plan).off_gq);
+      const float* dcs = fsm + L.oDC;
       for (int e = 0; e < EG; ++e) {
         const int32_t q = __ldg(gq + e * kThreads + tid);
         if (q >= 0) dst[q] = dcs[e * kThreads + tid];
       }
     }
   }
+};
+
+// Rows (columns) of C whose entries were split between chunks: add the
+// later pieces, stored in overflow slots, to the first piece.  Needs a
+// barrier before (pieces written) and after (sums complete).  Element
+// (token t, slot s) at s * T + t (minor) or t * stride + s.
+template <int MODE, bool MINOR>
+__device__ __forceinline__ void fixup(const uint8_t* plan, const FfbTileLayout& L, float* fsm, int T, int Tc,
+                                      int tid) {
+  constexpr bool F = MODE & MODE_F, D = MODE & MODE_D;
+  const FfbPlanHeader& h = hdr(plan);
+  const int nfZ = F ? h.nfixZ : 0, nfG = D ? h.nfixG : 0;
+  for (int i = tid; i < nfZ + nfG; i += kThreads) {
+    const bool z = i < nfZ;
+    const int4 it = z ? __ldg(table<int4>(plan, h.off_fixZ) + i) : __ldg(table<int4>(plan, h.off_fixG) + (i - nfZ));
+    float* R = fsm + (z ? L.oRZ : L.oRG);
+    const int stride = z ? L.sRZ : L.sRG;
+    const int dst = ffb_slot(it.x, z ? h.m : h.n);
+    for (int t = 0; t < Tc; ++t) {
+      float* Rt = MINOR ? R + t : R + t * stride;
+      const int sc = MINOR ? T : 1;
+      float sacc = Rt[dst * sc];
+      for (int c2 = 0; c2 < it.z; ++c2) sacc += Rt[(it.y + c2) * sc];
+      Rt[dst * sc] = sacc;
+    }
+  }
+}
+
+__device__ __forceinline__ int fix_count(const uint8_t* plan, int mode) {
+  const FfbPlanHeader& h = hdr(plan);
+  return ((mode & MODE_F) ? h.nfixZ : 0) + ((mode & MODE_D) ? h.nfixG : 0);
 }
 
 // ---------------------------------------------------------------------------
-// Tile kernel.  Persistent CTAs walk a contiguous range of units (matrix,
-// tile of T tokens), matrix-major.  Per tile:
-//   A  analysis: V = X Phi_in, U = dY Phi_out for every group touched by the
-//      support (FFT_16 per token and group), into shared memory;
-//   B1 coefficient SpMM by balanced chunks: row sums of c V[b] for Y (RZ),
-//      column sums of c U[a] for dX (RG), and dC += U[a] V[b];
-//   B2 fix-up of rows/columns whose entries were split between chunks;
+// fp32 tile kernel (exact radix-4 FFT_16 on CUDA cores).  Persistent CTAs
+// walk a contiguous range of units (matrix, tile of T tokens), matrix-major:
+//   A  analysis: V = X Phi_in, U = dY Phi_out per 32-coordinate group;
+//   B1 the sparse phase (Chunk::sparse); B2 fix-up;
 //   B3 synthesis: FFT_16 of RZ / RG per group and y += (s/16) * result.
 // dC accumulates over the CTA's tiles of a matrix and is written to the
 // workspace slot (cta + matrix) when the CTA leaves the matrix.
 // ---------------------------------------------------------------------------
-template <typename Elem, int MODE, bool REG>
-__global__ void __launch_bounds__(kThreads, 1) tile_kernel(const __grid_constant__ LaunchK args) {
+template <int MODE, bool REG>
+__global__ void __launch_bounds__(kThreads, 1) fft_tile_kernel(const __grid_constant__ LaunchK args) {
+  using Elem = float;
   constexpr bool F = MODE & MODE_F, D = MODE & MODE_D, C = MODE & MODE_C;
   constexpr bool NEED_V = F || C, NEED_U = D || C;
-  constexpr int E = REG ? kEreg : 1;
   constexpr size_t ELEM = sizeof(Elem);
   extern __shared__ float4 smem4[];
-  float* smem = reinterpret_cast<float*>(smem4);
+  float* fsm = reinterpret_cast<float*>(smem4);
   const int tid = threadIdx.x;
 
   const int64_t units = args.total_units;
@@ -322,81 +598,43 @@ __global__ void __launch_bounds__(kThreads, 1) tile_kernel(const __grid_constant
   const int64_t u_end = (static_cast<int64_t>(blockIdx.x + 1) * units) / gridDim.x;
   if (u_begin >= u_end) return;
 
-  // register-resident chunk (REG) -- by row for Y, by column for dX / dC
-  uint32_t zb[E], ga[E], gb[E];
-  float zc[E], gc[E], dc[E];
-#pragma unroll
-  for (int e = 0; e < E; ++e) {
-    zb[e] = ga[e] = gb[e] = 0;
-    zc[e] = gc[e] = dc[e] = 0.f;
-  }
-
+  Chunk<MODE, REG> ch;
   int j = 0;
   while (j + 1 < args.nmats && u_begin >= args.m[j].ubeg + args.m[j].ntiles) ++j;
   int cur = -1;
   const uint8_t* plan = nullptr;
   FfbTileLayout L{};
   Tw tw_in{}, tw_out{};
-  int EZ = 0, EG = 0, Gn = 0, Gm = 0, nfixZ = 0, nfixG = 0, T = 1;
-  float* dcs = nullptr;
+  int Gn = 0, Gm = 0, T = 1;
 
   for (int64_t u = u_begin; u < u_end; ++u) {
     while (u >= args.m[j].ubeg + args.m[j].ntiles) ++j;
     const MatK& M = args.m[j];
     if (j != cur) {
-      if (cur >= 0) flush_dc<C, REG, E>(plan, EG, args.partial + static_cast<size_t>(blockIdx.x + cur) * args.stride, dc, dcs, tid);
+      if (cur >= 0) ch.flush(plan, args.partial + static_cast<size_t>(blockIdx.x + cur) * args.stride, L, fsm, tid);
       cur = j;
       plan = M.plan;
       const FfbPlanHeader& h = hdr(plan);
-      EZ = h.EZ;
-      EG = h.EG;
       Gn = h.Gn;
       Gm = h.Gm;
-      nfixZ = h.nfixZ;
-      nfixG = h.nfixG;
       T = M.T;
       FfbPlanHeader hc = h;
-      L = ffb_tile_layout(hc, MODE, T, C && !REG);
-      tw_in = load_tw(M.tw_in);
-      tw_out = load_tw(M.tw_out);
+      L = ffb_tile_layout(hc, MODE, T, C);
+      tw_in = load_tw(M.fval_in + 32 * M.rho_in);
+      tw_out = load_tw(M.fval_out + 32 * M.rho_out);
       __syncthreads();  // every thread is done with the previous matrix's shared memory
-      for (int i = tid; i < L.total - L.oRZ; i += kThreads) smem[L.oRZ + i] = 0.f;
-      dcs = smem + L.oDC;
-      if constexpr (REG) {
-        const int32_t* tzb = table<int32_t>(plan, h.off_zb);
-        const int32_t* tzq = table<int32_t>(plan, h.off_zq);
-        const int32_t* tga = table<int32_t>(plan, h.off_ga);
-        const int32_t* tgb = table<int32_t>(plan, h.off_gb);
-        const int32_t* tgq = table<int32_t>(plan, h.off_gq);
-#pragma unroll
-        for (int e = 0; e < E; ++e) {
-          zb[e] = FFB_NO_STORE << 16;
-          ga[e] = FFB_NO_STORE << 16;
-          gb[e] = 0;
-          zc[e] = gc[e] = dc[e] = 0.f;
-          if (F && e < EZ) {
-            zb[e] = static_cast<uint32_t>(__ldg(tzb + e * kThreads + tid));
-            const int32_t q = __ldg(tzq + e * kThreads + tid);
-            zc[e] = q >= 0 ? __ldg(M.c_val + q) : 0.f;
-          }
-          if ((D || C) && e < EG) {
-            ga[e] = static_cast<uint32_t>(__ldg(tga + e * kThreads + tid));
-            gb[e] = static_cast<uint32_t>(__ldg(tgb + e * kThreads + tid));
-            const int32_t q = __ldg(tgq + e * kThreads + tid);
-            gc[e] = (D && q >= 0) ? __ldg(M.c_val + q) : 0.f;
-          }
-        }
-      }
+      for (int i = tid; i < L.total - L.oRZ; i += kThreads) fsm[L.oRZ + i] = 0.f;
+      ch.load(plan, M.c_val, tid);
       __syncthreads();
     }
 
     const int64_t t0 = static_cast<int64_t>(u - M.ubeg) * T;
     const int64_t left = static_cast<int64_t>(M.N) - t0;
     const int Tc = static_cast<int>(left < T ? left : T);
-    float* V = smem + L.oV;
-    float* U = smem + L.oU;
-    float* RZ = smem + L.oRZ;
-    float* RG = smem + L.oRG;
+    float* V = fsm + L.oV;
+    float* U = fsm + L.oU;
+    float* RZ = fsm + L.oRZ;
+    float* RG = fsm + L.oRG;
     const uint32_t* zmask = table<uint32_t>(plan, hdr(plan).off_zmask);
     const uint32_t* gmask = table<uint32_t>(plan, hdr(plan).off_gmask);
 
@@ -429,104 +667,13 @@ __global__ void __launch_bounds__(kThreads, 1) tile_kernel(const __grid_constant
     }
     __syncthreads();
 
-    // ---- B1: coefficient SpMM / SDDMM over this thread's chunk -------------
-    // Y side (by row): RZ[st] = sum over a run of equal rows of c * V[b].
-    // dX side (by column): RG[st] = sum over a run of equal columns of c * U[a];
-    // dC: dc += U[a] V[b] summed over the tile's tokens.
-    if constexpr (F) {
-      float acc[kTmax] = {0.f, 0.f, 0.f, 0.f};
-      auto step = [&](uint32_t pk, float c) {
-        const uint32_t bo = pk & 0xFFFFu, st = pk >> 16;
-#pragma unroll
-        for (int t = 0; t < kTmax; ++t)
-          if (t < Tc) acc[t] = fmaf(c, V[t * L.sV + bo], acc[t]);
-        if (st != FFB_NO_STORE) {
-#pragma unroll
-          for (int t = 0; t < kTmax; ++t) {
-            if (t < Tc) RZ[t * L.sRZ + st] = acc[t];
-            acc[t] = 0.f;
-          }
-        }
-      };
-      if constexpr (REG) {
-#pragma unroll
-        for (int e = 0; e < E; ++e)
-          if (e < EZ) step(zb[e], zc[e]);
-      } else {
-        const int32_t* tzb = table<int32_t>(plan, hdr(plan).off_zb);
-        const int32_t* tzq = table<int32_t>(plan, hdr(plan).off_zq);
-        for (int e = 0; e < EZ; ++e) {
-          const uint32_t pk = static_cast<uint32_t>(__ldg(tzb + e * kThreads + tid));
-          const int32_t q = __ldg(tzq + e * kThreads + tid);
-          step(pk, q >= 0 ? __ldg(M.c_val + q) : 0.f);
-        }
-      }
-    }
-    if constexpr (D || C) {
-      float acc[kTmax] = {0.f, 0.f, 0.f, 0.f};
-      auto step = [&](uint32_t pa, uint32_t pb, float c) -> float {
-        const uint32_t ao = pa & 0xFFFFu, st = pa >> 16;
-        float dcv = 0.f;
-#pragma unroll
-        for (int t = 0; t < kTmax; ++t) {
-          if (t < Tc) {
-            const float uv = U[t * L.sU + ao];
-            if constexpr (D) acc[t] = fmaf(c, uv, acc[t]);
-            if constexpr (C) dcv = fmaf(uv, V[t * L.sV + pb], dcv);
-          }
-        }
-        if constexpr (D) {
-          if (st != FFB_NO_STORE) {
-#pragma unroll
-            for (int t = 0; t < kTmax; ++t) {
-              if (t < Tc) RG[t * L.sRG + st] = acc[t];
-              acc[t] = 0.f;
-            }
-          }
-        }
-        return dcv;
-      };
-      if constexpr (REG) {
-#pragma unroll
-        for (int e = 0; e < E; ++e)
-          if (e < EG) {
-            const float dcv = step(ga[e], gb[e], gc[e]);
-            if constexpr (C) dc[e] += dcv;
-          }
-      } else {
-        const int32_t* tga = table<int32_t>(plan, hdr(plan).off_ga);
-        const int32_t* tgb = table<int32_t>(plan, hdr(plan).off_gb);
-        const int32_t* tgq = table<int32_t>(plan, hdr(plan).off_gq);
-        for (int e = 0; e < EG; ++e) {
-          const uint32_t pa = static_cast<uint32_t>(__ldg(tga + e * kThreads + tid));
-          const uint32_t pb = static_cast<uint32_t>(__ldg(tgb + e * kThreads + tid));
-          float c = 0.f;
-          if constexpr (D) {
-            const int32_t q = __ldg(tgq + e * kThreads + tid);
-            c = q >= 0 ? __ldg(M.c_val + q) : 0.f;
-          }
-          const float dcv = step(pa, pb, c);
-          if constexpr (C) dcs[e * kThreads + tid] += dcv;
-        }
-      }
-    }
+    // ---- B1: sparse phase -------------------------------------------------
+    ch.template sparse<false>(plan, M.c_val, tid, L, fsm, Tc);
     if constexpr (F || D) {
-      // ---- B2: rows / columns split between chunks ----------------------
-      const int nfix = (F ? nfixZ : 0) + (D ? nfixG : 0);
-      if (nfix > 0) {
+      // ---- B2: fix-up ---------------------------------------------------
+      if (fix_count(plan, MODE) > 0) {
         __syncthreads();
-        for (int i = tid; i < nfix; i += kThreads) {
-          const bool z = F && i < (F ? nfixZ : 0);
-          const int4 it = z ? __ldg(table<int4>(plan, hdr(plan).off_fixZ) + i)
-                            : __ldg(table<int4>(plan, hdr(plan).off_fixG) + (i - (F ? nfixZ : 0)));
-          float* R = z ? RZ : RG;
-          const int stride = z ? L.sRZ : L.sRG;
-          for (int t = 0; t < Tc; ++t) {
-            float sacc = R[t * stride + it.x];
-            for (int c2 = 0; c2 < it.z; ++c2) sacc += R[t * stride + it.y + c2];
-            R[t * stride + it.x] = sacc;
-          }
-        }
+        fixup<MODE, false>(plan, L, fsm, T, Tc, tid);
       }
       __syncthreads();
 
@@ -559,11 +706,10 @@ __global__ void __launch_bounds__(kThreads, 1) tile_kernel(const __grid_constant
       }
     }
     // The next tile's analysis writes V/U only: ordered after this tile's
-    // B1 reads by the barrier above (or the one below for dC-only runs).
+    // sparse-phase reads by the barrier above (or the one below for dC-only runs).
     if constexpr (!(F || D)) __syncthreads();
   }
-  if (cur >= 0)
-    flush_dc<C, REG, E>(plan, EG, args.partial + static_cast<size_t>(blockIdx.x + cur) * args.stride, dc, dcs, tid);
+  if (cur >= 0) ch.flush(plan, args.partial + static_cast<size_t>(blockIdx.x + cur) * args.stride, L, fsm, tid);
 }
 
 // dC_q = (s/16) * sum over the CTAs that visited the matrix, in CTA order.

@@ -9,10 +9,11 @@
 // columns [32 r, 32 r + 32): its coefficient vector is the 16 complex values
 // (Re, Im interleaved) of the DFT_16 of that coordinate block.
 //
-// Inside shared memory a token row of frame coefficients is stored with its
-// 16-byte chunks XOR-swizzled inside each 128-byte group, so that a warp
-// writing or reading 32 consecutive groups hits 32 distinct banks:
-//     phys(x) = 32 g + 4 ((x/4 mod 8) xor (g mod 8)) + x mod 4,   g = x / 32.
+// The tables hold these group-major indices.  A store target t < K (K = m
+// for the row side, n for the column side) is the index of the run's own
+// row or column; t >= K is an overflow slot, kept after the K regular slots.
+// Each kernel maps indices to its own shared-memory slots (ffb_slot below
+// for the tile layouts) when it loads the tables.
 #pragma once
 #include <stdint.h>
 
@@ -29,6 +30,7 @@
 #define FFB_PLAN_VERSION 1
 #define FFB_GROUP 32               /* real coordinates (and frame columns) per group */
 #define FFB_NO_STORE 0xFFFFu
+#define FFB_ENTRY_BLOCK 8          /* entries a thread loads together in the sparse phase */
 
 struct FfbPlanHeader {
   int32_t magic, version;
@@ -49,16 +51,24 @@ struct FfbPlanHeader {
   int32_t reserved[6];
 };
 
-static inline __host__ __device__ int32_t ffb_phys(int32_t x) {
-  const int32_t g = x >> 5;
-  return (g << 5) | ((((x >> 2) & 7) ^ (g & 7)) << 2) | (x & 3);
+// Slot of group-major index x (x < K) in a tile buffer.  Slots come in
+// pairs (x even, x + 1); the 16 pairs of a group are permuted so that the
+// MMA epilogue and prologue -- lane (g, t) touching pairs 4t..4t+3 of group
+// G0 + g, g = 0..7 -- spread every quarter-warp over distinct banks:
+//     pair p of group r -> pair p ^ (((p >> 3) & 1) << 1) ^ (r & 1).
+// Overflow slots (x >= K) are used as they are.
+static inline __host__ __device__ int32_t ffb_slot(int32_t x, int32_t K) {
+  if (x >= K) return x;
+  const int32_t r = x >> 5, p = (x >> 1) & 15;
+  const int32_t pp = p ^ (((p >> 3) & 1) << 1) ^ (r & 1);
+  return (r << 5) | (pp << 1) | (x & 1);
 }
 
 // Shared-memory layout of one tile of T tokens (floats).  MODE bits:
 // 1 = forward (Y), 2 = backward dX, 4 = coefficient gradient.  V = X Phi_in
 // rows (n), U = dY Phi_out rows (m), RZ = coefficient-SpMM row sums for Y
 // (m + ovfZ), RG = the same for dX (n + ovfG); DC = per-thread dC
-// accumulators when the chunks do not fit in registers.
+// accumulators ([entry][thread]).
 struct FfbTileLayout {
   int32_t sV, sU, sRZ, sRG;      // token-row strides
   int32_t oV, oU, oRZ, oRG, oDC; // region offsets
@@ -78,6 +88,8 @@ static inline __host__ __device__ FfbTileLayout ffb_tile_layout(const FfbPlanHea
   L.oRZ = L.oU + ((bdx || gc) ? T * L.sU : 0);
   L.oRG = L.oRZ + (fwd ? T * L.sRZ : 0);
   L.oDC = L.oRG + (bdx ? T * L.sRG : 0);
-  L.total = L.oDC + ((gc && dc_in_smem) ? h.EG * h.P : 0);
+  // whole blocks of entries: padding entries of the last block are updated too
+  const int32_t eg = (h.EG + FFB_ENTRY_BLOCK - 1) / FFB_ENTRY_BLOCK * FFB_ENTRY_BLOCK;
+  L.total = L.oDC + ((gc && dc_in_smem) ? eg * h.P : 0);
   return L;
 }

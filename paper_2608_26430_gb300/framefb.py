@@ -27,6 +27,7 @@ EXPORTED = [
     "framefb_support_build", "framefb_plan_build", "framefb_plan_bytes", "framefb_plan_data", "framefb_plan_free",
     "framefb_workspace_size", "framefb_run", "framefb_forward", "framefb_backward_dx", "framefb_grad_coeff",
     "framefb_backward", "framefb_fused_fwd_bwd", "framefb_merge", "framefb_run_static_ws",
+    "framefb_wait_timeouts",
 ]
 STATIC_WS_BYTES = 8 << 20
 
@@ -107,6 +108,8 @@ def lib() -> ct.CDLL:
             f.argtypes = [ct.POINTER(framefb_mat), i32, i32, vp, sz, vp]
         L.framefb_run_static_ws.restype = i32
         L.framefb_run_static_ws.argtypes = [ct.POINTER(framefb_mat), i32, i32, i32, vp]
+        L.framefb_wait_timeouts.restype = i32
+        L.framefb_wait_timeouts.argtypes = [ct.POINTER(ct.c_uint32)]
         L.framefb_merge.restype = i32
         L.framefb_merge.argtypes = [vp, i32, i32, i32, i64, ct.POINTER(framefb_dev_frame),
                                     ct.POINTER(framefb_dev_frame), vp, vp, vp, i32, ct.c_float, vp, vp]
@@ -323,6 +326,12 @@ def framefb_merge(W0, fin: DevFrame, fout: DevFrame, plan: Plan, plan_dev, c_val
     _check(lib().framefb_merge(_ptr(W0), _dtype_code(W0), m, n, W0.stride(0), ct.byref(fin.struct),
                                ct.byref(fout.struct), plan.handle.value, _ptr(plan_dev), _ptr(c_vals), T,
                                float(scale), _ptr(Wout), _stream(stream)), "framefb_merge")
+
+
+def framefb_wait_timeouts() -> int:
+    n = ct.c_uint32(0)
+    _check(lib().framefb_wait_timeouts(ct.byref(n)), "framefb_wait_timeouts")
+    return int(n.value)
 
 
 def exported_symbols(names: Iterable[str] = EXPORTED) -> dict:

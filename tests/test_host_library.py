@@ -134,10 +134,27 @@ def group_major(c, rho):
     return 32 * (rr // 2) + 2 * i + (rr & 1)
 
 
-def phys(x):
+def slot(x, K):
+    """Tile-buffer slot of group-major index x (the map documented in plan_layout.h)."""
     x = np.asarray(x)
-    g = x >> 5
-    return (g << 5) | ((((x >> 2) & 7) ^ (g & 7)) << 2) | (x & 3)
+    r, p = x >> 5, (x >> 1) & 15
+    pp = p ^ (((p >> 3) & 1) << 1) ^ (r & 1)
+    return np.where(x >= K, x, (r << 5) | (pp << 1) | (x & 1))
+
+
+def test_slot_map_is_a_pair_preserving_bijection_and_bank_spread():
+    K = 4096
+    s = slot(np.arange(K), K)
+    assert sorted(s.tolist()) == list(range(K))
+    assert np.all(s >> 5 == np.arange(K) >> 5)            # stays inside its group
+    assert np.all((s[0::2] ^ 1) == s[1::2])               # pairs stay adjacent, even first
+    # the MMA prologue / epilogue: lane (g, t) touches pair 4t + k of group G0 + g;
+    # a quarter-warp (g in {0, 1}, t in 0..3) must hit 8 distinct 16-byte bank groups
+    # in the two-token layout (one 16-byte chunk per pair)
+    for G0 in range(0, 64, 2):
+        for k in range(4):
+            chunks = [(slot(32 * (G0 + g) + 2 * (4 * t + k), K) >> 1) % 8 for g in (0, 1) for t in range(4)]
+            assert len(set(chunks)) == 8
 
 
 PLAN_CASES = [(256, 256, 128, 0), (768, 768, 1000, 0), (768, 3072, 2000, 0), (4096, 1024, 8192, 1),
@@ -171,8 +188,7 @@ def test_plan_replays_coefficient_products(n, m, nnz, mode):
     c = rng.standard_normal(nnz)
     Vint = rng.standard_normal((Tn, n))
     Uint = rng.standard_normal((Tn, m))
-    Vs = np.zeros((Tn, n)); Vs[:, phys(np.arange(n))] = Vint
-    Us = np.zeros((Tn, m)); Us[:, phys(np.arange(m))] = Uint
+    Vs, Us = Vint, Uint                  # the tables hold group-major indices
     RZ = np.zeros((Tn, m + h["ovfZ"]))
     RG = np.zeros((Tn, n + h["ovfG"]))
     dC = np.zeros(nnz)
@@ -200,8 +216,8 @@ def test_plan_replays_coefficient_products(n, m, nnz, mode):
         RZ[:, dst] += RZ[:, src:src + cnt].sum(axis=1)
     for dst, src, cnt, _ in t["fixG"]:
         RG[:, dst] += RG[:, src:src + cnt].sum(axis=1)
-    Z = RZ[:, phys(np.arange(m))]
-    G = RG[:, phys(np.arange(n))]
+    Z = RZ[:, :m]
+    G = RG[:, :n]
     Cint = adapter.dense_C(m, n, a_int, b_int, c)
     np.testing.assert_allclose(Z, Vint @ Cint.T, atol=1e-12)
     np.testing.assert_allclose(G, Uint @ Cint, atol=1e-12)
