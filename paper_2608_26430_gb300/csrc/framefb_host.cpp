@@ -438,7 +438,7 @@ extern "C" framefb_status framefb_plan_build(const framefb_frame* fin, const fra
         const int32_t idx = p * EZ + e;
         const size_t slot = static_cast<size_t>(e) * P + p;
         if (idx < nz) {
-          zb[slot] = byrow[idx].key1 | (storeZ[idx] << 16);
+          zb[slot] = byrow[idx].key1 | ((byrow[idx].key0 & 1) << 15) | (storeZ[idx] << 16);
           zq[slot] = byrow[idx].q;
         } else {
           zb[slot] = (FFB_NO_STORE << 16);
@@ -449,7 +449,7 @@ extern "C" framefb_status framefb_plan_build(const framefb_frame* fin, const fra
         const int32_t idx = p * EG + e;
         const size_t slot = static_cast<size_t>(e) * P + p;
         if (idx < nz) {
-          ga[slot] = bycol[idx].key1 | (storeG[idx] << 16);
+          ga[slot] = bycol[idx].key1 | ((bycol[idx].key0 & 1) << 15) | (storeG[idx] << 16);
           gb[slot] = bycol[idx].key0;
           gq[slot] = bycol[idx].q;
         } else {

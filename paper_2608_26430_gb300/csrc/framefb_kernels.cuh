@@ -304,7 +304,10 @@ struct Vecs<2, true> {
   static __device__ __forceinline__ float dot(const float2& a, const float2& b) { return fmaf(a.x, b.x, a.y * b.y); }
 };
 
-template <int MODE, bool REG>
+// FLIP: fold the sign pattern S = diag(+1, -1, +1, ...) of the row / column
+// index into the coefficient values (the tensor-core synthesis reuses the
+// analysis block through D^T = S D S, so it wants S Z and S G).
+template <int MODE, bool REG, bool FLIP = false>
 struct Chunk {
   static constexpr bool F = MODE & MODE_F, D = MODE & MODE_D, C = MODE & MODE_C;
   static constexpr int E = REG ? kEreg : 1;
@@ -314,9 +317,14 @@ struct Chunk {
   float zc[E], gc[E];
   int EZ, EG, n, m;
 
-  // plan word (index | target << 16) -> (slot | slot << 16)
+  // coefficient value with the parity sign of plan word w (bit 15) folded in
+  static __device__ __forceinline__ float signed_c(float c, uint32_t w) {
+    return (FLIP && (w & 0x8000u)) ? -c : c;
+  }
+
+  // plan word (index | parity << 15 | target << 16) -> (slot | slot << 16)
   static __device__ __forceinline__ uint32_t slots(uint32_t w, int Klo, int Khi) {
-    const uint32_t lo = w & 0xFFFFu, hi = w >> 16;
+    const uint32_t lo = w & 0x7FFFu, hi = w >> 16;
     const uint32_t slo = static_cast<uint32_t>(ffb_slot(static_cast<int32_t>(lo), Klo));
     const uint32_t shi = hi == FFB_NO_STORE ? FFB_NO_STORE : static_cast<uint32_t>(ffb_slot(static_cast<int32_t>(hi), Khi));
     return slo | (shi << 16);
@@ -344,15 +352,17 @@ struct Chunk {
 #pragma unroll
       for (int e = 0; e < E; ++e) {
         if (F && e < EZ) {
-          zb[e] = slots(static_cast<uint32_t>(__ldg(tzb + e * kThreads + tid)), n, m);
+          const uint32_t w = static_cast<uint32_t>(__ldg(tzb + e * kThreads + tid));
+          zb[e] = slots(w, n, m);
           const int32_t q = __ldg(tzq + e * kThreads + tid);
-          zc[e] = q >= 0 ? __ldg(c_val + q) : 0.f;
+          zc[e] = q >= 0 ? signed_c(__ldg(c_val + q), w) : 0.f;
         }
         if ((D || C) && e < EG) {
-          ga[e] = slots(static_cast<uint32_t>(__ldg(tga + e * kThreads + tid)), m, n);
+          const uint32_t w = static_cast<uint32_t>(__ldg(tga + e * kThreads + tid));
+          ga[e] = slots(w, m, n);
           gb[e] = static_cast<uint32_t>(ffb_slot(__ldg(tgb + e * kThreads + tid), n));
           const int32_t q = __ldg(tgq + e * kThreads + tid);
-          gc[e] = (D && q >= 0) ? __ldg(c_val + q) : 0.f;
+          gc[e] = (D && q >= 0) ? signed_c(__ldg(c_val + q), w) : 0.f;
         }
       }
     }
@@ -369,9 +379,10 @@ struct Chunk {
       w = zb[e];
       c = zc[e];
     } else {
-      w = slots(static_cast<uint32_t>(__ldg(table<int32_t>(plan, hdr(plan).off_zb) + e * kThreads + tid)), n, m);
+      const uint32_t raw = static_cast<uint32_t>(__ldg(table<int32_t>(plan, hdr(plan).off_zb) + e * kThreads + tid));
+      w = slots(raw, n, m);
       const int32_t q = __ldg(table<int32_t>(plan, hdr(plan).off_zq) + e * kThreads + tid);
-      c = q >= 0 ? __ldg(c_val + q) : 0.f;
+      c = q >= 0 ? signed_c(__ldg(c_val + q), raw) : 0.f;
     }
   }
   __device__ __forceinline__ void g_entry(const uint8_t* plan, const float* c_val, int tid, int e, uint32_t& wa,
@@ -384,12 +395,13 @@ struct Chunk {
       wb = gb[e];
       c = gc[e];
     } else {
-      wa = slots(static_cast<uint32_t>(__ldg(table<int32_t>(plan, hdr(plan).off_ga) + e * kThreads + tid)), m, n);
+      const uint32_t raw = static_cast<uint32_t>(__ldg(table<int32_t>(plan, hdr(plan).off_ga) + e * kThreads + tid));
+      wa = slots(raw, m, n);
       wb = static_cast<uint32_t>(ffb_slot(__ldg(table<int32_t>(plan, hdr(plan).off_gb) + e * kThreads + tid), n));
       c = 0.f;
       if constexpr (D) {
         const int32_t q = __ldg(table<int32_t>(plan, hdr(plan).off_gq) + e * kThreads + tid);
-        c = q >= 0 ? __ldg(c_val + q) : 0.f;
+        c = q >= 0 ? signed_c(__ldg(c_val + q), raw) : 0.f;
       }
     }
   }

@@ -7,14 +7,17 @@
 // DFT_16 / 4, Sec. 3.2 construction) applied to every (token, group) row:
 //     analysis   V_row = X_row D          (per group of Phi_in, U likewise with Phi_out)
 //     synthesis  dY_row = Z_row D^T       (Z = coefficient-SpMM row sums)
-// Each is a [rows x 32] x [32 x 32] contraction, run with warp-level MMA:
-// data rows are the M side (16 rows per instruction group), D the N side,
-// held as per-lane fragments for the whole matrix.  Analysis multiplies the
-// exact bf16 inputs by D split into bf16 hi + lo (error ~2^-16); synthesis
-// multiplies the fp32 row sums by D in tf32.  Coordinates and coefficient
-// slots are permuted so that every lane reads or writes 16 contiguous bytes
-// of a row: 8 consecutive coordinates 8t..8t+7 (lane t = lane % 4) for rows
-// g and g + 8 (g = lane / 4) of the 16-row block.
+// Each is a [rows x 32] x [32 x 32] contraction, run with warp-level tf32
+// MMA: data rows are the M side (16 rows per instruction group), D the N
+// side, held as per-lane fragments for the whole matrix.  The DFT_16 matrix
+// is symmetric, so its realified block satisfies D^T = S D S exactly, with
+// S = diag(+1, -1, +1, -1, ...): synthesis runs on the same fragments as
+// analysis, from S Z (the sign folded into the coefficient values) and with
+// S applied to the result (the sign folded into the output scale).  bf16
+// inputs are exact in tf32; D and the fp32 row sums are rounded to tf32.
+// Index slots are permuted so that every lane reads or writes 16 contiguous
+// bytes of a row: 8 consecutive indices 8t..8t+7 (t = lane % 4) for rows g
+// and g + 8 (g = lane / 4) of the 16-row block.
 #pragma once
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -108,31 +111,21 @@ __device__ __forceinline__ int an_coord(int k) { return 8 * ((k & 7) >> 1) + 4 *
 __device__ __forceinline__ int nslot_pos(int n) { return 8 * ((n & 7) >> 1) + 2 * (n >> 3) + (n & 1); }
 __device__ __forceinline__ int sy_coef(int k) { return 8 * (k & 3) + 2 * (k >> 3) + ((k >> 2) & 1); }
 
+// B fragments of D (tf32) for m16n8k8: N-tile j, k-step s.  K slot
+// 8s + 4h + t <-> row index 8t + 2s + h of D (sy_coef); N slot 8j + 2t + e
+// <-> column index 8t + 2j + e (nslot_pos).
 struct DFrags {
-  uint32_t an_hi[4][2][2], an_lo[4][2][2];  // analysis B fragments [n-tile][k-step][reg]
-  uint32_t sy[4][4][2];                     // synthesis B fragments [n-tile][k-step][reg]
+  uint32_t b[4][4][2];
 
   __device__ __forceinline__ void load(const float* val, int rho, int lane) {
     const int g = lane >> 2, t = lane & 3;
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
-      const int x = nslot_pos(8 * j + g);  // coefficient of this lane's B column (analysis)
-#pragma unroll
-      for (int s = 0; s < 2; ++s) {
-#pragma unroll
-        for (int r = 0; r < 2; ++r) {
-          const int k0 = 16 * s + 8 * r + 2 * t;
-          const float v0 = d4(val, rho, an_coord(k0), x), v1 = d4(val, rho, an_coord(k0 + 1), x);
-          const __nv_bfloat16 h0 = __float2bfloat16_rn(v0), h1 = __float2bfloat16_rn(v1);
-          an_hi[j][s][r] = pack_bf16(__bfloat162float(h0), __bfloat162float(h1));
-          an_lo[j][s][r] = pack_bf16(v0 - __bfloat162float(h0), v1 - __bfloat162float(h1));
-        }
-      }
-      const int w = nslot_pos(8 * j + g);  // coordinate of this lane's B column (synthesis)
+      const int x = nslot_pos(8 * j + g);
 #pragma unroll
       for (int s = 0; s < 4; ++s) {
-        sy[j][s][0] = to_tf32(d4(val, rho, w, sy_coef(8 * s + t)));
-        sy[j][s][1] = to_tf32(d4(val, rho, w, sy_coef(8 * s + t + 4)));
+        b[j][s][0] = to_tf32(d4(val, rho, sy_coef(8 * s + t), x));
+        b[j][s][1] = to_tf32(d4(val, rho, sy_coef(8 * s + t + 4), x));
       }
     }
   }
@@ -143,138 +136,194 @@ __device__ __forceinline__ int pair_slot(int p, int r) { return p ^ (((p >> 3) &
 
 __device__ __forceinline__ uint4 lds128(const uint8_t* p) { return *reinterpret_cast<const uint4*>(p); }
 
-// y += seff * d for 8 bf16 values (one 16-byte chunk), returns the new chunk.
-__device__ __forceinline__ uint4 axpy_bf16x8(uint4 y, const float (&d)[8], float seff) {
+// y += seff * S d for 8 bf16 values (one 16-byte chunk of 8 consecutive
+// coordinates starting at an even one), returns the new chunk.
+__device__ __forceinline__ uint4 axpy_sd_bf16x8(uint4 y, const float (&d)[8], float seff) {
   uint32_t w[4] = {y.x, y.y, y.z, y.w};
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
     const float lo = fmaf(seff, d[2 * i], __uint_as_float(w[i] << 16));
-    const float hi = fmaf(seff, d[2 * i + 1], __uint_as_float(w[i] & 0xFFFF0000u));
+    const float hi = fmaf(-seff, d[2 * i + 1], __uint_as_float(w[i] & 0xFFFF0000u));
     w[i] = pack_bf16(lo, hi);
   }
   return make_uint4(w[0], w[1], w[2], w[3]);
 }
 
-// Analysis of one 16-row MMA block into V (or U).  T = 2: rows g and g + 8
-// of the block are tokens 0 and 1 of group 8b + g, and the fp32 buffer is
-// token-minor (float2 per slot); T = 1: rows g and g + 8 are groups 16b + g
-// and 16b + g + 8 of the single token.  src = staged bf16 token rows (stride
-// rs bytes), Tc = tokens present.
+__device__ __forceinline__ uint32_t word_of(const uint4& w, int s) {
+  return s == 0 ? w.x : s == 1 ? w.y : s == 2 ? w.z : w.w;
+}
+
+// One 16-row MMA block.  T = 2: rows g and g + 8 of block b are tokens 0 and
+// 1 of group 8b + g, and the fp32 buffer is token-minor (float2 per slot);
+// T = 1: rows g and g + 8 are groups 16b + g and 16b + g + 8 of the single
+// token.
+struct Blk {
+  const uint8_t* stg;  // staged bf16 token rows (stride rs bytes), or NULL
+  float* buf;          // fp32 slot buffer (V / U written, RZ / RG read)
+  __nv_bfloat16* out;  // synthesis: global output rows
+  const uint32_t* mask;
+  int64_t ld;
+  int rs, G, b;
+};
+
 template <int T>
-__device__ __forceinline__ void analysis_block(const DFrags& Df, const uint8_t* src, int rs, float* dst, int G, int b,
-                                               int Tc, int lane) {
-  const int g = lane >> 2, t = lane & 3;
-  const int grp0 = T == 2 ? 8 * b + g : 16 * b + g;
-  const int grp1 = T == 2 ? grp0 : grp0 + 8;
-  const bool v0 = grp0 < G, v1 = T == 2 ? (v0 && Tc > 1) : grp1 < G;
-  const uint4 w0 = v0 ? lds128(src + grp0 * 64 + t * 16) : make_uint4(0, 0, 0, 0);
-  const uint4 w1 = v1 ? lds128(src + (T == 2 ? rs : 0) + grp1 * 64 + t * 16) : make_uint4(0, 0, 0, 0);
-  float c[4][4];
+__device__ __forceinline__ void blk_rows(const Blk& k, int Tc, int lane, int& grp0, int& grp1, bool& v0, bool& v1,
+                                         bool masked) {
+  const int g = lane >> 2;
+  grp0 = T == 2 ? 8 * k.b + g : 16 * k.b + g;
+  grp1 = T == 2 ? grp0 : grp0 + 8;
+  v0 = grp0 < k.G && (!masked || k.mask[grp0] != 0u);
+  v1 = T == 2 ? (v0 && Tc > 1) : (grp1 < k.G && (!masked || k.mask[grp1] != 0u));
+}
+
+// Analysis of NB blocks into V (or U): K slot 8s + 4h + t reads coordinate
+// 8t + 2s + h, i.e. half h of bf16 word s of the lane's 16-byte chunk (a bf16
+// value is exact as tf32); N slot 8j + 2t + e writes coefficient 8t + 2j + e.
+// Tc = tokens present.
+template <int T, int NB>
+__device__ __forceinline__ void analysis_blocks(const DFrags& Df, const Blk (&k)[NB], int Tc, int lane) {
+  const int t = lane & 3;
+  int grp0[NB], grp1[NB];
+  bool v0[NB], v1[NB];
+  uint4 w0[NB], w1[NB];
 #pragma unroll
-  for (int j = 0; j < 4; ++j) c[j][0] = c[j][1] = c[j][2] = c[j][3] = 0.f;
+  for (int i = 0; i < NB; ++i) {
+    blk_rows<T>(k[i], Tc, lane, grp0[i], grp1[i], v0[i], v1[i], false);
+    w0[i] = v0[i] ? lds128(k[i].stg + grp0[i] * 64 + t * 16) : make_uint4(0, 0, 0, 0);
+    w1[i] = v1[i] ? lds128(k[i].stg + (T == 2 ? k[i].rs : 0) + grp1[i] * 64 + t * 16) : make_uint4(0, 0, 0, 0);
+  }
+  float c[NB][4][4];
 #pragma unroll
-  for (int s = 0; s < 2; ++s) {
-    const uint32_t a0 = s ? w0.z : w0.x, a1 = s ? w1.z : w1.x;
-    const uint32_t a2 = s ? w0.w : w0.y, a3 = s ? w1.w : w1.y;
+  for (int i = 0; i < NB; ++i)
 #pragma unroll
-    for (int j = 0; j < 4; ++j) mma_bf16(c[j], a0, a1, a2, a3, Df.an_hi[j][s][0], Df.an_hi[j][s][1]);
+    for (int j = 0; j < 4; ++j) c[i][j][0] = c[i][j][1] = c[i][j][2] = c[i][j][3] = 0.f;
 #pragma unroll
-    for (int j = 0; j < 4; ++j) mma_bf16(c[j], a0, a1, a2, a3, Df.an_lo[j][s][0], Df.an_lo[j][s][1]);
+  for (int s = 0; s < 4; ++s) {
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+#pragma unroll
+      for (int i = 0; i < NB; ++i) {
+        const uint32_t x0 = word_of(w0[i], s), x1 = word_of(w1[i], s);
+        mma_tf32(c[i][j], x0 << 16, x1 << 16, x0 & 0xFFFF0000u, x1 & 0xFFFF0000u, Df.b[j][s][0], Df.b[j][s][1]);
+      }
   }
   // row g holds coefficients 8t + 2j + e in c[j][e], row g + 8 in c[j][2 + e]
-  if constexpr (T == 2) {
-    if (v0) {
-      float* grow = dst + 64 * grp0;
 #pragma unroll
-      for (int j = 0; j < 4; ++j)  // pair 4t + j: (x, tok0), (x, tok1), (x + 1, tok0), (x + 1, tok1)
-        *reinterpret_cast<float4*>(grow + 4 * pair_slot(4 * t + j, grp0)) =
-            make_float4(c[j][0], c[j][2], c[j][1], c[j][3]);
-    }
-  } else {
+  for (int i = 0; i < NB; ++i) {
+    if constexpr (T == 2) {
+      if (v0[i]) {
+        float* grow = k[i].buf + 64 * grp0[i];
 #pragma unroll
-    for (int r = 0; r < 2; ++r) {
-      const int grp = r ? grp1 : grp0;
-      if (r ? v1 : v0) {
-        float* grow = dst + 32 * grp;
-        const int o = 2 * r;
+        for (int j = 0; j < 4; ++j)  // pair 4t + j: (x, tok0), (x, tok1), (x + 1, tok0), (x + 1, tok1)
+          *reinterpret_cast<float4*>(grow + 4 * pair_slot(4 * t + j, grp0[i])) =
+              make_float4(c[i][j][0], c[i][j][2], c[i][j][1], c[i][j][3]);
+      }
+    } else {
 #pragma unroll
-        for (int k = 0; k < 2; ++k) {  // float4 chunk q = 2t + k holds pairs 2q, 2q + 1
-          const int q = 2 * t + k;
-          const float4 lo = make_float4(c[2 * k][o], c[2 * k][o + 1], c[2 * k + 1][o], c[2 * k + 1][o + 1]);
-          const float4 v = (grp & 1) ? make_float4(lo.z, lo.w, lo.x, lo.y) : lo;
-          *reinterpret_cast<float4*>(grow + 4 * (q ^ ((q >> 2) & 1))) = v;
+      for (int r = 0; r < 2; ++r) {
+        const int grp = r ? grp1[i] : grp0[i];
+        if (r ? v1[i] : v0[i]) {
+          float* grow = k[i].buf + 32 * grp;
+          const int o = 2 * r;
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {  // float4 chunk q = 2t + h holds pairs 2q, 2q + 1
+            const int q = 2 * t + h;
+            const float4 lo =
+                make_float4(c[i][2 * h][o], c[i][2 * h][o + 1], c[i][2 * h + 1][o], c[i][2 * h + 1][o + 1]);
+            const float4 v = (grp & 1) ? make_float4(lo.z, lo.w, lo.x, lo.y) : lo;
+            *reinterpret_cast<float4*>(grow + 4 * (q ^ ((q >> 2) & 1))) = v;
+          }
         }
       }
     }
   }
 }
 
-// Synthesis of one 16-row block: Z from the fp32 buffer (same layout as the
-// analysis output), the output rows from staging (stg, stride rs bytes) or,
-// when stg is NULL, from global memory; y += seff * (Z D^T) written to the
-// global rows out + (t0 + token) * ld.  Groups whose mask is zero have no
-// support entries and are left untouched.
-template <int T>
-__device__ __forceinline__ void synthesis_block(const DFrags& Df, const float* zsrc, const uint8_t* stg, int rs,
-                                                __nv_bfloat16* out, int64_t ld, int64_t t0, int G, int b, int Tc,
-                                                const uint32_t* mask, float seff, int lane) {
-  const int g = lane >> 2, t = lane & 3;
-  const int grp0 = T == 2 ? 8 * b + g : 16 * b + g;
-  const int grp1 = T == 2 ? grp0 : grp0 + 8;
-  const bool v0 = grp0 < G && mask[grp0] != 0u;
-  const bool v1 = T == 2 ? (v0 && Tc > 1) : (grp1 < G && mask[grp1] != 0u);
+// Synthesis of NB blocks: S Z (the row sums, with the sign pattern S folded
+// into the coefficient values) from the fp32 buffer in the analysis layout,
+// the output rows from staging or, when stg is NULL, from global memory;
+// y += seff * S (S Z) D^T-fragments = seff * Z D^T, written to the global rows
+// out + (t0 + token) * ld.  K slot 8s + 4h + t reads coefficient 8t + 2s + h;
+// N slot 8j + 2t + e writes coordinate 8t + 2j + e.  Groups whose mask is
+// zero have no support entries and are left untouched.
+template <int T, int NB>
+__device__ __forceinline__ void synthesis_blocks(const DFrags& Df, const Blk (&k)[NB], int64_t t0, int Tc, float seff,
+                                                 int lane) {
+  const int t = lane & 3;
+  int grp0[NB], grp1[NB];
+  bool v0[NB], v1[NB];
   // A fragment of k-step s: (row g, coef 8t + 2s), (row g + 8, same), (row g, +1), (row g + 8, +1)
-  float4 a[4];
-  if constexpr (T == 2) {
-    const float* grow = zsrc + 64 * grp0;
+  float4 a[NB][4];
 #pragma unroll
-    for (int s = 0; s < 4; ++s)
-      a[s] = v0 ? *reinterpret_cast<const float4*>(grow + 4 * pair_slot(4 * t + s, grp0)) : make_float4(0.f, 0.f, 0.f, 0.f);
-  } else {
-    float z[2][8];
+  for (int i = 0; i < NB; ++i) {
+    blk_rows<T>(k[i], Tc, lane, grp0[i], grp1[i], v0[i], v1[i], true);
+    if constexpr (T == 2) {
+      const float* grow = k[i].buf + 64 * grp0[i];
 #pragma unroll
-    for (int r = 0; r < 2; ++r) {
-      const int grp = r ? grp1 : grp0;
-      const bool v = r ? v1 : v0;
+      for (int s = 0; s < 4; ++s)
+        a[i][s] = v0[i] ? *reinterpret_cast<const float4*>(grow + 4 * pair_slot(4 * t + s, grp0[i]))
+                        : make_float4(0.f, 0.f, 0.f, 0.f);
+    } else {
+      float z[2][8];
 #pragma unroll
-      for (int k = 0; k < 2; ++k) {
-        const int q = 2 * t + k;
-        float4 f = v ? *reinterpret_cast<const float4*>(zsrc + 32 * grp + 4 * (q ^ ((q >> 2) & 1)))
-                     : make_float4(0.f, 0.f, 0.f, 0.f);
-        if (grp & 1) f = make_float4(f.z, f.w, f.x, f.y);
-        z[r][4 * k] = f.x;
-        z[r][4 * k + 1] = f.y;
-        z[r][4 * k + 2] = f.z;
-        z[r][4 * k + 3] = f.w;
+      for (int r = 0; r < 2; ++r) {
+        const int grp = r ? grp1[i] : grp0[i];
+        const bool v = r ? v1[i] : v0[i];
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          const int q = 2 * t + h;
+          float4 f = v ? *reinterpret_cast<const float4*>(k[i].buf + 32 * grp + 4 * (q ^ ((q >> 2) & 1)))
+                       : make_float4(0.f, 0.f, 0.f, 0.f);
+          if (grp & 1) f = make_float4(f.z, f.w, f.x, f.y);
+          z[r][4 * h] = f.x;
+          z[r][4 * h + 1] = f.y;
+          z[r][4 * h + 2] = f.z;
+          z[r][4 * h + 3] = f.w;
+        }
       }
+#pragma unroll
+      for (int s = 0; s < 4; ++s) a[i][s] = make_float4(z[0][2 * s], z[1][2 * s], z[0][2 * s + 1], z[1][2 * s + 1]);
     }
-#pragma unroll
-    for (int s = 0; s < 4; ++s) a[s] = make_float4(z[0][2 * s], z[1][2 * s], z[0][2 * s + 1], z[1][2 * s + 1]);
   }
-  uint4 y0 = make_uint4(0, 0, 0, 0), y1 = y0;
-  const int64_t row0 = t0, row1 = T == 2 ? t0 + 1 : t0;
-  if (v0) y0 = stg ? lds128(stg + grp0 * 64 + t * 16) : *reinterpret_cast<const uint4*>(out + row0 * ld + 32 * grp0 + 8 * t);
-  if (v1)
-    y1 = stg ? lds128(stg + (T == 2 ? rs : 0) + grp1 * 64 + t * 16)
-             : *reinterpret_cast<const uint4*>(out + row1 * ld + 32 * grp1 + 8 * t);
-  float c[4][4];
+  uint4 y0[NB], y1[NB];
 #pragma unroll
-  for (int j = 0; j < 4; ++j) c[j][0] = c[j][1] = c[j][2] = c[j][3] = 0.f;
+  for (int i = 0; i < NB; ++i) {
+    const int64_t row0 = t0, row1 = T == 2 ? t0 + 1 : t0;
+    y0[i] = y1[i] = make_uint4(0, 0, 0, 0);
+    if (v0[i])
+      y0[i] = k[i].stg ? lds128(k[i].stg + grp0[i] * 64 + t * 16)
+                       : *reinterpret_cast<const uint4*>(k[i].out + row0 * k[i].ld + 32 * grp0[i] + 8 * t);
+    if (v1[i])
+      y1[i] = k[i].stg ? lds128(k[i].stg + (T == 2 ? k[i].rs : 0) + grp1[i] * 64 + t * 16)
+                       : *reinterpret_cast<const uint4*>(k[i].out + row1 * k[i].ld + 32 * grp1[i] + 8 * t);
+  }
+  float c[NB][4][4];
+#pragma unroll
+  for (int i = 0; i < NB; ++i)
+#pragma unroll
+    for (int j = 0; j < 4; ++j) c[i][j][0] = c[i][j][1] = c[i][j][2] = c[i][j][3] = 0.f;
 #pragma unroll
   for (int s = 0; s < 4; ++s) {
 #pragma unroll
     for (int j = 0; j < 4; ++j)
-      mma_tf32(c[j], __float_as_uint(a[s].x), __float_as_uint(a[s].y), __float_as_uint(a[s].z),
-               __float_as_uint(a[s].w), Df.sy[j][s][0], Df.sy[j][s][1]);
+#pragma unroll
+      for (int i = 0; i < NB; ++i)
+        mma_tf32(c[i][j], __float_as_uint(a[i][s].x), __float_as_uint(a[i][s].y), __float_as_uint(a[i][s].z),
+                 __float_as_uint(a[i][s].w),
+                 Df.b[j][s][0], Df.b[j][s][1]);
   }
   // N slot 8j + 2t + e holds coordinate 8t + 2j + e
-  if (v0) {
-    const float d[8] = {c[0][0], c[0][1], c[1][0], c[1][1], c[2][0], c[2][1], c[3][0], c[3][1]};
-    *reinterpret_cast<uint4*>(out + row0 * ld + 32 * grp0 + 8 * t) = axpy_bf16x8(y0, d, seff);
-  }
-  if (v1) {
-    const float d[8] = {c[0][2], c[0][3], c[1][2], c[1][3], c[2][2], c[2][3], c[3][2], c[3][3]};
-    *reinterpret_cast<uint4*>(out + row1 * ld + 32 * grp1 + 8 * t) = axpy_bf16x8(y1, d, seff);
+#pragma unroll
+  for (int i = 0; i < NB; ++i) {
+    const int64_t row0 = t0, row1 = T == 2 ? t0 + 1 : t0;
+    if (v0[i]) {
+      const float d[8] = {c[i][0][0], c[i][0][1], c[i][1][0], c[i][1][1], c[i][2][0], c[i][2][1], c[i][3][0], c[i][3][1]};
+      *reinterpret_cast<uint4*>(k[i].out + row0 * k[i].ld + 32 * grp0[i] + 8 * t) = axpy_sd_bf16x8(y0[i], d, seff);
+    }
+    if (v1[i]) {
+      const float d[8] = {c[i][0][2], c[i][0][3], c[i][1][2], c[i][1][3], c[i][2][2], c[i][2][3], c[i][3][2], c[i][3][3]};
+      *reinterpret_cast<uint4*>(k[i].out + row1 * k[i].ld + 32 * grp1[i] + 8 * t) = axpy_sd_bf16x8(y1[i], d, seff);
+    }
   }
 }
 
@@ -374,7 +423,7 @@ __global__ void __launch_bounds__(kThreads, 1) mma_tile_kernel(const __grid_cons
   uint32_t ph_in = 0, ph_out = 0;
   int jn = j;  // matrix of the next unit to stage (warp 0)
 
-  Chunk<MODE, REG> ch;
+  Chunk<MODE, REG, true> ch;
   DFrags Df;
   int cur = -1;
   const uint8_t* plan = nullptr;
@@ -417,11 +466,24 @@ __global__ void __launch_bounds__(kThreads, 1) mma_tile_kernel(const __grid_cons
       const uint8_t* xs = smem + args.stg_in;
       const uint8_t* dys = smem + args.stg_in + (NEED_V ? T * rx : 0);
       const int bV = NEED_V ? (Gn + GB - 1) / GB : 0, bU = NEED_U ? (Gm + GB - 1) / GB : 0;
-      for (int b = warp; b < bV + bU; b += kThreads / 32) {
-        if (b < bV)
-          analysis_block<T>(Df, xs, rx, fsm + L.oV, Gn, b, Tc, lane);
-        else
-          analysis_block<T>(Df, dys, ry, fsm + L.oU, Gm, b - bV, Tc, lane);
+      auto blk = [&](int b) {
+        Blk k{};
+        if (b < bV) {
+          k.stg = xs, k.rs = rx, k.buf = fsm + L.oV, k.G = Gn, k.b = b;
+        } else {
+          k.stg = dys, k.rs = ry, k.buf = fsm + L.oU, k.G = Gm, k.b = b - bV;
+        }
+        return k;
+      };
+      constexpr int W = kThreads / 32;
+      int b = warp;
+      for (; b + W < bV + bU; b += 2 * W) {
+        const Blk k[2] = {blk(b), blk(b + W)};
+        analysis_blocks<T, 2>(Df, k, Tc, lane);
+      }
+      if (b < bV + bU) {
+        const Blk k[1] = {blk(b)};
+        analysis_blocks<T, 1>(Df, k, Tc, lane);
       }
     }
     __syncthreads();
@@ -460,13 +522,26 @@ __global__ void __launch_bounds__(kThreads, 1) mma_tile_kernel(const __grid_cons
       const uint32_t* zmask = table<uint32_t>(plan, hdr(plan).off_zmask);
       const uint32_t* gmask = table<uint32_t>(plan, hdr(plan).off_gmask);
       const int bY = F ? (Gm + GB - 1) / GB : 0, bX = D ? (Gn + GB - 1) / GB : 0;
-      for (int b = warp; b < bY + bX; b += kThreads / 32) {
-        if (b < bY)
-          synthesis_block<T>(Df, fsm + L.oRZ, ys, ry, static_cast<__nv_bfloat16*>(M.Y), M.ldy, t0, Gm, b, Tc, zmask,
-                             M.seff, lane);
-        else
-          synthesis_block<T>(Df, fsm + L.oRG, dxs, rx, static_cast<__nv_bfloat16*>(M.dX), M.ldx, t0, Gn, b - bY, Tc,
-                             gmask, M.seff, lane);
+      auto blk = [&](int b) {
+        Blk k{};
+        if (b < bY) {
+          k.stg = ys, k.rs = ry, k.buf = fsm + L.oRZ, k.out = static_cast<__nv_bfloat16*>(M.Y), k.ld = M.ldy;
+          k.mask = zmask, k.G = Gm, k.b = b;
+        } else {
+          k.stg = dxs, k.rs = rx, k.buf = fsm + L.oRG, k.out = static_cast<__nv_bfloat16*>(M.dX), k.ld = M.ldx;
+          k.mask = gmask, k.G = Gn, k.b = b - bY;
+        }
+        return k;
+      };
+      constexpr int W = kThreads / 32;
+      int b = warp;
+      for (; b + W < bY + bX; b += 2 * W) {
+        const Blk k[2] = {blk(b), blk(b + W)};
+        synthesis_blocks<T, 2>(Df, k, t0, Tc, M.seff, lane);
+      }
+      if (b < bY + bX) {
+        const Blk k[1] = {blk(b)};
+        synthesis_blocks<T, 1>(Df, k, t0, Tc, M.seff, lane);
       }
       __syncthreads();
       if (warp == 0 && u + 1 < u_end && args.stage_out)

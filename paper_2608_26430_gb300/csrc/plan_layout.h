@@ -41,8 +41,8 @@ struct FfbPlanHeader {
   int32_t EZ, EG;          // chunk length (entries per thread) by row / by column
   int32_t ovfZ, ovfG;      // overflow slots after the m (resp. n) row slots, multiple of 4
   int32_t nfixZ, nfixG;    // fix-up items (rows / columns split between chunks)
-  int32_t off_zb, off_zq;  // [EZ][P]: packed (phys b | store << 16), c index (-1 = padding)
-  int32_t off_ga, off_gb, off_gq;  // [EG][P]: packed (phys a | store << 16), phys b, c index
+  int32_t off_zb, off_zq;  // [EZ][P]: b | parity(a) << 15 | store << 16, c index (-1 = padding)
+  int32_t off_ga, off_gb, off_gq;  // [EG][P]: a | parity(b) << 15 | store << 16, b, c index
   int32_t off_fixZ, off_fixG;      // int4 {dst phys, first overflow slot, count, 0}
   int32_t off_zmask, off_gmask;    // uint32 per group: bit w = row (col) 32g+w is in the support
   int32_t off_blkptr;              // merge: [Gm*Gn + 1] entry ranges of each 32x32 block (g, h)

@@ -197,7 +197,9 @@ def test_plan_replays_coefficient_products(n, m, nnz, mode):
         for e in range(h["EZ"]):
             pk, q = int(t["zb"][e, p]), int(t["zq"][e, p])
             cv = c[q] if q >= 0 else 0.0
-            acc += cv * Vs[:, pk & 0xFFFF]
+            if q >= 0:  # bit 15 carries the parity of the entry's row
+                assert (pk >> 15) & 1 == a_int[q] & 1
+            acc += cv * Vs[:, pk & 0x7FFF]
             if (pk >> 16) != 0xFFFF:
                 RZ[:, pk >> 16] = acc
                 acc = np.zeros(Tn)
@@ -205,7 +207,9 @@ def test_plan_replays_coefficient_products(n, m, nnz, mode):
         for e in range(h["EG"]):
             pa, pb, q = int(t["ga"][e, p]), int(t["gb"][e, p]), int(t["gq"][e, p])
             cv = c[q] if q >= 0 else 0.0
-            uv = Us[:, pa & 0xFFFF]
+            if q >= 0:  # bit 15 carries the parity of the entry's column
+                assert (pa >> 15) & 1 == b_int[q] & 1
+            uv = Us[:, pa & 0x7FFF]
             acc += cv * uv
             if q >= 0:
                 dC[q] += np.dot(uv, Vs[:, pb])
