@@ -5,6 +5,7 @@
 
 #include <algorithm>
 #include <cmath>
+#include <cstdlib>
 #include <cstring>
 #include <mutex>
 #include <vector>
@@ -12,6 +13,7 @@
 #include "framefb.h"
 #include "framefb_kernels.cuh"
 #include "framefb_mma.cuh"
+#include "framefb_pipe.cuh"
 #include "plan_internal.h"
 #include "plan_layout.h"
 
@@ -45,8 +47,20 @@ struct Prepared {
   size_t smem;
   size_t ws_bytes;
   bool reg;
-  int T;  // tile tokens of the bf16 kernel
+  bool pipe;  // bf16: pipelined kernel (one token per tile)
+  int T;      // tile tokens of the bf16 kernel
 };
+
+void* pipe_kernel_ptr(int mode) {
+  switch (mode) {
+    case 1: return reinterpret_cast<void*>(ffb::pipe_tile_kernel<1>);
+    case 2: return reinterpret_cast<void*>(ffb::pipe_tile_kernel<2>);
+    case 4: return reinterpret_cast<void*>(ffb::pipe_tile_kernel<4>);
+    case 6: return reinterpret_cast<void*>(ffb::pipe_tile_kernel<6>);
+    case 7: return reinterpret_cast<void*>(ffb::pipe_tile_kernel<7>);
+    default: return nullptr;
+  }
+}
 
 // bf16 activations: tensor-core kernel with staged rows (tile of T = 1 or 2
 // tokens); fp32: exact FFT kernel.
@@ -113,6 +127,58 @@ size_t mma_smem_map(const framefb_mat* mats, int32_t nmats, int32_t ops, bool re
   return mbar + 16;
 }
 
+// Shared-memory map of the pipelined kernel: a ring of S staging buffers
+// (one token of X and dY each), two fp32 sets (V, U, RZ, RG of one token),
+// S mbarriers.  Returns the total bytes.
+size_t pipe_smem_map(const framefb_mat* mats, int32_t nmats, int32_t ops, int S, ffb::LaunchK* a) {
+  const bool F = ops & FRAMEFB_OP_FORWARD, D = ops & FRAMEFB_OP_BACKWARD_DX, C = ops & FRAMEFB_OP_GRAD_COEFF;
+  size_t stage = 0;
+  // one set layout for all matrices: the largest n, m and overflow counts
+  FfbPlanHeader hmax;
+  std::memset(&hmax, 0, sizeof(hmax));
+  for (int32_t j = 0; j < nmats; ++j) {
+    const FfbPlanHeader* h = plan_header(mats[j].plan);
+    const size_t rx = round_up(2 * static_cast<size_t>(h->n), 128), ry = round_up(2 * static_cast<size_t>(h->m), 128);
+    stage = std::max(stage, ((F || C) ? rx : 0) + ((D || C) ? ry : 0));
+    hmax.n = std::max(hmax.n, h->n);
+    hmax.m = std::max(hmax.m, h->m);
+    hmax.ovfZ = std::max(hmax.ovfZ, h->ovfZ);
+    hmax.ovfG = std::max(hmax.ovfG, h->ovfG);
+  }
+  const FfbTileLayout L = ffb_tile_layout(hmax, ops, 1, false);
+  const size_t set = round_up(static_cast<size_t>(L.total), 32);
+  size_t nfix = 0;  // fix-up items of the largest list
+  for (int32_t j = 0; j < nmats; ++j) {
+    const FfbPlanHeader* h = plan_header(mats[j].plan);
+    nfix = std::max<size_t>(nfix, (F ? h->nfixZ : 0) + (D ? h->nfixG : 0));
+  }
+  const size_t fbase = round_up(S * stage, 128);
+  const size_t fixc = round_up(fbase + 2 * set * 4, 16);
+  const size_t mbar = round_up(fixc + 16 * nfix, 16);
+  if (a) {
+    a->stg_in = 0;
+    a->stg_out = static_cast<int32_t>(stage);
+    a->stage_out = S;
+    a->fbase = static_cast<int32_t>(fbase);
+    a->mbar = static_cast<int32_t>(mbar);
+    a->set_oU = L.oU;
+    a->set_oRZ = L.oRZ;
+    a->set_oRG = L.oRG;
+    a->set_total = static_cast<int32_t>(set);
+    a->fixc = static_cast<int32_t>(fixc);
+    a->fixc_items = static_cast<int32_t>(nfix);
+    a->pad = kThreads - ffb::kPipeSpmm;  // first SpMM thread issues the copies
+  }
+  return mbar + 8 * static_cast<size_t>(S);
+}
+
+// Kernel choice for bf16: FRAMEFB_KERNEL=pipe selects the pipelined kernel
+// where it applies; by default the one-phase-at-a-time tile kernel runs.
+bool pipe_allowed() {
+  const char* e = std::getenv("FRAMEFB_KERNEL");
+  return e && std::strcmp(e, "pipe") == 0;
+}
+
 // Validate one chunk of matrices and fill the launch parameters.
 framefb_status prepare(const framefb_mat* mats, int32_t nmats, int32_t ops, framefb_dtype dt, Prepared& P) {
   const size_t esz = dt == FRAMEFB_BF16 ? 2 : 4;
@@ -130,7 +196,25 @@ framefb_status prepare(const framefb_mat* mats, int32_t nmats, int32_t ops, fram
   int64_t units = 0;
   size_t smem = 0;
   int T_mma = 0;
-  if (dt == FRAMEFB_BF16) {
+  bool pipe = false;
+  if (dt == FRAMEFB_BF16 && reg && pipe_allowed()) {
+    // pipelined kernel: deepest staging ring (2..4) that fits next to its
+    // static shared memory
+    int dev = 0, optin = 0;
+    cudaFuncAttributes fa{};
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess ||
+        cudaFuncGetAttributes(&fa, pipe_kernel_ptr(ops)) != cudaSuccess)
+      return FRAMEFB_ECUDA;
+    const size_t budget = static_cast<size_t>(optin) - fa.sharedSizeBytes;
+    for (int S = 4; S >= 2 && !pipe; --S)
+      if (pipe_smem_map(mats, nmats, ops, S, nullptr) <= budget) {
+        pipe = true;
+        T_mma = 1;
+        smem = pipe_smem_map(mats, nmats, ops, S, P.args);
+      }
+  }
+  if (dt == FRAMEFB_BF16 && !pipe) {
     // one tile size for the launch; stage the output rows too when they fit,
     // else the synthesis reads them from global memory
     bool staged = false;
@@ -210,12 +294,13 @@ framefb_status prepare(const framefb_mat* mats, int32_t nmats, int32_t ops, fram
   P.red->total_units = static_cast<int32_t>(units);
   P.red->stride = P.args->stride;
   P.reg = reg;
+  P.pipe = pipe;
   P.T = T_mma;
   P.smem = std::max<size_t>(smem, 16);
   P.grid = 0;
   P.ws_bytes = 0;
   if (units == 0) return FRAMEFB_OK;
-  void* fn = tile_kernel_ptr(dt, ops, reg, T_mma);
+  void* fn = pipe ? pipe_kernel_ptr(ops) : tile_kernel_ptr(dt, ops, reg, T_mma);
   if (!fn) return FRAMEFB_EINVAL;
   int dev = 0, sms = 0, per_sm = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return FRAMEFB_ECUDA;
@@ -293,7 +378,7 @@ extern "C" framefb_status framefb_run(const framefb_mat* mats, int32_t nmats, in
     }
     P.args->partial = static_cast<float*>(ws);
     P.red->partial = static_cast<const float*>(ws);
-    void* fn = tile_kernel_ptr(dtype, ops, P.reg, P.T);
+    void* fn = P.pipe ? pipe_kernel_ptr(ops) : tile_kernel_ptr(dtype, ops, P.reg, P.T);
     void* kargs[] = {P.args};
     if (cudaLaunchKernel(fn, dim3(P.grid), dim3(kThreads), kargs, P.smem, st) != cudaSuccess)
       return FRAMEFB_ECUDA;

@@ -55,6 +55,12 @@ struct LaunchK {
   // then dX) at stg_out when stage_out is set (else read from global
   // memory), the fp32 region of the tile layout at fbase, two mbarriers
   int32_t stg_in, stg_out, stage_out, fbase, mbar, pad2;
+  // pipelined kernel: one fp32 set layout for every matrix of the launch
+  // (offsets of U, RZ, RG and the set size in floats, from the largest n, m
+  // and overflow counts), so that sets of consecutive tiles of different
+  // matrices never overlap
+  int32_t set_oU, set_oRZ, set_oRG, set_total;
+  int32_t fixc, fixc_items;  // pipelined kernel: fix-up item cache (bytes offset, capacity)
   MatK m[kMaxMats];
 };
 
@@ -204,14 +210,14 @@ struct Seg<float> {
 
 // Store the 32 coefficients of one group (analysis output, slot order) into a
 // token row laid out by ffb_slot: float4 chunk j (pairs 2j, 2j + 1) goes to
-// chunk j ^ ((j >> 2) & 1), its two pairs swapped when the group is odd.
+// chunk j ^ ((j >> 2) & 1) ^ 4 (g odd), its two pairs swapped when g is odd.
 __device__ __forceinline__ void store_group(float* row, int g, const float (&xr)[16], const float (&xi)[16]) {
   float* base = row + 32 * g;
 #pragma unroll
   for (int c = 0; c < 8; ++c) {
     const int p0 = slot_of(2 * c), p1 = slot_of(2 * c + 1);
     const float4 v = (g & 1) ? make_float4(xr[p1], xi[p1], xr[p0], xi[p0]) : make_float4(xr[p0], xi[p0], xr[p1], xi[p1]);
-    *reinterpret_cast<float4*>(base + 4 * (c ^ ((c >> 2) & 1))) = v;
+    *reinterpret_cast<float4*>(base + 4 * (c ^ ((c >> 2) & 1) ^ ((g & 1) << 2))) = v;
   }
 }
 
@@ -220,7 +226,7 @@ __device__ __forceinline__ void load_group(const float* row, int g, float (&xr)[
   const float* base = row + 32 * g;
 #pragma unroll
   for (int c = 0; c < 8; ++c) {
-    const float4 v = *reinterpret_cast<const float4*>(base + 4 * (c ^ ((c >> 2) & 1)));
+    const float4 v = *reinterpret_cast<const float4*>(base + 4 * (c ^ ((c >> 2) & 1) ^ ((g & 1) << 2)));
     const bool sw = g & 1;
     xr[2 * c] = sw ? v.z : v.x;
     xi[2 * c] = sw ? v.w : v.y;
@@ -559,13 +565,13 @@ struct Chunk {
 // later pieces, stored in overflow slots, to the first piece.  Needs a
 // barrier before (pieces written) and after (sums complete).  Element
 // (token t, slot s) at s * T + t (minor) or t * stride + s.
-template <int MODE, bool MINOR>
+template <int MODE, bool MINOR, int NT = kThreads>
 __device__ __forceinline__ void fixup(const uint8_t* plan, const FfbTileLayout& L, float* fsm, int T, int Tc,
                                       int tid) {
   constexpr bool F = MODE & MODE_F, D = MODE & MODE_D;
   const FfbPlanHeader& h = hdr(plan);
   const int nfZ = F ? h.nfixZ : 0, nfG = D ? h.nfixG : 0;
-  for (int i = tid; i < nfZ + nfG; i += kThreads) {
+  for (int i = tid; i < nfZ + nfG; i += NT) {
     const bool z = i < nfZ;
     const int4 it = z ? __ldg(table<int4>(plan, h.off_fixZ) + i) : __ldg(table<int4>(plan, h.off_fixG) + (i - nfZ));
     float* R = fsm + (z ? L.oRZ : L.oRG);

@@ -132,7 +132,11 @@ struct DFrags {
 };
 
 // Pair p (0..15) of group r in a tile buffer: see ffb_slot.
-__device__ __forceinline__ int pair_slot(int p, int r) { return p ^ (((p >> 3) & 1) << 1) ^ (r & 1); }
+__device__ __forceinline__ int pair_slot(int p, int r) { return p ^ (((p >> 3) & 1) << 1) ^ (r & 1) ^ ((r & 1) << 3); }
+
+// One token per slot: 16-byte chunk position of chunk q (pairs 2q, 2q + 1;
+// stored swapped in odd groups) of group r, see ffb_slot.
+__device__ __forceinline__ int chunk_slot(int q, int r) { return q ^ ((q >> 2) & 1) ^ ((r & 1) << 2); }
 
 __device__ __forceinline__ uint4 lds128(const uint8_t* p) { return *reinterpret_cast<const uint4*>(p); }
 
@@ -161,10 +165,15 @@ struct Blk {
   const uint8_t* stg;  // staged bf16 token rows (stride rs bytes), or NULL
   float* buf;          // fp32 slot buffer (V / U written, RZ / RG read)
   __nv_bfloat16* out;  // synthesis: global output rows
-  const uint32_t* mask;
+  const uint32_t* mask;   // group masks of the plan (a group is skipped when its word is 0)
+  const uint32_t* mbits;  // or, when set: one bit per group (0: skipped)
   int64_t ld;
   int rs, G, b;
 };
+
+__device__ __forceinline__ bool blk_group_on(const Blk& k, int grp) {
+  return k.mbits ? ((k.mbits[grp >> 5] >> (grp & 31)) & 1u) != 0u : k.mask[grp] != 0u;
+}
 
 template <int T>
 __device__ __forceinline__ void blk_rows(const Blk& k, int Tc, int lane, int& grp0, int& grp1, bool& v0, bool& v1,
@@ -172,8 +181,8 @@ __device__ __forceinline__ void blk_rows(const Blk& k, int Tc, int lane, int& gr
   const int g = lane >> 2;
   grp0 = T == 2 ? 8 * k.b + g : 16 * k.b + g;
   grp1 = T == 2 ? grp0 : grp0 + 8;
-  v0 = grp0 < k.G && (!masked || k.mask[grp0] != 0u);
-  v1 = T == 2 ? (v0 && Tc > 1) : (grp1 < k.G && (!masked || k.mask[grp1] != 0u));
+  v0 = grp0 < k.G && (!masked || blk_group_on(k, grp0));
+  v1 = T == 2 ? (v0 && Tc > 1) : (grp1 < k.G && (!masked || blk_group_on(k, grp1)));
 }
 
 // Analysis of NB blocks into V (or U): K slot 8s + 4h + t reads coordinate
@@ -231,7 +240,7 @@ __device__ __forceinline__ void analysis_blocks(const DFrags& Df, const Blk (&k)
             const float4 lo =
                 make_float4(c[i][2 * h][o], c[i][2 * h][o + 1], c[i][2 * h + 1][o], c[i][2 * h + 1][o + 1]);
             const float4 v = (grp & 1) ? make_float4(lo.z, lo.w, lo.x, lo.y) : lo;
-            *reinterpret_cast<float4*>(grow + 4 * (q ^ ((q >> 2) & 1))) = v;
+            *reinterpret_cast<float4*>(grow + 4 * chunk_slot(q, grp)) = v;
           }
         }
       }
@@ -239,16 +248,38 @@ __device__ __forceinline__ void analysis_blocks(const DFrags& Df, const Blk (&k)
   }
 }
 
-// Synthesis of NB blocks: S Z (the row sums, with the sign pattern S folded
-// into the coefficient values) from the fp32 buffer in the analysis layout,
-// the output rows from staging or, when stg is NULL, from global memory;
-// y += seff * S (S Z) D^T-fragments = seff * Z D^T, written to the global rows
-// out + (t0 + token) * ld.  K slot 8s + 4h + t reads coefficient 8t + 2s + h;
-// N slot 8j + 2t + e writes coordinate 8t + 2j + e.  Groups whose mask is
-// zero have no support entries and are left untouched.
+// Output rows of NB synthesis blocks (the two rows of each lane's 16-byte
+// chunk), from staging or, when stg is NULL, from global memory.  Rows of
+// groups outside the matrix or with an empty mask are not read.
 template <int T, int NB>
-__device__ __forceinline__ void synthesis_blocks(const DFrags& Df, const Blk (&k)[NB], int64_t t0, int Tc, float seff,
-                                                 int lane) {
+__device__ __forceinline__ void syn_load(const Blk (&k)[NB], int64_t t0, int Tc, int lane, uint4 (&y)[NB][2]) {
+  const int t = lane & 3;
+#pragma unroll
+  for (int i = 0; i < NB; ++i) {
+    int grp0, grp1;
+    bool v0, v1;
+    blk_rows<T>(k[i], Tc, lane, grp0, grp1, v0, v1, true);
+    const int64_t row0 = t0, row1 = T == 2 ? t0 + 1 : t0;
+    y[i][0] = y[i][1] = make_uint4(0, 0, 0, 0);
+    if (v0)
+      y[i][0] = k[i].stg ? lds128(k[i].stg + grp0 * 64 + t * 16)
+                         : *reinterpret_cast<const uint4*>(k[i].out + row0 * k[i].ld + 32 * grp0 + 8 * t);
+    if (v1)
+      y[i][1] = k[i].stg ? lds128(k[i].stg + (T == 2 ? k[i].rs : 0) + grp1 * 64 + t * 16)
+                         : *reinterpret_cast<const uint4*>(k[i].out + row1 * k[i].ld + 32 * grp1 + 8 * t);
+  }
+}
+
+// Synthesis of NB blocks: S Z (the row sums, with the sign pattern S folded
+// into the coefficient values) from the fp32 buffer in the analysis layout;
+// y += seff * S (S Z) D^T-fragments = seff * Z D^T, with y the output rows
+// read by syn_load, written to the global rows out + (t0 + token) * ld.
+// K slot 8s + 4h + t reads coefficient 8t + 2s + h; N slot 8j + 2t + e writes
+// coordinate 8t + 2j + e.  Groups whose mask is zero have no support entries
+// and are left untouched.
+template <int T, int NB>
+__device__ __forceinline__ void syn_compute(const DFrags& Df, const Blk (&k)[NB], int64_t t0, int Tc, float seff,
+                                            int lane, const uint4 (&y)[NB][2]) {
   const int t = lane & 3;
   int grp0[NB], grp1[NB];
   bool v0[NB], v1[NB];
@@ -272,7 +303,7 @@ __device__ __forceinline__ void synthesis_blocks(const DFrags& Df, const Blk (&k
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
           const int q = 2 * t + h;
-          float4 f = v ? *reinterpret_cast<const float4*>(k[i].buf + 32 * grp + 4 * (q ^ ((q >> 2) & 1)))
+          float4 f = v ? *reinterpret_cast<const float4*>(k[i].buf + 32 * grp + 4 * chunk_slot(q, grp))
                        : make_float4(0.f, 0.f, 0.f, 0.f);
           if (grp & 1) f = make_float4(f.z, f.w, f.x, f.y);
           z[r][4 * h] = f.x;
@@ -284,18 +315,6 @@ __device__ __forceinline__ void synthesis_blocks(const DFrags& Df, const Blk (&k
 #pragma unroll
       for (int s = 0; s < 4; ++s) a[i][s] = make_float4(z[0][2 * s], z[1][2 * s], z[0][2 * s + 1], z[1][2 * s + 1]);
     }
-  }
-  uint4 y0[NB], y1[NB];
-#pragma unroll
-  for (int i = 0; i < NB; ++i) {
-    const int64_t row0 = t0, row1 = T == 2 ? t0 + 1 : t0;
-    y0[i] = y1[i] = make_uint4(0, 0, 0, 0);
-    if (v0[i])
-      y0[i] = k[i].stg ? lds128(k[i].stg + grp0[i] * 64 + t * 16)
-                       : *reinterpret_cast<const uint4*>(k[i].out + row0 * k[i].ld + 32 * grp0[i] + 8 * t);
-    if (v1[i])
-      y1[i] = k[i].stg ? lds128(k[i].stg + (T == 2 ? k[i].rs : 0) + grp1[i] * 64 + t * 16)
-                       : *reinterpret_cast<const uint4*>(k[i].out + row1 * k[i].ld + 32 * grp1[i] + 8 * t);
   }
   float c[NB][4][4];
 #pragma unroll
@@ -309,8 +328,7 @@ __device__ __forceinline__ void synthesis_blocks(const DFrags& Df, const Blk (&k
 #pragma unroll
       for (int i = 0; i < NB; ++i)
         mma_tf32(c[i][j], __float_as_uint(a[i][s].x), __float_as_uint(a[i][s].y), __float_as_uint(a[i][s].z),
-                 __float_as_uint(a[i][s].w),
-                 Df.b[j][s][0], Df.b[j][s][1]);
+                 __float_as_uint(a[i][s].w), Df.b[j][s][0], Df.b[j][s][1]);
   }
   // N slot 8j + 2t + e holds coordinate 8t + 2j + e
 #pragma unroll
@@ -318,13 +336,21 @@ __device__ __forceinline__ void synthesis_blocks(const DFrags& Df, const Blk (&k
     const int64_t row0 = t0, row1 = T == 2 ? t0 + 1 : t0;
     if (v0[i]) {
       const float d[8] = {c[i][0][0], c[i][0][1], c[i][1][0], c[i][1][1], c[i][2][0], c[i][2][1], c[i][3][0], c[i][3][1]};
-      *reinterpret_cast<uint4*>(k[i].out + row0 * k[i].ld + 32 * grp0[i] + 8 * t) = axpy_sd_bf16x8(y0[i], d, seff);
+      *reinterpret_cast<uint4*>(k[i].out + row0 * k[i].ld + 32 * grp0[i] + 8 * t) = axpy_sd_bf16x8(y[i][0], d, seff);
     }
     if (v1[i]) {
       const float d[8] = {c[i][0][2], c[i][0][3], c[i][1][2], c[i][1][3], c[i][2][2], c[i][2][3], c[i][3][2], c[i][3][3]};
-      *reinterpret_cast<uint4*>(k[i].out + row1 * k[i].ld + 32 * grp1[i] + 8 * t) = axpy_sd_bf16x8(y1[i], d, seff);
+      *reinterpret_cast<uint4*>(k[i].out + row1 * k[i].ld + 32 * grp1[i] + 8 * t) = axpy_sd_bf16x8(y[i][1], d, seff);
     }
   }
+}
+
+template <int T, int NB>
+__device__ __forceinline__ void synthesis_blocks(const DFrags& Df, const Blk (&k)[NB], int64_t t0, int Tc, float seff,
+                                                 int lane) {
+  uint4 y[NB][2];
+  syn_load<T, NB>(k, t0, Tc, lane, y);
+  syn_compute<T, NB>(Df, k, t0, Tc, seff, lane, y);
 }
 
 // Staged row strides (bytes) of a matrix: n-wide rows and m-wide rows.

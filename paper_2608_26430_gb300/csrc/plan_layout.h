@@ -54,13 +54,16 @@ struct FfbPlanHeader {
 // Slot of group-major index x (x < K) in a tile buffer.  Slots come in
 // pairs (x even, x + 1); the 16 pairs of a group are permuted so that the
 // MMA epilogue and prologue -- lane (g, t) touching pairs 4t..4t+3 of group
-// G0 + g, g = 0..7 -- spread every quarter-warp over distinct banks:
-//     pair p of group r -> pair p ^ (((p >> 3) & 1) << 1) ^ (r & 1).
+// G0 + g, g = 0..7 -- spread every quarter-warp over distinct banks, both
+// with two tokens per slot (a pair is one 16-byte chunk) and with one (a
+// 16-byte chunk holds two pairs; odd groups use the other half of the
+// 128-byte line):
+//     pair p of group r -> pair p ^ (((p >> 3) & 1) << 1) ^ (r & 1) ^ ((r & 1) << 3).
 // Overflow slots (x >= K) are used as they are.
 static inline __host__ __device__ int32_t ffb_slot(int32_t x, int32_t K) {
   if (x >= K) return x;
   const int32_t r = x >> 5, p = (x >> 1) & 15;
-  const int32_t pp = p ^ (((p >> 3) & 1) << 1) ^ (r & 1);
+  const int32_t pp = p ^ (((p >> 3) & 1) << 1) ^ (r & 1) ^ ((r & 1) << 3);
   return (r << 5) | (pp << 1) | (x & 1);
 }
 

@@ -138,7 +138,7 @@ def slot(x, K):
     """Tile-buffer slot of group-major index x (the map documented in plan_layout.h)."""
     x = np.asarray(x)
     r, p = x >> 5, (x >> 1) & 15
-    pp = p ^ (((p >> 3) & 1) << 1) ^ (r & 1)
+    pp = p ^ (((p >> 3) & 1) << 1) ^ (r & 1) ^ ((r & 1) << 3)
     return np.where(x >= K, x, (r << 5) | (pp << 1) | (x & 1))
 
 
@@ -154,6 +154,13 @@ def test_slot_map_is_a_pair_preserving_bijection_and_bank_spread():
     for G0 in range(0, 64, 2):
         for k in range(4):
             chunks = [(slot(32 * (G0 + g) + 2 * (4 * t + k), K) >> 1) % 8 for g in (0, 1) for t in range(4)]
+            assert len(set(chunks)) == 8
+    # one-token layout (a 16-byte chunk holds two pairs): lane (g, t) touches
+    # chunk q = 2t + h of group G0 + g; a quarter-warp (g in {0, 1}) must hit
+    # 8 distinct 16-byte positions of the 128-byte line
+    for G0 in range(0, 64, 2):
+        for h in range(2):
+            chunks = [(slot(32 * (G0 + g) + 4 * (2 * t + h), K) >> 2) % 8 for g in (0, 1) for t in range(4)]
             assert len(set(chunks)) == 8
 
 
