@@ -14,6 +14,7 @@
 #include "framefb_kernels.cuh"
 #include "framefb_mma.cuh"
 #include "framefb_pipe.cuh"
+#include "framefb_tc.cuh"
 #include "plan_internal.h"
 #include "plan_layout.h"
 
@@ -42,14 +43,28 @@ bool frame_ok(const framefb_dev_frame* f, int32_t d) {
 
 struct Prepared {
   ffb::LaunchK* args;  // heap: too large for the stack of some callers
+  ffb::TcLaunchK* tcargs;
   ffb::ReduceK* red;
   int grid;
   size_t smem;
   size_t ws_bytes;
   bool reg;
   bool pipe;  // bf16: pipelined kernel (one token per tile)
+  bool tc;    // bf16: pipelined kernel on tcgen05 tensor cores
   int T;      // tile tokens of the bf16 kernel
+  int threads;
 };
+
+void* tc_kernel_ptr(int mode) {
+  switch (mode) {
+    case 1: return reinterpret_cast<void*>(ffb::tc_tile_kernel<1>);
+    case 2: return reinterpret_cast<void*>(ffb::tc_tile_kernel<2>);
+    case 4: return reinterpret_cast<void*>(ffb::tc_tile_kernel<4>);
+    case 6: return reinterpret_cast<void*>(ffb::tc_tile_kernel<6>);
+    case 7: return reinterpret_cast<void*>(ffb::tc_tile_kernel<7>);
+    default: return nullptr;
+  }
+}
 
 void* pipe_kernel_ptr(int mode) {
   switch (mode) {
@@ -172,12 +187,99 @@ size_t pipe_smem_map(const framefb_mat* mats, int32_t nmats, int32_t ops, int S,
   return mbar + 8 * static_cast<size_t>(S);
 }
 
-// Kernel choice for bf16: FRAMEFB_KERNEL=pipe selects the pipelined kernel
-// where it applies; by default the one-phase-at-a-time tile kernel runs.
-bool pipe_allowed() {
-  const char* e = std::getenv("FRAMEFB_KERNEL");
-  return e && std::strcmp(e, "pipe") == 0;
+// Shared-memory map of the tensor-core pipelined kernel: a ring of S stages
+// (one token row of X then dY, each landed by a tensor copy as a swizzled
+// K-major operand padded to whole 128-group tiles), B operands (8 KB), two
+// fp32 sets in the canonical tf32 layout (RZ / RG padded to whole tiles), the
+// fix-up item cache, S + 1 mbarriers.  Returns the total bytes, or 0 when a
+// matrix does not fit the kernel's shape rules.
+size_t tc_smem_map(const framefb_mat* mats, int32_t nmats, int32_t ops, int S, ffb::TcLaunchK* a) {
+  const bool F = ops & FRAMEFB_OP_FORWARD, D = ops & FRAMEFB_OP_BACKWARD_DX, C = ops & FRAMEFB_OP_GRAD_COEFF;
+  const bool needV = F || C, needU = D || C;
+  size_t nfix = 0;
+  int32_t nmax = 0, mmax = 0, ovfZ = 0, ovfG = 0;
+  for (int32_t j = 0; j < nmats; ++j) {
+    const FfbPlanHeader* h = plan_header(mats[j].plan);
+    if (h->Gn % 8 || h->Gm % 8 || h->Gn > 128 * ffb::kTcMaxTiles || h->Gm > 128 * ffb::kTcMaxTiles) return 0;
+    nmax = std::max(nmax, h->n);
+    mmax = std::max(mmax, h->m);
+    ovfZ = std::max(ovfZ, h->ovfZ);
+    ovfG = std::max(ovfG, h->ovfG);
+    nfix = std::max<size_t>(nfix, (F ? h->nfixZ : 0) + (D ? h->nfixG : 0));
+  }
+  auto tiles = [](int32_t d) { return static_cast<size_t>((d / 32 + 127) / 128); };
+  const size_t xbox = needV ? tiles(nmax) * 8192 : 0;
+  const size_t stage = xbox + (needU ? tiles(mmax) * 8192 : 0);
+  const size_t bops = S * stage;
+  const size_t fbase = bops + 8192;
+  // set layout (floats)
+  const size_t oU = needV ? nmax : 0;
+  const size_t oRZ = round_up(oU + (needU ? mmax : 0), 32);
+  const size_t szRZ = F ? round_up(std::max<size_t>(tiles(mmax) * 128 * 32, mmax + ovfZ), 32) : 0;
+  const size_t oRG = oRZ + szRZ;
+  const size_t szRG = D ? round_up(std::max<size_t>(tiles(nmax) * 128 * 32, nmax + ovfG), 32) : 0;
+  const size_t set = oRG + szRG;
+  const size_t fixc = fbase + 2 * set * 4;
+  const size_t mbar = round_up(fixc + 16 * nfix, 16);
+  if (a) {
+    a->S = S;
+    a->stage = static_cast<int32_t>(stage);
+    a->xbox_u = static_cast<int32_t>(xbox);
+    a->bops = static_cast<int32_t>(bops);
+    a->fbase = static_cast<int32_t>(fbase);
+    a->set_oU = static_cast<int32_t>(oU);
+    a->set_oRZ = static_cast<int32_t>(oRZ);
+    a->set_oRG = static_cast<int32_t>(oRG);
+    a->set_total = static_cast<int32_t>(set);
+    a->fixc = static_cast<int32_t>(fixc);
+    a->fixc_items = static_cast<int32_t>(nfix);
+    a->mbar = static_cast<int32_t>(mbar);
+  }
+  return mbar + 8 * static_cast<size_t>(S + 1);
 }
+
+// cuTensorMapEncodeTiled through the runtime's driver entry point (no link
+// against the driver library).
+using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+EncodeTiledFn encode_tiled() {
+  static const EncodeTiledFn fn = [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q{};
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) !=
+            cudaSuccess ||
+        q != cudaDriverEntryPointSuccess)
+      return static_cast<EncodeTiledFn>(nullptr);
+    return reinterpret_cast<EncodeTiledFn>(p);
+  }();
+  return fn;
+}
+
+// Tensor map of the bf16 rows of one activation tensor (d features, N
+// tokens, leading dimension ld elements): {32 coordinates, d / 32 groups, N
+// tokens}, box {32, d / 32, 1}, 64-byte swizzle.
+bool encode_rows(CUtensorMap* map, const void* base, int32_t d, int32_t N, int64_t ld) {
+  const EncodeTiledFn fn = encode_tiled();
+  if (!fn) return false;
+  const cuuint64_t dims[3] = {32, static_cast<cuuint64_t>(d / 32), static_cast<cuuint64_t>(N)};
+  const cuuint64_t strides[2] = {64, static_cast<cuuint64_t>(ld) * 2};
+  const cuuint32_t box[3] = {32, static_cast<cuuint32_t>(d / 32), 1};
+  const cuuint32_t estr[3] = {1, 1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// Kernel choice for bf16 (FRAMEFB_KERNEL): "tc" the tensor-core pipelined
+// kernel, "pipe" the warp-MMA pipelined kernel, where they apply; by default
+// the one-phase-at-a-time tile kernel runs.
+bool kernel_is(const char* name) {
+  const char* e = std::getenv("FRAMEFB_KERNEL");
+  return e && std::strcmp(e, name) == 0;
+}
+bool pipe_allowed() { return kernel_is("pipe"); }
+bool tc_allowed() { return kernel_is("tc"); }
 
 // Validate one chunk of matrices and fill the launch parameters.
 framefb_status prepare(const framefb_mat* mats, int32_t nmats, int32_t ops, framefb_dtype dt, Prepared& P) {
@@ -196,8 +298,27 @@ framefb_status prepare(const framefb_mat* mats, int32_t nmats, int32_t ops, fram
   int64_t units = 0;
   size_t smem = 0;
   int T_mma = 0;
-  bool pipe = false;
-  if (dt == FRAMEFB_BF16 && reg && pipe_allowed()) {
+  bool pipe = false, tc = false;
+  if (dt == FRAMEFB_BF16 && reg && tc_allowed() && nmats <= ffb::kTcMaxMats && encode_tiled()) {
+    // tensor-core pipelined kernel: deepest staging ring (2..4) that fits
+    int dev = 0, optin = 0;
+    cudaFuncAttributes fa{};
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess ||
+        cudaFuncGetAttributes(&fa, tc_kernel_ptr(ops)) != cudaSuccess)
+      return FRAMEFB_ECUDA;
+    const size_t budget = static_cast<size_t>(optin) - fa.sharedSizeBytes;
+    for (int S = 4; S >= 2 && !tc; --S) {
+      const size_t need = tc_smem_map(mats, nmats, ops, S, nullptr);
+      if (need > 0 && need <= budget) {
+        tc = true;
+        T_mma = 1;
+        std::memset(P.tcargs, 0, sizeof(ffb::TcLaunchK));
+        smem = tc_smem_map(mats, nmats, ops, S, P.tcargs);
+      }
+    }
+  }
+  if (dt == FRAMEFB_BF16 && reg && !tc && pipe_allowed()) {
     // pipelined kernel: deepest staging ring (2..4) that fits next to its
     // static shared memory
     int dev = 0, optin = 0;
@@ -214,7 +335,7 @@ framefb_status prepare(const framefb_mat* mats, int32_t nmats, int32_t ops, fram
         smem = pipe_smem_map(mats, nmats, ops, S, P.args);
       }
   }
-  if (dt == FRAMEFB_BF16 && !pipe) {
+  if (dt == FRAMEFB_BF16 && !pipe && !tc) {
     // one tile size for the launch; stage the output rows too when they fit,
     // else the synthesis reads them from global memory
     bool staged = false;
@@ -290,17 +411,32 @@ framefb_status prepare(const framefb_mat* mats, int32_t nmats, int32_t ops, fram
   P.args->nmats = nmats;
   P.args->total_units = static_cast<int32_t>(units);
   P.args->stride = (nnz_max + 63) & ~63;
+  if (tc) {
+    ffb::TcLaunchK& A = *P.tcargs;
+    A.nmats = nmats;
+    A.total_units = P.args->total_units;
+    A.stride = P.args->stride;
+    for (int32_t j = 0; j < nmats; ++j) {
+      A.m[j] = P.args->m[j];
+      const framefb_mat& M = mats[j];
+      if (M.N == 0) continue;
+      if ((F || C) && !encode_rows(&A.maps[2 * j], M.X, M.n, M.N, M.ldx)) return FRAMEFB_ECUDA;
+      if ((D || C) && !encode_rows(&A.maps[2 * j + 1], M.dY, M.m, M.N, M.ldy)) return FRAMEFB_ECUDA;
+    }
+  }
   P.red->nmats = nmats;
   P.red->total_units = static_cast<int32_t>(units);
   P.red->stride = P.args->stride;
   P.reg = reg;
   P.pipe = pipe;
+  P.tc = tc;
+  P.threads = tc ? ffb::kTcThreads : kThreads;
   P.T = T_mma;
   P.smem = std::max<size_t>(smem, 16);
   P.grid = 0;
   P.ws_bytes = 0;
   if (units == 0) return FRAMEFB_OK;
-  void* fn = pipe ? pipe_kernel_ptr(ops) : tile_kernel_ptr(dt, ops, reg, T_mma);
+  void* fn = tc ? tc_kernel_ptr(ops) : pipe ? pipe_kernel_ptr(ops) : tile_kernel_ptr(dt, ops, reg, T_mma);
   if (!fn) return FRAMEFB_EINVAL;
   int dev = 0, sms = 0, per_sm = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return FRAMEFB_ECUDA;
@@ -308,7 +444,7 @@ framefb_status prepare(const framefb_mat* mats, int32_t nmats, int32_t ops, fram
   if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(P.smem)) !=
       cudaSuccess)
     return FRAMEFB_ECUDA;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, kThreads, P.smem) != cudaSuccess)
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, P.threads, P.smem) != cudaSuccess)
     return FRAMEFB_ECUDA;
   if (per_sm < 1) return FRAMEFB_EUNSUPPORTED;
   P.grid = static_cast<int>(std::min<int64_t>(static_cast<int64_t>(sms) * per_sm, units));
@@ -318,15 +454,22 @@ framefb_status prepare(const framefb_mat* mats, int32_t nmats, int32_t ops, fram
 }
 
 struct Buffers {
-  std::vector<uint8_t> a, r;
-  Buffers() : a(sizeof(ffb::LaunchK)), r(sizeof(ffb::ReduceK)) {}
+  std::vector<uint8_t> a, t, r;
+  Buffers() : a(sizeof(ffb::LaunchK)), t(sizeof(ffb::TcLaunchK) + 64), r(sizeof(ffb::ReduceK)) {}
   Prepared prep() {
     Prepared p{};
     p.args = reinterpret_cast<ffb::LaunchK*>(a.data());
+    // tensor maps want 64-byte alignment
+    const uintptr_t ta = (reinterpret_cast<uintptr_t>(t.data()) + 63) & ~uintptr_t{63};
+    p.tcargs = reinterpret_cast<ffb::TcLaunchK*>(ta);
     p.red = reinterpret_cast<ffb::ReduceK*>(r.data());
     return p;
   }
 };
+
+// Matrices per launch: the tensor-core kernel carries tensor maps in its
+// parameters and takes fewer.
+int32_t chunk_mats(framefb_dtype dt) { return (dt == FRAMEFB_BF16 && tc_allowed()) ? ffb::kTcMaxMats : kMaxMats; }
 
 bool ops_ok(int32_t ops) { return ops == 1 || ops == 2 || ops == 4 || ops == 6 || ops == 7; }
 
@@ -336,10 +479,12 @@ extern "C" size_t framefb_workspace_size(const framefb_mat* mats, int32_t nmats,
   if (!mats || nmats <= 0 || !ops_ok(ops)) return 0;
   Buffers b;
   size_t need = 0;
-  for (int32_t j0 = 0; j0 < nmats; j0 += kMaxMats) {
+  const int32_t cm = chunk_mats(FRAMEFB_BF16);
+  for (int32_t j0 = 0; j0 < nmats; j0 += cm) {
     Prepared P = b.prep();
-    // dtype does not change the workspace; bf16 is used for the occupancy query
-    if (prepare(mats + j0, std::min(kMaxMats, nmats - j0), ops, FRAMEFB_BF16, P) != FRAMEFB_OK) return 0;
+    // the workspace depends on the launch chunking and the grid; bf16 is used
+    // for the occupancy query (the fp32 kernels run with the same grid bound)
+    if (prepare(mats + j0, std::min(cm, nmats - j0), ops, FRAMEFB_BF16, P) != FRAMEFB_OK) return 0;
     need = std::max(need, P.ws_bytes);
   }
   return need;
@@ -352,18 +497,19 @@ extern "C" framefb_status framefb_run(const framefb_mat* mats, int32_t nmats, in
   if (nmats == 0) return FRAMEFB_OK;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   Buffers b;
+  const int32_t cm = chunk_mats(dtype);
   // validate every chunk before queueing anything
-  for (int32_t j0 = 0; j0 < nmats; j0 += kMaxMats) {
+  for (int32_t j0 = 0; j0 < nmats; j0 += cm) {
     Prepared P = b.prep();
-    const framefb_status s = prepare(mats + j0, std::min(kMaxMats, nmats - j0), ops, dtype, P);
+    const framefb_status s = prepare(mats + j0, std::min(cm, nmats - j0), ops, dtype, P);
     if (s != FRAMEFB_OK) return s;
     if (P.ws_bytes > 0) {
       if (!ws || ws_bytes < P.ws_bytes) return FRAMEFB_EWORKSPACE;
       if (reinterpret_cast<uintptr_t>(ws) & 255u) return FRAMEFB_EINVAL;
     }
   }
-  for (int32_t j0 = 0; j0 < nmats; j0 += kMaxMats) {
-    const int32_t nm = std::min(kMaxMats, nmats - j0);
+  for (int32_t j0 = 0; j0 < nmats; j0 += cm) {
+    const int32_t nm = std::min(cm, nmats - j0);
     Prepared P = b.prep();
     const framefb_status s = prepare(mats + j0, nm, ops, dtype, P);
     if (s != FRAMEFB_OK) return s;
@@ -377,10 +523,11 @@ extern "C" framefb_status framefb_run(const framefb_mat* mats, int32_t nmats, in
       continue;
     }
     P.args->partial = static_cast<float*>(ws);
+    P.tcargs->partial = static_cast<float*>(ws);
     P.red->partial = static_cast<const float*>(ws);
-    void* fn = P.pipe ? pipe_kernel_ptr(ops) : tile_kernel_ptr(dtype, ops, P.reg, P.T);
-    void* kargs[] = {P.args};
-    if (cudaLaunchKernel(fn, dim3(P.grid), dim3(kThreads), kargs, P.smem, st) != cudaSuccess)
+    void* fn = P.tc ? tc_kernel_ptr(ops) : P.pipe ? pipe_kernel_ptr(ops) : tile_kernel_ptr(dtype, ops, P.reg, P.T);
+    void* kargs[] = {P.tc ? static_cast<void*>(P.tcargs) : static_cast<void*>(P.args)};
+    if (cudaLaunchKernel(fn, dim3(P.grid), dim3(P.threads), kargs, P.smem, st) != cudaSuccess)
       return FRAMEFB_ECUDA;
     if (ops & FRAMEFB_OP_GRAD_COEFF) {
       int nnz_max = 0;

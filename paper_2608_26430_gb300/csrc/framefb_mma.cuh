@@ -393,7 +393,8 @@ __device__ __forceinline__ void stage_rows(const MatK& M, const LaunchK& args, u
   }
 }
 
-__device__ __forceinline__ int matrix_of(const LaunchK& args, int j, int64_t u) {
+template <typename Args>
+__device__ __forceinline__ int matrix_of(const Args& args, int j, int64_t u) {
   while (u >= args.m[j].ubeg + args.m[j].ntiles) ++j;
   return j;
 }

@@ -1,0 +1,657 @@
+// Pipelined bf16 tile kernel on 5th-generation tensor cores (tcgen05, TMEM).
+// Included by framefb_cuda.cu after framefb_pipe.cuh.
+//
+// The work per one-token tile is that of mma_tile_kernel (Sec. 3.1 update and
+// the Lemma 1 gradient of Appendix A); the schedule is that of
+// pipe_tile_kernel (step s: analysis of tile s and synthesis of tile s-2 on
+// the tensor side, coefficient SpMM of tile s-1, one barrier per step), with
+// these differences:
+//   * the group contractions are UMMA instructions issued by one thread:
+//       analysis   V (M = 128 groups x N = 32 coefficients) = X_rows (K = 32
+//                  coordinates, bf16) x D, D split into bf16 hi + lo parts
+//                  (kind::f16, fp32 accumulate in TMEM);
+//       synthesis  dY_rows (M = 128 groups x N = 32 coordinates) = Z (K = 32
+//                  coefficients, fp32 read as tf32) x D^T (kind::tf32);
+//     the results are read back with tcgen05.ld, one TMEM lane per group;
+//   * X / dY token rows land by tensor copies (TMA) directly as the
+//     SWIZZLE_64B K-major bf16 operand (one 64-byte row per group);
+//   * the fp32 coefficient buffers V, U, RZ, RG use the canonical K-major
+//     core-matrix layout of a tf32 operand (8 groups x 4 coefficients per
+//     128-byte core matrix), so RZ / RG feed the tensor core directly and a
+//     warp's row writes are bank-conflict free;
+//   * 4 tensor warps (one per TMEM lane quarter) and 8 SpMM warps: SpMM
+//     thread t owns plan column t, its entries and dC sums in registers.
+// Shapes: every group count a multiple of 8 and at most 256 (n, m <= 8192).
+//
+// All waits (copies, MMA completion) are bounded; a wait that gives up
+// increments g_wait_timeouts, the CTA stops at the end of the step, lets its
+// copies and MMAs finish, frees its TMEM and exits.
+#pragma once
+#include <cuda.h>
+
+#include "framefb_pipe.cuh"
+
+namespace ffb {
+
+constexpr int kTcThreads = 384;            // 4 tensor warps + 8 SpMM warps
+constexpr int kTcSpmm = kTcThreads - 128;  // SpMM threads (= plan columns)
+constexpr int kTcMaxTiles = 2;             // 128-group tiles per side
+constexpr uint32_t kTcTmemCols = 256;      // 4 sides x 2 tiles x 32 columns
+
+static_assert(kTcSpmm == kThreads, "one SpMM thread per plan column");
+
+// Canonical K-major, no-swizzle operand layouts (core matrix = 8 rows x 16 B,
+// rows 16 B apart; K-adjacent core matrices LBO = 128 B apart; 8-row blocks
+// SBO apart).  bf16 rows of 32 elements: SBO = 512 B.  fp32 rows of 32
+// elements: SBO = 1024 B.
+__host__ __device__ __forceinline__ int can_bf16_off(int row, int k) {  // bytes
+  return ((row >> 3) * 4 + (k >> 3)) * 128 + (row & 7) * 16 + (k & 7) * 2;
+}
+__host__ __device__ __forceinline__ int can_f32_off(int row, int k) {  // floats
+  return ((row >> 3) * 8 + (k >> 2)) * 32 + (row & 7) * 4 + (k & 3);
+}
+// Slot of group-major index x (x < K) in a canonical fp32 buffer; overflow
+// slots (x >= K) as they are.
+__host__ __device__ __forceinline__ int32_t tc_slot(int32_t x, int32_t K) {
+  return x >= K ? x : can_f32_off(x >> 5, x & 31);
+}
+
+// Shared-memory descriptor, no swizzle.
+__device__ __forceinline__ uint64_t umma_sdesc(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+  uint64_t d = static_cast<uint64_t>((saddr >> 4) & 0x3FFFu);
+  d |= static_cast<uint64_t>((lbo >> 4) & 0x3FFFu) << 16;
+  d |= static_cast<uint64_t>((sbo >> 4) & 0x3FFFu) << 32;
+  d |= static_cast<uint64_t>(1) << 46;  // descriptor version of tcgen05
+  return d;
+}
+
+// SWIZZLE_64B K-major descriptor (layout type 4): SBO = 512 B between 8-row
+// atoms, K steps by advancing the start address inside the 64-byte row.
+__device__ __forceinline__ uint64_t umma_sdesc_sw64(uint32_t saddr) {
+  uint64_t d = static_cast<uint64_t>((saddr >> 4) & 0x3FFFu);
+  d |= static_cast<uint64_t>(1) << 16;         // LBO (unused within the atom)
+  d |= static_cast<uint64_t>(512 >> 4) << 32;  // SBO
+  d |= static_cast<uint64_t>(1) << 46;         // descriptor version
+  d |= static_cast<uint64_t>(4) << 61;         // SWIZZLE_64B
+  return d;
+}
+
+// Instruction descriptor: fp32 accumulator, A / B format (kind::f16: 1 = bf16;
+// kind::tf32: 2 = tf32), both K-major, M x N.
+__host__ __device__ constexpr uint32_t umma_idesc(uint32_t fmt, uint32_t M, uint32_t N) {
+  return (1u << 4) | (fmt << 7) | (fmt << 10) | ((N >> 3) << 17) | ((M >> 4) << 24);
+}
+
+__device__ __forceinline__ void umma_f16(uint32_t tmem_d, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem_d),
+      "l"(a), "l"(b), "r"(idesc), "r"(acc)
+      : "memory");
+}
+
+__device__ __forceinline__ void umma_tf32(uint32_t tmem_d, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::tf32 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem_d),
+      "l"(a), "l"(b), "r"(idesc), "r"(acc)
+      : "memory");
+}
+
+__device__ __forceinline__ void umma_commit(uint64_t* bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
+               : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void fence_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+__device__ __forceinline__ void tensor_bar() { asm volatile("bar.sync 2, 128;" ::: "memory"); }
+// barrier of the 128 tensor threads that also ORs a flag over them
+__device__ __forceinline__ bool tensor_bar_or(bool f) {
+  uint32_t out;
+  asm volatile(
+      "{\n .reg .pred p, q;\n setp.ne.u32 p, %1, 0;\n bar.red.or.pred q, 2, 128, p;\n selp.u32 %0, 1, 0, q;\n}\n"
+      : "=r"(out)
+      : "r"(static_cast<uint32_t>(f))
+      : "memory");
+  return out != 0;
+}
+__device__ __forceinline__ void tc_spmm_bar() { asm volatile("bar.sync 1, %0;" ::"n"(kTcSpmm) : "memory"); }
+
+// 32 consecutive fp32 columns of this thread's TMEM lane.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];\n"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+        "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+        "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// y (8 bf16 of one 16-byte chunk) += seff * d[0..7]
+__device__ __forceinline__ uint4 axpy8(uint4 y, const float* d, float seff) {
+  uint32_t w[4] = {y.x, y.y, y.z, y.w};
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const float lo = fmaf(seff, d[2 * i], __uint_as_float(w[i] << 16));
+    const float hi = fmaf(seff, d[2 * i + 1], __uint_as_float(w[i] & 0xFFFF0000u));
+    w[i] = pack_bf16(lo, hi);
+  }
+  return make_uint4(w[0], w[1], w[2], w[3]);
+}
+
+// Coefficient SpMM of one register chunk for one token (canonical fp32 slots,
+// no sign folding): run sums of c V[b] into RZ, of c U[a] into RG; dc += U V.
+template <int MODE>
+__device__ __forceinline__ void tc_spmm(const Chunk<MODE, true, false>& ch, float (&dc)[kEreg], float* fs,
+                                        const FfbTileLayout& L) {
+  constexpr bool F = MODE & MODE_F, D = MODE & MODE_D, C = MODE & MODE_C;
+  constexpr int B = FFB_ENTRY_BLOCK;
+  const float* __restrict__ V = fs + L.oV;
+  const float* __restrict__ U = fs + L.oU;
+  float* __restrict__ RZ = fs + L.oRZ;
+  float* __restrict__ RG = fs + L.oRG;
+  if constexpr (F) {
+    float acc = 0.f;
+#pragma unroll
+    for (int e0 = 0; e0 < kEreg; e0 += B) {
+      if (e0 < ch.EZ) {
+        float v[B];
+#pragma unroll
+        for (int e = 0; e < B; ++e) v[e] = V[ch.zb[e0 + e] & 0xFFFFu];
+#pragma unroll
+        for (int e = 0; e < B; ++e) {
+          acc = fmaf(ch.zc[e0 + e], v[e], acc);
+          const uint32_t st = ch.zb[e0 + e] >> 16;
+          if (st != FFB_NO_STORE) {
+            RZ[st] = acc;
+            acc = 0.f;
+          }
+        }
+      }
+    }
+  }
+  if constexpr (D || C) {
+    float acc = 0.f, vlast = 0.f;
+#pragma unroll
+    for (int e0 = 0; e0 < kEreg; e0 += B) {
+      if (e0 < ch.EG) {
+        float u[B], v[B];
+#pragma unroll
+        for (int e = 0; e < B; ++e) {
+          u[e] = U[ch.ga[e0 + e] & 0xFFFFu];
+          if constexpr (C) {
+            const int ep = e0 + e - 1;
+            if (ep < 0 || ch.gb[e0 + e] != ch.gb[ep])
+              v[e] = V[ch.gb[e0 + e]];
+            else
+              v[e] = e > 0 ? v[e - 1] : vlast;
+          }
+        }
+        if constexpr (C) vlast = v[B - 1];
+#pragma unroll
+        for (int e = 0; e < B; ++e) {
+          if constexpr (C) dc[e0 + e] = fmaf(u[e], v[e], dc[e0 + e]);
+          if constexpr (D) {
+            acc = fmaf(ch.gc[e0 + e], u[e], acc);
+            const uint32_t st = ch.ga[e0 + e] >> 16;
+            if (st != FFB_NO_STORE) {
+              RG[st] = acc;
+              acc = 0.f;
+            }
+          }
+        }
+      }
+    }
+  }
+}
+
+// Register chunk of plan column `col` with canonical slots (the plan words
+// hold group-major indices, mapped here with tc_slot; no sign folding).
+template <int MODE>
+__device__ __forceinline__ void tc_load_chunk(Chunk<MODE, true, false>& ch, const uint8_t* plan, const float* c_val,
+                                              int col) {
+  constexpr bool F = MODE & MODE_F, D = MODE & MODE_D, C = MODE & MODE_C;
+  const FfbPlanHeader& h = hdr(plan);
+  ch.EZ = h.EZ;
+  ch.EG = h.EG;
+  ch.n = h.n;
+  ch.m = h.m;
+  const int32_t* tzb = table<int32_t>(plan, h.off_zb);
+  const int32_t* tzq = table<int32_t>(plan, h.off_zq);
+  const int32_t* tga = table<int32_t>(plan, h.off_ga);
+  const int32_t* tgb = table<int32_t>(plan, h.off_gb);
+  const int32_t* tgq = table<int32_t>(plan, h.off_gq);
+  auto slots = [](uint32_t w, int Klo, int Khi) {
+    const uint32_t lo = w & 0x7FFFu, hi = w >> 16;
+    const uint32_t slo = static_cast<uint32_t>(tc_slot(static_cast<int32_t>(lo), Klo));
+    const uint32_t shi =
+        hi == FFB_NO_STORE ? FFB_NO_STORE : static_cast<uint32_t>(tc_slot(static_cast<int32_t>(hi), Khi));
+    return slo | (shi << 16);
+  };
+#pragma unroll
+  for (int e = 0; e < kEreg; ++e) {
+    ch.zb[e] = FFB_NO_STORE << 16;
+    ch.ga[e] = FFB_NO_STORE << 16;
+    ch.gb[e] = 0;
+    ch.zc[e] = ch.gc[e] = 0.f;
+    if (F && e < ch.EZ) {
+      const uint32_t w = static_cast<uint32_t>(__ldg(tzb + e * kThreads + col));
+      ch.zb[e] = slots(w, ch.n, ch.m);
+      const int32_t q = __ldg(tzq + e * kThreads + col);
+      ch.zc[e] = q >= 0 ? __ldg(c_val + q) : 0.f;
+    }
+    if ((D || C) && e < ch.EG) {
+      const uint32_t w = static_cast<uint32_t>(__ldg(tga + e * kThreads + col));
+      ch.ga[e] = slots(w, ch.m, ch.n);
+      ch.gb[e] = static_cast<uint32_t>(tc_slot(__ldg(tgb + e * kThreads + col), ch.n));
+      const int32_t q = __ldg(tgq + e * kThreads + col);
+      ch.gc[e] = (D && q >= 0) ? __ldg(c_val + q) : 0.f;
+    }
+  }
+}
+
+// Launch parameters of the tensor-core kernel: the fields of LaunchK it
+// uses, at most kTcMaxMats matrices, and one TMA tensor map per activation
+// tensor (X of matrix j at 2j, dY at 2j + 1): a 3-D view {32 coordinates,
+// groups, tokens} of the row-major bf16 rows, box {32, G, 1}, 64-byte
+// swizzle, which lands one token row as the canonical SWIZZLE_64B K-major
+// UMMA operand (8-row atoms of 512 bytes).
+constexpr int kTcMaxMats = 64;
+struct TcLaunchK {
+  int32_t nmats, total_units, stride, S;
+  float* partial;
+  int32_t stage, xbox_u, fbase, mbar;  // staging ring: stage stride, dY box offset (bytes)
+  int32_t set_oU, set_oRZ, set_oRG, set_total;
+  int32_t fixc, fixc_items, bops, pad;
+  MatK m[kTcMaxMats];
+  alignas(64) CUtensorMap maps[2 * kTcMaxMats];
+};
+
+__device__ __forceinline__ void tma_row3d(void* dst, const CUtensorMap* map, int32_t token, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4}], [%5];" ::
+          "r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(0), "r"(0), "r"(token), "r"(smem_u32(bar))
+      : "memory");
+}
+
+template <int MODE>
+__global__ void __launch_bounds__(kTcThreads, 1) tc_tile_kernel(const __grid_constant__ TcLaunchK args) {
+  constexpr bool F = MODE & MODE_F, D = MODE & MODE_D, C = MODE & MODE_C;
+  constexpr bool NEED_V = F || C, NEED_U = D || C, SYN = F || D;
+  extern __shared__ __align__(1024) uint8_t smem[];
+  __shared__ MatK mats_sm[kDescRing];
+  __shared__ int32_t mat_idx[kDescRing];
+  __shared__ int32_t tile_mat[kDescRing];
+  __shared__ uint32_t mat_bits[kDescRing][2][kGroupWords];
+  __shared__ uint32_t tmem_slot;
+  const int S = args.S;
+  uint8_t* stg0 = smem;              // stage b at b * stage: X box, dY box at xbox_u
+  float* fset0 = reinterpret_cast<float*>(smem + args.fbase);
+  uint8_t* bops = smem + args.bops;  // B operands: D hi, D lo (bf16), D^T (tf32)
+  uint64_t* bar = reinterpret_cast<uint64_t*>(smem + args.mbar);
+  uint64_t* mma_bar = bar + S;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  FfbTileLayout PL{};
+  PL.oV = 0;
+  PL.oU = args.set_oU;
+  PL.oRZ = args.set_oRZ;
+  PL.oRG = args.set_oRG;
+  PL.total = args.set_total;
+
+  const int64_t units = args.total_units;
+  const int64_t u_begin = (static_cast<int64_t>(blockIdx.x) * units) / gridDim.x;
+  const int64_t u_end = (static_cast<int64_t>(blockIdx.x + 1) * units) / gridDim.x;
+  const int count = static_cast<int>(u_end - u_begin);
+  if (count <= 0) return;
+
+  if (tid == 0) {
+    for (int b = 0; b <= S; ++b) mbar_init(bar + b, 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 0) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&tmem_slot)),
+                 "r"(kTcTmemCols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+
+  // ---- copy issue (thread 32): descriptors, group bitmaps, tensor copies
+  constexpr int kIssuer = 32;
+  int jn = 0, jn_end = 0, jn_loaded = -1, nq = -1, issued = 0;
+  auto issue = [&]() {
+    const int64_t u = u_begin + issued;
+    while (u >= jn_end) {
+      ++jn;
+      jn_end = args.m[jn].ubeg + args.m[jn].ntiles;
+    }
+    if (jn != jn_loaded) {
+      ++nq;
+      const int q = nq % kDescRing;
+      mats_sm[q] = args.m[jn];
+      mat_idx[q] = jn;
+      jn_loaded = jn;
+      if constexpr (SYN) {
+        const uint8_t* plan = args.m[jn].plan;
+        const FfbPlanHeader& h = hdr(plan);
+        for (int side = 0; side < 2; ++side) {
+          const uint32_t* mask = table<uint32_t>(plan, side ? h.off_gmask : h.off_zmask);
+          const int G = side ? h.Gn : h.Gm;
+          for (int w = 0; w < (G + 31) / 32; ++w) {
+            uint32_t bits = 0;
+#pragma unroll 8
+            for (int i = 0; i < 32; ++i)
+              if (32 * w + i < G && __ldg(mask + 32 * w + i) != 0u) bits |= 1u << i;
+            mat_bits[q][side][w] = bits;
+          }
+        }
+      }
+    }
+    tile_mat[issued % kDescRing] = nq;
+    const MatK& M = args.m[jn];
+    const int32_t t = static_cast<int32_t>(u - M.ubeg);
+    uint8_t* dst = stg0 + (issued % S) * args.stage;
+    uint64_t* b = bar + (issued % S);
+    mbar_arrive_expect_tx(b, (NEED_V ? 2u * M.n : 0u) + (NEED_U ? 2u * M.m : 0u));
+    if (NEED_V) tma_row3d(dst, &args.maps[2 * jn], t, b);
+    if (NEED_U) tma_row3d(dst + args.xbox_u, &args.maps[2 * jn + 1], t, b);
+    ++issued;
+  };
+  if (tid == kIssuer) {
+    jn = matrix_of(args, 0, u_begin);
+    jn_end = args.m[jn].ubeg + args.m[jn].ntiles;
+    while (issued < S - 1 && issued < count) issue();
+  }
+  tc_fence_before();
+  __syncthreads();  // TMEM address, barriers and the first descriptors are ready
+  tc_fence_after();
+  const uint32_t tmem = tmem_slot;
+
+  if (warp < 4) {
+    // ------------------------------------------------------------ tensor warps
+    {
+      // B operands from the k = 16 group block (the same for every matrix):
+      // analysis B[n = coefficient][k = coordinate] = D4[k][n] as bf16 hi + lo;
+      // synthesis B[n = coordinate][k = coefficient] = D4[n][k] as tf32
+      const MatK& M0 = mats_sm[tile_mat[0] % kDescRing];
+      __nv_bfloat16* bhi = reinterpret_cast<__nv_bfloat16*>(bops);
+      __nv_bfloat16* blo = reinterpret_cast<__nv_bfloat16*>(bops + 2048);
+      float* bsy = reinterpret_cast<float*>(bops + 4096);
+      for (int i = tid; i < 1024; i += 128) {
+        const int r = i >> 5, k = i & 31;
+        const float dk = d4(M0.fval_in, M0.rho_in, k, r);  // D4[k][r]
+        const __nv_bfloat16 hi = __float2bfloat16_rn(dk);
+        const __nv_bfloat16 lo = __float2bfloat16_rn(dk - __bfloat162float(hi));
+        bhi[can_bf16_off(r, k) / 2] = hi;
+        blo[can_bf16_off(r, k) / 2] = lo;
+        bsy[can_f32_off(r, k)] = __uint_as_float(to_tf32(d4(M0.fval_in, M0.rho_in, r, k)));  // D4[r][k]
+      }
+      fence_async_smem();
+      tensor_bar();
+    }
+    const uint32_t id_an = umma_idesc(1, 128, 32), id_sy = umma_idesc(2, 128, 32);
+    const uint64_t d_bhi = umma_sdesc(smem_u32(bops), 128, 512), d_blo = umma_sdesc(smem_u32(bops + 2048), 128, 512);
+    const uint64_t d_bsy = umma_sdesc(smem_u32(bops + 4096), 128, 1024);
+    uint32_t mma_phase = 0;
+    bool failed = false, mma_pending = false;
+    const uint32_t lane_base = static_cast<uint32_t>(32 * warp) << 16;
+    for (int s = 0; s < count + 2; ++s) {
+      if (tid == kIssuer && issued < count) issue();  // tile s + S - 1 into the stage tile s - 1 used
+      const int i2 = s - 2;
+      const bool syn = SYN && i2 >= 0;
+      const bool ana = s < count;
+      // output rows of tile s-2 for this thread's group of the first tile of
+      // each side (read now, used after the MMAs)
+      const MatK* M2 = nullptr;
+      const uint32_t* bits2 = nullptr;
+      int64_t t2 = 0;
+      int Gm2 = 0, Gn2 = 0;
+      uint4 yp[2][4];
+      if (syn) {
+        const int q2 = tile_mat[i2 % kDescRing] % kDescRing;
+        M2 = &mats_sm[q2];
+        bits2 = mat_bits[q2][0];
+        t2 = u_begin + i2 - M2->ubeg;
+        Gm2 = M2->m / FFB_GROUP;
+        Gn2 = M2->n / FFB_GROUP;
+#pragma unroll
+        for (int side = 0; side < 2; ++side) {
+          const bool on = side == 0 ? F : D;
+          const int G = side == 0 ? Gm2 : Gn2;
+          const int r = 32 * warp + lane;
+          const uint32_t* bits = bits2 + side * kGroupWords;
+          if (on && r < G && ((bits[r >> 5] >> (r & 31)) & 1u)) {
+            const __nv_bfloat16* row = side == 0 ? static_cast<const __nv_bfloat16*>(M2->Y) + t2 * M2->ldy
+                                                 : static_cast<const __nv_bfloat16*>(M2->dX) + t2 * M2->ldx;
+            const uint4* p = reinterpret_cast<const uint4*>(row + 32 * r);
+#pragma unroll
+            for (int j = 0; j < 4; ++j) yp[side][j] = p[j];
+          }
+        }
+      }
+      const MatK* M0 = nullptr;
+      int Gn0 = 0, Gm0 = 0;
+      if (ana) {
+        if (!mbar_wait_bounded(bar + (s % S), static_cast<uint32_t>((s / S) & 1))) failed = true;
+        M0 = &mats_sm[tile_mat[s % kDescRing] % kDescRing];
+        Gn0 = M0->n / FFB_GROUP;
+        Gm0 = M0->m / FFB_GROUP;
+      }
+      // one thread issues the MMAs of this step
+      failed = tensor_bar_or(failed);
+      const bool any = (ana || syn) && !failed;
+      if (tid == 0 && any) {
+        tc_fence_after();
+        if (ana) {
+          const uint32_t st0 = smem_u32(stg0 + (s % S) * args.stage);
+#pragma unroll
+          for (int side = 0; side < 2; ++side) {
+            const bool on = side == 0 ? NEED_V : NEED_U;
+            const int G = side == 0 ? Gn0 : Gm0;
+            const uint32_t abase = st0 + (side == 0 ? 0 : args.xbox_u);
+            if (on) {
+              for (int mt = 0; mt * 128 < G; ++mt) {
+                const uint32_t d = tmem + (side * kTcMaxTiles + mt) * 32;
+#pragma unroll
+                for (int ks = 0; ks < 2; ++ks) {
+                  const uint64_t a = umma_sdesc_sw64(abase + mt * 8192 + ks * 32);
+                  umma_f16(d, a, d_bhi + ((ks * 256) >> 4), id_an, ks > 0);
+                  umma_f16(d, a, d_blo + ((ks * 256) >> 4), id_an, 1);
+                }
+              }
+            }
+          }
+        }
+        if (syn) {
+          float* fs2 = fset0 + (i2 & 1) * PL.total;
+#pragma unroll
+          for (int side = 0; side < 2; ++side) {
+            const bool on = side == 0 ? F : D;
+            const int G = side == 0 ? Gm2 : Gn2;
+            const uint64_t abase = umma_sdesc(smem_u32(fs2 + (side == 0 ? PL.oRZ : PL.oRG)), 128, 1024);
+            if (on) {
+              for (int mt = 0; mt * 128 < G; ++mt) {
+                const uint32_t d = tmem + ((2 + side) * kTcMaxTiles + mt) * 32;
+#pragma unroll
+                for (int ks = 0; ks < 4; ++ks)
+                  umma_tf32(d, abase + ((mt * 16 * 1024 + ks * 256) >> 4), d_bsy + ((ks * 256) >> 4), id_sy,
+                            ks > 0);
+              }
+            }
+          }
+        }
+        umma_commit(mma_bar);
+      }
+      if (any) {
+        const bool ok = mbar_wait_bounded(mma_bar, mma_phase);
+        if (ok)
+          mma_phase ^= 1u;
+        else
+          mma_pending = true;
+        failed = tensor_bar_or(!ok);
+        tc_fence_after();
+      }
+      if (!failed) {
+        // analysis results -> V / U (canonical slots), one group per thread
+        if (ana) {
+          float* fs0 = fset0 + (s & 1) * PL.total;
+#pragma unroll
+          for (int side = 0; side < 2; ++side) {
+            const bool on = side == 0 ? NEED_V : NEED_U;
+            const int G = side == 0 ? Gn0 : Gm0;
+            float* dst = fs0 + (side == 0 ? PL.oV : PL.oU);
+            if (on) {
+              for (int mt = 0; mt * 128 < G; ++mt) {
+                float v[32];
+                tmem_ld32(tmem + lane_base + (side * kTcMaxTiles + mt) * 32, v);
+                const int r = mt * 128 + 32 * warp + lane;
+                if (r < G) {
+#pragma unroll
+                  for (int c = 0; c < 8; ++c)
+                    *reinterpret_cast<float4*>(dst + can_f32_off(r, 4 * c)) =
+                        make_float4(v[4 * c], v[4 * c + 1], v[4 * c + 2], v[4 * c + 3]);
+                }
+              }
+            }
+          }
+        }
+        // synthesis results: y += seff * delta for groups with support entries
+        if (syn) {
+#pragma unroll
+          for (int side = 0; side < 2; ++side) {
+            const bool on = side == 0 ? F : D;
+            const int G = side == 0 ? Gm2 : Gn2;
+            const uint32_t* bits = bits2 + side * kGroupWords;
+            if (on) {
+              for (int mt = 0; mt * 128 < G; ++mt) {
+                float v[32];
+                tmem_ld32(tmem + lane_base + ((2 + side) * kTcMaxTiles + mt) * 32, v);
+                const int r = mt * 128 + 32 * warp + lane;
+                if (r < G && ((bits[r >> 5] >> (r & 31)) & 1u)) {
+                  __nv_bfloat16* row = side == 0 ? static_cast<__nv_bfloat16*>(M2->Y) + t2 * M2->ldy
+                                                 : static_cast<__nv_bfloat16*>(M2->dX) + t2 * M2->ldx;
+                  uint4* p = reinterpret_cast<uint4*>(row + 32 * r);
+#pragma unroll
+                  for (int j = 0; j < 4; ++j) {
+                    const uint4 y = mt == 0 ? yp[side][j] : p[j];
+                    p[j] = axpy8(y, v + 8 * j, M2->seff);
+                  }
+                }
+              }
+            }
+          }
+        }
+      }
+      tc_fence_before();
+      if (__syncthreads_or(failed)) break;
+    }
+    if (failed) {
+      if (tid == 0) {
+        atomicAdd(&g_wait_timeouts, 1u);
+        if (mma_pending) mbar_wait_bounded(mma_bar, mma_phase);  // MMAs still in flight (bounded)
+      }
+      if (tid == kIssuer) {
+        // the last tile issued into each stage: let its copy land (bounded)
+        for (int i = issued > S ? issued - S : 0; i < issued; ++i)
+          mbar_wait_bounded(bar + (i % S), static_cast<uint32_t>((i / S) & 1));
+      }
+    }
+  } else {
+    // ------------------------------------------------------------ SpMM warps
+    const int st = tid - 128;
+    Chunk<MODE, true, false> ch;
+    float dc[kEreg];
+#pragma unroll
+    for (int e = 0; e < kEreg; ++e) dc[e] = 0.f;
+    int cur = -1, cur_j = -1;
+    const uint8_t* splan = nullptr;
+    int4* fixc = reinterpret_cast<int4*>(smem + args.fixc);
+    int nfZ = 0, nfix = 0;
+    uint32_t zero_pending = 3u;
+    bool failed = false;
+    for (int s = 0; s < count + 2; ++s) {
+      const int i1 = s - 1;
+      if (i1 >= 0 && i1 < count) {
+        const int q = tile_mat[i1 % kDescRing];
+        const MatK& M1 = mats_sm[q % kDescRing];
+        if (q != cur) {
+          if constexpr (C) {
+            if (cur >= 0) {
+              float* dst = args.partial + static_cast<size_t>(blockIdx.x + cur_j) * args.stride;
+              pipe_flush(splan, dst, dc, st);
+            }
+          }
+          cur = q;
+          cur_j = mat_idx[q % kDescRing];
+          splan = M1.plan;
+          tc_load_chunk<MODE>(ch, splan, M1.c_val, st);
+#pragma unroll
+          for (int e = 0; e < kEreg; ++e) dc[e] = 0.f;
+          zero_pending = 3u;
+          if constexpr (SYN) {
+            const FfbPlanHeader& h = hdr(splan);
+            nfZ = F ? h.nfixZ : 0;
+            nfix = nfZ + (D ? h.nfixG : 0);
+            for (int i = st; i < nfix; i += kTcSpmm)
+              fixc[i] = i < nfZ ? __ldg(table<int4>(splan, h.off_fixZ) + i)
+                                : __ldg(table<int4>(splan, h.off_fixG) + (i - nfZ));
+            tc_spmm_bar();
+          }
+        }
+        float* fs1 = fset0 + (i1 & 1) * PL.total;
+        if constexpr (SYN) {
+          if ((zero_pending >> (i1 & 1)) & 1u) {
+            for (int x = PL.oRZ + st; x < PL.total; x += kTcSpmm) fs1[x] = 0.f;
+            zero_pending &= ~(1u << (i1 & 1));
+            tc_spmm_bar();
+          }
+        }
+        tc_spmm<MODE>(ch, dc, fs1, PL);
+        if constexpr (SYN) {
+          if (nfix > 0) {
+            tc_spmm_bar();
+            for (int i = st; i < nfix; i += kTcSpmm) {
+              const int4 it = fixc[i];
+              const bool z = i < nfZ;
+              float* R = fs1 + (z ? PL.oRZ : PL.oRG);
+              const int dst = tc_slot(it.x, z ? M1.m : M1.n);
+              float sacc = R[dst];
+              for (int c2 = 0; c2 < it.z; ++c2) sacc += R[it.y + c2];
+              R[dst] = sacc;
+            }
+          }
+          fence_async_smem();  // RZ / RG are read by the tensor cores next step
+        }
+      }
+      if (__syncthreads_or(false)) {
+        failed = true;
+        break;
+      }
+    }
+    if (!failed) {
+      if constexpr (C) {
+        if (cur >= 0) {
+          float* dst = args.partial + static_cast<size_t>(blockIdx.x + cur_j) * args.stride;
+          pipe_flush(splan, dst, dc, st);
+        }
+      }
+    }
+  }
+  // every thread is past its last TMEM access
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTcTmemCols) : "memory");
+  }
+}
+
+}  // namespace ffb

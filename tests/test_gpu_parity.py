@@ -68,7 +68,7 @@ def test_single_256_fp32(ops, unit):
     check_batch(b, ops)
 
 
-@pytest.mark.parametrize("kernel", ["tile", "pipe"])
+@pytest.mark.parametrize("kernel", ["tile", "pipe", "tc"])
 @pytest.mark.parametrize("N", [37, 1, 4])
 def test_roberta_base_all_matrices(N, kernel, monkeypatch):
     monkeypatch.setenv("FRAMEFB_KERNEL", kernel)
@@ -77,7 +77,7 @@ def test_roberta_base_all_matrices(N, kernel, monkeypatch):
     check_batch(b, ALL)
 
 
-@pytest.mark.parametrize("kernel", ["tile", "pipe"])
+@pytest.mark.parametrize("kernel", ["tile", "pipe", "tc"])
 def test_vit_b16_mixed_shapes(kernel, monkeypatch):
     # many matrices of three shapes per launch: CTAs cross matrix boundaries
     monkeypatch.setenv("FRAMEFB_KERNEL", kernel)
@@ -94,12 +94,13 @@ def test_llama2_shape_small_n():
     check_batch(b, ALL)
 
 
-@pytest.mark.parametrize("kernel", ["pipe", "tile"])
+@pytest.mark.parametrize("kernel", ["tc", "pipe", "tile"])
 @pytest.mark.parametrize("ops", [ffb.OP_FORWARD, ffb.OP_BACKWARD_DX, ffb.OP_GRAD_COEFF,
                                  ffb.OP_BACKWARD_DX | ffb.OP_GRAD_COEFF, ALL])
 def test_bf16_kernels_every_mode(kernel, ops, monkeypatch):
     # FRAMEFB_KERNEL selects the bf16 kernel: the one-phase-at-a-time tile
-    # kernel (two tokens per tile here, the default) or the pipelined one
+    # kernel (two tokens per tile here, the default), the warp-MMA pipelined
+    # kernel or the tcgen05 pipelined kernel
     monkeypatch.setenv("FRAMEFB_KERNEL", kernel)
     w = wl.WORKLOADS["llama2_7b_qkvo"]
     b = AdapterBatch(w, DEV, N=13, indices=[0, 5], ops=ops)
