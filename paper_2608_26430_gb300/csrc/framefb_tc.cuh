@@ -6,10 +6,13 @@
 // pipe_tile_kernel (step s: analysis of tile s and synthesis of tile s-2 on
 // the tensor side, coefficient SpMM of tile s-1, one barrier per step), with
 // these differences:
-//   * the group contractions are UMMA instructions issued by one thread:
-//       analysis   V (M = 128 groups x N = 32 coefficients) = X_rows (K = 32
-//                  coordinates, bf16) x D, D split into bf16 hi + lo parts
-//                  (kind::f16, fp32 accumulate in TMEM);
+//   * the group contractions are UMMA instructions, issued by four threads
+//     in parallel (one per operand side; a single issuing thread spends about
+//     150 cycles per instruction at these small shapes):
+//       analysis   [V D_hi | V D_lo] (M = 128 groups x N = 64) = X_rows (K = 32
+//                  coordinates, bf16) x [D_hi | D_lo], D split into bf16 hi +
+//                  lo parts side by side (kind::f16, fp32 accumulate in TMEM),
+//                  the two halves added when read back;
 //       synthesis  dY_rows (M = 128 groups x N = 32 coordinates) = Z (K = 32
 //                  coefficients, fp32 read as tf32) x D^T (kind::tf32);
 //     the results are read back with tcgen05.ld, one TMEM lane per group;
@@ -36,7 +39,10 @@ namespace ffb {
 constexpr int kTcThreads = 384;            // 4 tensor warps + 8 SpMM warps
 constexpr int kTcSpmm = kTcThreads - 128;  // SpMM threads (= plan columns)
 constexpr int kTcMaxTiles = 2;             // 128-group tiles per side
-constexpr uint32_t kTcTmemCols = 256;      // 4 sides x 2 tiles x 32 columns
+// TMEM columns: analysis (X, dY) x 2 tiles x 64 (hi | lo), then synthesis
+// (Y, dX) x 2 tiles x 32
+constexpr uint32_t kTcTmemCols = 512;
+constexpr uint32_t kTcColSyn = 256;
 
 static_assert(kTcSpmm == kThreads, "one SpMM thread per plan column");
 
@@ -118,6 +124,25 @@ __device__ __forceinline__ bool tensor_bar_or(bool f) {
   return out != 0;
 }
 __device__ __forceinline__ void tc_spmm_bar() { asm volatile("bar.sync 1, %0;" ::"n"(kTcSpmm) : "memory"); }
+
+// Completion test of phase `parity` that never suspends the thread.
+__device__ __forceinline__ bool mbar_test_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// Bounded wait with a non-suspending first test (the common case here: the
+// phase completed long ago).
+__device__ __forceinline__ bool tc_wait_bounded(uint64_t* bar, uint32_t parity) {
+  return mbar_test_wait(bar, parity) || mbar_wait_bounded(bar, parity);
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
 
 // 32 consecutive fp32 columns of this thread's TMEM lane.
 __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
@@ -314,7 +339,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc_tile_kernel(const __grid_con
   if (count <= 0) return;
 
   if (tid == 0) {
-    for (int b = 0; b <= S; ++b) mbar_init(bar + b, 1);
+    for (int b = 0; b < S; ++b) mbar_init(bar + b, 1);
+    mbar_init(mma_bar, 4);  // the four MMA issuers
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (warp == 0) {
@@ -379,26 +405,27 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc_tile_kernel(const __grid_con
     // ------------------------------------------------------------ tensor warps
     {
       // B operands from the k = 16 group block (the same for every matrix):
-      // analysis B[n = coefficient][k = coordinate] = D4[k][n] as bf16 hi + lo;
-      // synthesis B[n = coordinate][k = coefficient] = D4[n][k] as tf32
+      // analysis B[n][k = coordinate], n < 32: D4[k][n] rounded to bf16 (hi),
+      // n >= 32: the bf16 remainder D4[k][n - 32] - hi (lo), so that one
+      // N = 64 MMA gives both partial products; synthesis B[n = coordinate]
+      // [k = coefficient] = D4[n][k] as tf32
       const MatK& M0 = mats_sm[tile_mat[0] % kDescRing];
-      __nv_bfloat16* bhi = reinterpret_cast<__nv_bfloat16*>(bops);
-      __nv_bfloat16* blo = reinterpret_cast<__nv_bfloat16*>(bops + 2048);
+      __nv_bfloat16* ban = reinterpret_cast<__nv_bfloat16*>(bops);
       float* bsy = reinterpret_cast<float*>(bops + 4096);
       for (int i = tid; i < 1024; i += 128) {
         const int r = i >> 5, k = i & 31;
         const float dk = d4(M0.fval_in, M0.rho_in, k, r);  // D4[k][r]
         const __nv_bfloat16 hi = __float2bfloat16_rn(dk);
         const __nv_bfloat16 lo = __float2bfloat16_rn(dk - __bfloat162float(hi));
-        bhi[can_bf16_off(r, k) / 2] = hi;
-        blo[can_bf16_off(r, k) / 2] = lo;
+        ban[can_bf16_off(r, k) / 2] = hi;
+        ban[can_bf16_off(32 + r, k) / 2] = lo;
         bsy[can_f32_off(r, k)] = __uint_as_float(to_tf32(d4(M0.fval_in, M0.rho_in, r, k)));  // D4[r][k]
       }
       fence_async_smem();
       tensor_bar();
     }
-    const uint32_t id_an = umma_idesc(1, 128, 32), id_sy = umma_idesc(2, 128, 32);
-    const uint64_t d_bhi = umma_sdesc(smem_u32(bops), 128, 512), d_blo = umma_sdesc(smem_u32(bops + 2048), 128, 512);
+    const uint32_t id_an = umma_idesc(1, 128, 64), id_sy = umma_idesc(2, 128, 32);
+    const uint64_t d_ban = umma_sdesc(smem_u32(bops), 128, 512);
     const uint64_t d_bsy = umma_sdesc(smem_u32(bops + 4096), 128, 1024);
     uint32_t mma_phase = 0;
     bool failed = false, mma_pending = false;
@@ -440,58 +467,49 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc_tile_kernel(const __grid_con
       const MatK* M0 = nullptr;
       int Gn0 = 0, Gm0 = 0;
       if (ana) {
-        if (!mbar_wait_bounded(bar + (s % S), static_cast<uint32_t>((s / S) & 1))) failed = true;
+        if (!tc_wait_bounded(bar + (s % S), static_cast<uint32_t>((s / S) & 1))) failed = true;
         M0 = &mats_sm[tile_mat[s % kDescRing] % kDescRing];
         Gn0 = M0->n / FFB_GROUP;
         Gm0 = M0->m / FFB_GROUP;
       }
-      // one thread issues the MMAs of this step
+      // four threads issue the MMAs of this step, one per operand side:
+      // thread 0 analysis of X, 32 of dY, 64 synthesis of Y, 96 of dX; each
+      // commits (or just arrives) on the 4-count MMA barrier
       failed = tensor_bar_or(failed);
       const bool any = (ana || syn) && !failed;
-      if (tid == 0 && any) {
-        tc_fence_after();
-        if (ana) {
-          const uint32_t st0 = smem_u32(stg0 + (s % S) * args.stage);
-#pragma unroll
-          for (int side = 0; side < 2; ++side) {
-            const bool on = side == 0 ? NEED_V : NEED_U;
+      if (lane == 0 && any) {
+        const int side = warp & 1;
+        const bool is_ana = warp < 2;
+        const bool on = is_ana ? (ana && (side == 0 ? NEED_V : NEED_U)) : (syn && (side == 0 ? F : D));
+        if (on) {
+          tc_fence_after();
+          if (is_ana) {
             const int G = side == 0 ? Gn0 : Gm0;
-            const uint32_t abase = st0 + (side == 0 ? 0 : args.xbox_u);
-            if (on) {
-              for (int mt = 0; mt * 128 < G; ++mt) {
-                const uint32_t d = tmem + (side * kTcMaxTiles + mt) * 32;
+            const uint32_t abase = smem_u32(stg0 + (s % S) * args.stage) + (side == 0 ? 0 : args.xbox_u);
+            for (int mt = 0; mt * 128 < G; ++mt) {
+              const uint32_t d = tmem + (side * kTcMaxTiles + mt) * 64;
 #pragma unroll
-                for (int ks = 0; ks < 2; ++ks) {
-                  const uint64_t a = umma_sdesc_sw64(abase + mt * 8192 + ks * 32);
-                  umma_f16(d, a, d_bhi + ((ks * 256) >> 4), id_an, ks > 0);
-                  umma_f16(d, a, d_blo + ((ks * 256) >> 4), id_an, 1);
-                }
-              }
+              for (int ks = 0; ks < 2; ++ks)
+                umma_f16(d, umma_sdesc_sw64(abase + mt * 8192 + ks * 32), d_ban + ((ks * 256) >> 4), id_an, ks > 0);
             }
-          }
-        }
-        if (syn) {
-          float* fs2 = fset0 + (i2 & 1) * PL.total;
-#pragma unroll
-          for (int side = 0; side < 2; ++side) {
-            const bool on = side == 0 ? F : D;
+          } else {
+            float* fs2 = fset0 + (i2 & 1) * PL.total;
             const int G = side == 0 ? Gm2 : Gn2;
             const uint64_t abase = umma_sdesc(smem_u32(fs2 + (side == 0 ? PL.oRZ : PL.oRG)), 128, 1024);
-            if (on) {
-              for (int mt = 0; mt * 128 < G; ++mt) {
-                const uint32_t d = tmem + ((2 + side) * kTcMaxTiles + mt) * 32;
+            for (int mt = 0; mt * 128 < G; ++mt) {
+              const uint32_t d = tmem + kTcColSyn + (side * kTcMaxTiles + mt) * 32;
 #pragma unroll
-                for (int ks = 0; ks < 4; ++ks)
-                  umma_tf32(d, abase + ((mt * 16 * 1024 + ks * 256) >> 4), d_bsy + ((ks * 256) >> 4), id_sy,
-                            ks > 0);
-              }
+              for (int ks = 0; ks < 4; ++ks)
+                umma_tf32(d, abase + ((mt * 16 * 1024 + ks * 256) >> 4), d_bsy + ((ks * 256) >> 4), id_sy, ks > 0);
             }
           }
+          umma_commit(mma_bar);
+        } else {
+          mbar_arrive(mma_bar);
         }
-        umma_commit(mma_bar);
       }
       if (any) {
-        const bool ok = mbar_wait_bounded(mma_bar, mma_phase);
+        const bool ok = tc_wait_bounded(mma_bar, mma_phase);
         if (ok)
           mma_phase ^= 1u;
         else
@@ -510,14 +528,17 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc_tile_kernel(const __grid_con
             float* dst = fs0 + (side == 0 ? PL.oV : PL.oU);
             if (on) {
               for (int mt = 0; mt * 128 < G; ++mt) {
-                float v[32];
-                tmem_ld32(tmem + lane_base + (side * kTcMaxTiles + mt) * 32, v);
+                float v[32], w[32];
+                const uint32_t col = tmem + lane_base + (side * kTcMaxTiles + mt) * 64;
+                tmem_ld32(col, v);       // X D_hi
+                tmem_ld32(col + 32, w);  // X D_lo
                 const int r = mt * 128 + 32 * warp + lane;
                 if (r < G) {
 #pragma unroll
                   for (int c = 0; c < 8; ++c)
                     *reinterpret_cast<float4*>(dst + can_f32_off(r, 4 * c)) =
-                        make_float4(v[4 * c], v[4 * c + 1], v[4 * c + 2], v[4 * c + 3]);
+                        make_float4(v[4 * c] + w[4 * c], v[4 * c + 1] + w[4 * c + 1], v[4 * c + 2] + w[4 * c + 2],
+                                    v[4 * c + 3] + w[4 * c + 3]);
                 }
               }
             }
@@ -533,7 +554,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc_tile_kernel(const __grid_con
             if (on) {
               for (int mt = 0; mt * 128 < G; ++mt) {
                 float v[32];
-                tmem_ld32(tmem + lane_base + ((2 + side) * kTcMaxTiles + mt) * 32, v);
+                tmem_ld32(tmem + lane_base + kTcColSyn + (side * kTcMaxTiles + mt) * 32, v);
                 const int r = mt * 128 + 32 * warp + lane;
                 if (r < G && ((bits[r >> 5] >> (r & 31)) & 1u)) {
                   __nv_bfloat16* row = side == 0 ? static_cast<__nv_bfloat16*>(M2->Y) + t2 * M2->ldy
