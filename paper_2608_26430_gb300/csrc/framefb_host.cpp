@@ -302,43 +302,101 @@ inline int32_t group_major(int32_t c, int32_t rho) {
 
 struct Entry { int32_t key0, key1, q; };
 
-// Cut `ent` (sorted by key0, key1) into P chunks of E entries.  Each run of
-// equal key0 inside a chunk stores its partial sum once, at its last entry:
-// the first run of a key goes to that key's own slot (target = key0); later
-// runs (the key continues from an earlier chunk) go to overflow slots
-// base + o (targets >= base).
-// Returns per-entry store targets and the fix-up list.
-void cut_chunks(const std::vector<Entry>& ent, int32_t P, int32_t E, int32_t base, int32_t nkeys,
-                std::vector<int32_t>& store, std::vector<int32_t>& fix, int32_t& novf) {
+// Arrange `ent` (sorted by key0, key1) into P chunks of E entries so that
+// every run of equal key0 stays inside one chunk where its length allows:
+// runs longer than E first fill whole chunks, then the pieces go, longest
+// first, to the chunk whose free room fits them most tightly (best fit
+// decreasing); a piece that fits nowhere is split over the roomiest chunks.
+// A chunk's pieces are consecutive, so each piece sums in registers and
+// stores once, at its last entry: the first piece of a key (in chunk order)
+// writes the key's own slot, later pieces write overflow slots base + o,
+// contiguous per key, which the fix-up list {key, first overflow slot, count,
+// 0} adds in.  With no run longer than E and enough room, nothing overflows.
+// Outputs: pos[p * E + e] = entry index or -1 (padding at chunk ends),
+// store[entry] = its store target or FFB_NO_STORE.
+void pack_runs(const std::vector<Entry>& ent, int32_t P, int32_t E, int32_t base, int32_t nkeys,
+               std::vector<int32_t>& pos, std::vector<int32_t>& store, std::vector<int32_t>& fix, int32_t& novf) {
   const int32_t nnz = static_cast<int32_t>(ent.size());
+  pos.assign(static_cast<size_t>(P) * E, -1);
   store.assign(nnz, FFB_NO_STORE);
-  std::vector<uint8_t> seen(nkeys, 0);
-  std::vector<int32_t> first_ovf(nkeys, -1), n_ovf(nkeys, 0);
+  fix.clear();
   novf = 0;
-  for (int32_t p = 0; p < P; ++p) {
-    const int32_t lo = p * E, hi = std::min(nnz, (p + 1) * E);
-    for (int32_t e = lo; e < hi; ++e) {
-      const bool run_end = (e + 1 == hi) || ent[e + 1].key0 != ent[e].key0;
-      if (!run_end) continue;
-      const int32_t key = ent[e].key0;
-      if (!seen[key]) {
-        seen[key] = 1;
-        store[e] = key;
-      } else {
-        if (first_ovf[key] < 0) first_ovf[key] = novf;
-        n_ovf[key]++;
-        store[e] = base + novf;
-        ++novf;
+  if (nnz == 0 || E == 0) return;
+  struct Piece { int32_t start, len; };
+  std::vector<Piece> pieces;
+  std::vector<std::vector<Piece>> chunk(P);
+  std::vector<int32_t> room(P, E);
+  int32_t next_full = 0;  // chunks handed out whole to long runs
+  for (int32_t i = 0; i < nnz;) {
+    int32_t j = i + 1;
+    while (j < nnz && ent[j].key0 == ent[i].key0) ++j;
+    int32_t start = i, len = j - i;
+    while (len >= E && next_full < P) {
+      chunk[next_full].push_back(Piece{start, E});
+      room[next_full++] = 0;
+      start += E;
+      len -= E;
+    }
+    if (len > 0) pieces.push_back(Piece{start, len});
+    i = j;
+  }
+  std::stable_sort(pieces.begin(), pieces.end(), [](const Piece& x, const Piece& y) { return x.len > y.len; });
+  // bucket[c] = chunks with free room c (taken from the back)
+  std::vector<std::vector<int32_t>> bucket(E + 1);
+  for (int32_t c = P - 1; c >= next_full; --c) bucket[E].push_back(c);
+  auto take = [&](int32_t c) {
+    const int32_t id = bucket[c].back();
+    bucket[c].pop_back();
+    return id;
+  };
+  for (size_t k = 0; k < pieces.size(); ++k) {
+    Piece pc = pieces[k];
+    while (pc.len > 0) {
+      int32_t c = pc.len;
+      while (c <= E && bucket[c].empty()) ++c;
+      if (c > E) {  // nowhere whole: fill the roomiest chunk and go on with the rest
+        c = pc.len - 1;
+        while (c > 0 && bucket[c].empty()) --c;
+        if (c == 0) return;  // cannot happen: P * E >= nnz
       }
+      const int32_t id = take(c);
+      const int32_t put = std::min(pc.len, c);
+      chunk[id].push_back(Piece{pc.start, put});
+      room[id] = c - put;
+      bucket[room[id]].push_back(id);
+      pc.start += put;
+      pc.len -= put;
     }
   }
-  fix.clear();
+  // positions, piece ends, own / overflow targets
+  std::vector<int32_t> first_chunk_end(nkeys, -1), n_ovf(nkeys, 0), first_ovf(nkeys, 0);
+  std::vector<int32_t> ends;
+  for (int32_t p = 0; p < P; ++p) {
+    int32_t e = 0;
+    for (const Piece& pc : chunk[p]) {
+      for (int32_t t = 0; t < pc.len; ++t) pos[static_cast<size_t>(p) * E + e++] = pc.start + t;
+      const int32_t last = pc.start + pc.len - 1;
+      const int32_t key = ent[last].key0;
+      if (first_chunk_end[key] < 0)
+        first_chunk_end[key] = last;
+      else
+        ++n_ovf[key];
+      ends.push_back(last);
+    }
+  }
   for (int32_t key = 0; key < nkeys; ++key) {
     if (n_ovf[key] == 0) continue;
+    first_ovf[key] = novf;
     fix.push_back(key);
-    fix.push_back(base + first_ovf[key]);
+    fix.push_back(base + novf);
     fix.push_back(n_ovf[key]);
     fix.push_back(0);
+    novf += n_ovf[key];
+  }
+  std::vector<int32_t> used(nkeys, 0);
+  for (int32_t last : ends) {
+    const int32_t key = ent[last].key0;
+    store[last] = last == first_chunk_end[key] ? key : base + first_ovf[key] + used[key]++;
   }
 }
 
@@ -380,10 +438,10 @@ extern "C" framefb_status framefb_plan_build(const framefb_frame* fin, const fra
     std::sort(bycol.begin(), bycol.end(), lt);
     const int32_t EZ = (nz + P - 1) / P, EG = EZ;
 
-    std::vector<int32_t> storeZ, fixZ, storeG, fixG;
+    std::vector<int32_t> posZ, storeZ, fixZ, posG, storeG, fixG;
     int32_t novfZ = 0, novfG = 0;
-    cut_chunks(byrow, P, EZ, m, m, storeZ, fixZ, novfZ);
-    cut_chunks(bycol, P, EG, n, n, storeG, fixG, novfG);
+    pack_runs(byrow, P, EZ, m, m, posZ, storeZ, fixZ, novfZ);
+    pack_runs(bycol, P, EG, n, n, posG, storeG, fixG, novfG);
 
     FfbPlanHeader h;
     std::memset(&h, 0, sizeof(h));
@@ -435,9 +493,9 @@ extern "C" framefb_status framefb_plan_build(const framefb_frame* fin, const fra
     int32_t* gq = arr(h.off_gq);
     for (int32_t p = 0; p < P; ++p) {
       for (int32_t e = 0; e < EZ; ++e) {
-        const int32_t idx = p * EZ + e;
+        const int32_t idx = posZ[static_cast<size_t>(p) * EZ + e];
         const size_t slot = static_cast<size_t>(e) * P + p;
-        if (idx < nz) {
+        if (idx >= 0) {
           zb[slot] = byrow[idx].key1 | ((byrow[idx].key0 & 1) << 15) | (storeZ[idx] << 16);
           zq[slot] = byrow[idx].q;
         } else {
@@ -446,9 +504,9 @@ extern "C" framefb_status framefb_plan_build(const framefb_frame* fin, const fra
         }
       }
       for (int32_t e = 0; e < EG; ++e) {
-        const int32_t idx = p * EG + e;
+        const int32_t idx = posG[static_cast<size_t>(p) * EG + e];
         const size_t slot = static_cast<size_t>(e) * P + p;
-        if (idx < nz) {
+        if (idx >= 0) {
           ga[slot] = bycol[idx].key1 | ((bycol[idx].key0 & 1) << 15) | (storeG[idx] << 16);
           gb[slot] = bycol[idx].key0;
           gq[slot] = bycol[idx].q;
