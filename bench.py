@@ -35,7 +35,7 @@ def parse():
     p.add_argument("--workload", default=None)
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu", action="store_true")
-    p.add_argument("--cpu-tokens", type=int, default=1024, help="token sample of the CPU oracle baseline")
+    p.add_argument("--cpu-tokens", type=int, default=8192, help="token sample of the CPU oracle baseline")
     p.add_argument("--mats", type=int, default=None, help="first MATS matrices only (small profiling cases)")
     return p.parse_args()
 
@@ -121,17 +121,37 @@ def algorithmic_bytes(batch) -> int:
     return total
 
 
+# sources of the dominant kernel (bf16: the tcgen05 kernel unless FRAMEFB_KERNEL forces another)
+KERNEL_SOURCES = ("framefb_kernels.cuh", "framefb_mma.cuh", "framefb_pipe.cuh", "framefb_tc.cuh", "plan_layout.h")
+
+
+def kernel_choice():
+    k = os.environ.get("FRAMEFB_KERNEL", "tc")
+    return k if k in ("tile", "pipe") else "tc"
+
+
+def launches_per_step(nmats: int) -> int:
+    """Kernel launches of one fused step: a tile kernel and a dC reduction per
+    launch chunk (the tcgen05 kernel takes 64 matrices per launch, the others 256)."""
+    chunk = 64 if kernel_choice() == "tc" else 256
+    return 2 * ((nmats + chunk - 1) // chunk)
+
+
 def measured_traffic():
-    """ncu DRAM bytes per launch of the dominant kernel, if taken on the current kernel source."""
+    """ncu DRAM bytes per launch of the dominant kernel, if taken on the current
+    kernel sources with the same kernel choice."""
     import hashlib
     try:
         csrc = os.path.join(ROOT, "paper_2608_26430_gb300", "csrc")
         hh = hashlib.sha256()
-        for name in ("framefb_kernels.cuh", "framefb_mma.cuh", "plan_layout.h"):
+        for name in KERNEL_SOURCES:
             hh.update(open(os.path.join(csrc, name), "rb").read())
         h = hh.hexdigest()[:16]
         with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
-            return json.load(f).get(h, {}).get("bytes_per_launch")
+            rec = json.load(f).get(h, {})
+        if rec.get("kernel_choice") != kernel_choice():
+            return None
+        return rec.get("bytes_per_launch")
     except Exception:
         return None
 
@@ -252,7 +272,8 @@ def main():
     value = w.N * world / (ms_step / 1e3)
     kernel_ms = statistics.mean(kern_ms)
     peak, peak_kind = peaks()
-    achieved = alg / (kernel_ms / 1e3) / 1e9
+    achieved = alg / (kernel_ms / 1e3) / 1e9  # = bytes per launch / time per launch (equal launches)
+    launches = launches_per_step(len(batch.bufs)) // 2
 
     # end to end through the same C-ABI call with host buffers: per step the
     # inputs X and dY are copied from pinned host memory and dC read back
@@ -308,9 +329,12 @@ def main():
                "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                             "frac": achieved / peak,
                             "traffic": measured_traffic() if args.mats is None and args.workload is None else None, "peak_kind": peak_kind,
-                            "kernel": "mma_tile_kernel<fwd|dx|dc> + dc_reduce", "kernel_ms": kernel_ms,
-                            "algorithmic_bytes": alg, "frac_of_8tbs": achieved / 8000.0},
-               "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": 2 * args.steps,
+                            "kernel": {"tc": "tc_tile_kernel<fwd|dx|dc>", "pipe": "pipe_tile_kernel<fwd|dx|dc>",
+                                       "tile": "mma_tile_kernel<fwd|dx|dc>"}[kernel_choice()] + " + dc_reduce",
+                            "kernel_ms": kernel_ms,
+                            "algorithmic_bytes": alg, "algorithmic_bytes_per_launch": alg / launches,
+                            "launches_per_step": launches, "frac_of_8tbs": achieved / 8000.0},
+               "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches_per_step(len(batch.bufs)) * args.steps,
                "clocks": clk.summary()}
         print(json.dumps(out), flush=True)
     if world > 1:

@@ -271,15 +271,17 @@ bool encode_rows(CUtensorMap* map, const void* base, int32_t d, int32_t N, int64
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// Kernel choice for bf16 (FRAMEFB_KERNEL): "tc" the tensor-core pipelined
-// kernel, "pipe" the warp-MMA pipelined kernel, where they apply; by default
-// the one-phase-at-a-time tile kernel runs.
+// Kernel choice for bf16: the tensor-core pipelined kernel wherever it
+// applies (register-resident plans, group counts a multiple of 8 and at most
+// 256, its shared-memory map fits), else the one-phase-at-a-time tile
+// kernel.  FRAMEFB_KERNEL=tile or =pipe forces the tile kernel or the
+// warp-MMA pipelined kernel instead (for comparison and tests).
 bool kernel_is(const char* name) {
   const char* e = std::getenv("FRAMEFB_KERNEL");
   return e && std::strcmp(e, name) == 0;
 }
 bool pipe_allowed() { return kernel_is("pipe"); }
-bool tc_allowed() { return kernel_is("tc"); }
+bool tc_allowed() { return !kernel_is("tile") && !kernel_is("pipe"); }
 
 // Validate one chunk of matrices and fill the launch parameters.
 framefb_status prepare(const framefb_mat* mats, int32_t nmats, int32_t ops, framefb_dtype dt, Prepared& P) {
@@ -467,9 +469,22 @@ struct Buffers {
   }
 };
 
-// Matrices per launch: the tensor-core kernel carries tensor maps in its
-// parameters and takes fewer.
-int32_t chunk_mats(framefb_dtype dt) { return (dt == FRAMEFB_BF16 && tc_allowed()) ? ffb::kTcMaxMats : kMaxMats; }
+// Matrices in the launch that starts at `mats` (`rest` left): the
+// tensor-core kernel carries tensor maps in its parameters and takes at most
+// kTcMaxMats; the chunk is that short only when the kernel applies to it.
+int32_t chunk_len(const framefb_mat* mats, int32_t rest, framefb_dtype dt) {
+  if (dt == FRAMEFB_BF16 && tc_allowed()) {
+    const int32_t k = std::min(rest, ffb::kTcMaxMats);
+    bool ok = true;
+    for (int32_t j = 0; j < k && ok; ++j) {
+      const FfbPlanHeader* h = plan_header(mats[j].plan);
+      ok = h && h->EZ <= ffb::kEreg && h->EG <= ffb::kEreg && h->Gn % 8 == 0 && h->Gm % 8 == 0 &&
+           h->Gn <= 128 * ffb::kTcMaxTiles && h->Gm <= 128 * ffb::kTcMaxTiles;
+    }
+    if (ok) return k;
+  }
+  return std::min(rest, kMaxMats);
+}
 
 bool ops_ok(int32_t ops) { return ops == 1 || ops == 2 || ops == 4 || ops == 6 || ops == 7; }
 
@@ -479,13 +494,16 @@ extern "C" size_t framefb_workspace_size(const framefb_mat* mats, int32_t nmats,
   if (!mats || nmats <= 0 || !ops_ok(ops)) return 0;
   Buffers b;
   size_t need = 0;
-  const int32_t cm = chunk_mats(FRAMEFB_BF16);
-  for (int32_t j0 = 0; j0 < nmats; j0 += cm) {
-    Prepared P = b.prep();
-    // the workspace depends on the launch chunking and the grid; bf16 is used
-    // for the occupancy query (the fp32 kernels run with the same grid bound)
-    if (prepare(mats + j0, std::min(cm, nmats - j0), ops, FRAMEFB_BF16, P) != FRAMEFB_OK) return 0;
-    need = std::max(need, P.ws_bytes);
+  // the workspace depends on the launch chunking, which depends on the dtype:
+  // the larger of the two (bf16 is used for the occupancy query, the fp32
+  // kernels run with the same grid bound)
+  for (const framefb_dtype dt : {FRAMEFB_BF16, FRAMEFB_F32}) {
+    for (int32_t j0 = 0, nm = 0; j0 < nmats; j0 += nm) {
+      nm = chunk_len(mats + j0, nmats - j0, dt);
+      Prepared P = b.prep();
+      if (prepare(mats + j0, nm, ops, FRAMEFB_BF16, P) != FRAMEFB_OK) return 0;
+      need = std::max(need, P.ws_bytes);
+    }
   }
   return need;
 }
@@ -497,19 +515,19 @@ extern "C" framefb_status framefb_run(const framefb_mat* mats, int32_t nmats, in
   if (nmats == 0) return FRAMEFB_OK;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   Buffers b;
-  const int32_t cm = chunk_mats(dtype);
   // validate every chunk before queueing anything
-  for (int32_t j0 = 0; j0 < nmats; j0 += cm) {
+  for (int32_t j0 = 0, nm = 0; j0 < nmats; j0 += nm) {
+    nm = chunk_len(mats + j0, nmats - j0, dtype);
     Prepared P = b.prep();
-    const framefb_status s = prepare(mats + j0, std::min(cm, nmats - j0), ops, dtype, P);
+    const framefb_status s = prepare(mats + j0, nm, ops, dtype, P);
     if (s != FRAMEFB_OK) return s;
     if (P.ws_bytes > 0) {
       if (!ws || ws_bytes < P.ws_bytes) return FRAMEFB_EWORKSPACE;
       if (reinterpret_cast<uintptr_t>(ws) & 255u) return FRAMEFB_EINVAL;
     }
   }
-  for (int32_t j0 = 0; j0 < nmats; j0 += cm) {
-    const int32_t nm = std::min(cm, nmats - j0);
+  for (int32_t j0 = 0, nm = 0; j0 < nmats; j0 += nm) {
+    nm = chunk_len(mats + j0, nmats - j0, dtype);
     Prepared P = b.prep();
     const framefb_status s = prepare(mats + j0, nm, ops, dtype, P);
     if (s != FRAMEFB_OK) return s;
