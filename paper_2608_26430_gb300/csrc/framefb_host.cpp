@@ -302,20 +302,40 @@ inline int32_t group_major(int32_t c, int32_t rho) {
 
 struct Entry { int32_t key0, key1, q; };
 
+// Bank (4-byte word mod 32) of the fp32 slot of group-major index x in the
+// tensor-core kernel's coefficient buffers (canonical K-major core-matrix
+// layout: group r, coefficient c at 256 (r / 8) + 32 (c / 4) + 4 (r % 8) +
+// c % 4 floats); overflow slots x >= K sit at x.
+inline int32_t slot_bank(int32_t x, int32_t K) { return x >= K ? (x & 31) : (((x >> 5) & 7) * 4 + (x & 3)); }
+
+// Shared-memory banks one coefficient path touches per entry: the gather of
+// the other index, the reload of the key's own input where the key changes
+// (dC, column path only) and the run-sum store at a piece end.
+struct PathBanks {
+  std::vector<int8_t> gather, key, store;  // per entry; key empty: no reload
+};
+
 // Arrange `ent` (sorted by key0, key1) into P chunks of E entries so that
 // every run of equal key0 stays inside one chunk where its length allows:
 // runs longer than E first fill whole chunks, then the pieces go, longest
 // first, to the chunk whose free room fits them most tightly (best fit
 // decreasing); a piece that fits nowhere is split over the roomiest chunks.
+// The pieces are then moved (equal-length pieces swapped between chunks,
+// entries reordered inside a piece) by a deterministic annealing search that
+// lowers shared-memory bank conflicts: for every SpMM instruction (32
+// consecutive chunks at one entry step) it counts the lanes that share a bank
+// with an earlier lane, over the gathers, the key reloads and the stores.
 // A chunk's pieces are consecutive, so each piece sums in registers and
-// stores once, at its last entry: the first piece of a key (in chunk order)
-// writes the key's own slot, later pieces write overflow slots base + o,
-// contiguous per key, which the fix-up list {key, first overflow slot, count,
-// 0} adds in.  With no run longer than E and enough room, nothing overflows.
-// Outputs: pos[p * E + e] = entry index or -1 (padding at chunk ends),
-// store[entry] = its store target or FFB_NO_STORE.
+// stores once, at its last position: the first piece of a key (in chunk
+// order) writes the key's own slot, later pieces write overflow slots
+// base + o, contiguous per key, which the fix-up list {key, first overflow
+// slot, count, 0} adds in.  With no run longer than E and enough room,
+// nothing overflows.
+// Outputs: pos[p * E + e] = entry index or -1 (padding), store[entry] = its
+// store target or FFB_NO_STORE.
 void pack_runs(const std::vector<Entry>& ent, int32_t P, int32_t E, int32_t base, int32_t nkeys,
-               std::vector<int32_t>& pos, std::vector<int32_t>& store, std::vector<int32_t>& fix, int32_t& novf) {
+               const PathBanks& bk, std::vector<int32_t>& pos, std::vector<int32_t>& store,
+               std::vector<int32_t>& fix, int32_t& novf) {
   const int32_t nnz = static_cast<int32_t>(ent.size());
   pos.assign(static_cast<size_t>(P) * E, -1);
   store.assign(nnz, FFB_NO_STORE);
@@ -368,21 +388,128 @@ void pack_runs(const std::vector<Entry>& ent, int32_t P, int32_t E, int32_t base
       pc.len -= put;
     }
   }
-  // positions, piece ends, own / overflow targets
-  std::vector<int32_t> first_chunk_end(nkeys, -1), n_ovf(nkeys, 0), first_ovf(nkeys, 0);
-  std::vector<int32_t> ends;
+
+  // placed pieces: chunk, offset, entries in order; grid of entry indices
+  struct Placed { int32_t col, off, len; std::vector<int32_t> ents; };
+  std::vector<Placed> pl;
+  std::vector<int32_t>& grid = pos;  // [p * E + e]
+  std::vector<int32_t> piece_of(nnz, -1);
   for (int32_t p = 0; p < P; ++p) {
     int32_t e = 0;
     for (const Piece& pc : chunk[p]) {
-      for (int32_t t = 0; t < pc.len; ++t) pos[static_cast<size_t>(p) * E + e++] = pc.start + t;
-      const int32_t last = pc.start + pc.len - 1;
-      const int32_t key = ent[last].key0;
-      if (first_chunk_end[key] < 0)
-        first_chunk_end[key] = last;
-      else
-        ++n_ovf[key];
-      ends.push_back(last);
+      Placed q{p, e, pc.len, {}};
+      for (int32_t t = 0; t < pc.len; ++t) {
+        q.ents.push_back(pc.start + t);
+        grid[static_cast<size_t>(p) * E + e + t] = pc.start + t;
+        piece_of[pc.start + t] = static_cast<int32_t>(pl.size());
+      }
+      e += pc.len;
+      pl.push_back(std::move(q));
     }
+  }
+
+  // bank-conflict search (groups of 32 chunks at one step)
+  const bool has_key = !bk.key.empty();
+  const int32_t W = (P + 31) / 32;
+  auto is_end = [&](int32_t idx, int32_t e) {
+    const Placed& q = pl[piece_of[idx]];
+    return q.off + q.len - 1 == e;
+  };
+  auto group_cost = [&](int32_t w, int32_t e) {
+    uint8_t cg[32] = {0}, ck[32] = {0}, cs[32] = {0};
+    int32_t ex = 0;
+    for (int32_t l = 0; l < 32; ++l) {
+      const int32_t p = 32 * w + l;
+      if (p >= P) break;
+      const int32_t idx = grid[static_cast<size_t>(p) * E + e];
+      if (idx < 0) continue;
+      ex += cg[bk.gather[idx]]++ > 0;
+      if (has_key) {
+        const int32_t prev = e > 0 ? grid[static_cast<size_t>(p) * E + e - 1] : -1;
+        if (prev < 0 || ent[prev].key0 != ent[idx].key0) ex += ck[bk.key[idx]]++ > 0;
+      }
+      if (is_end(idx, e)) ex += cs[bk.store[idx]]++ > 0;
+    }
+    return ex;
+  };
+  std::vector<std::vector<int32_t>> by_len(E + 1);
+  std::vector<int32_t> multi;  // pieces of two or more entries
+  for (size_t k = 0; k < pl.size(); ++k) {
+    by_len[pl[k].len].push_back(static_cast<int32_t>(k));
+    if (pl[k].len >= 2) multi.push_back(static_cast<int32_t>(k));
+  }
+  SplitMix64 rng{0x6A09E667F3BCC909ull ^ static_cast<uint64_t>(nnz)};
+  const int64_t iters = std::min<int64_t>(static_cast<int64_t>(nnz) * 200, 4000000);
+  std::vector<std::pair<int32_t, int32_t>> aff;
+  auto add_group = [&](int32_t col, int32_t e) {
+    if (e < 0 || e >= E) return;
+    const std::pair<int32_t, int32_t> g{col / 32, e};
+    for (const auto& x : aff)
+      if (x == g) return;
+    aff.push_back(g);
+  };
+  auto cost_of = [&]() {
+    int32_t c = 0;
+    for (const auto& g : aff) c += group_cost(g.first, g.second);
+    return c;
+  };
+  for (int64_t it = 0; it < iters; ++it) {
+    const double T = 1.0 - static_cast<double>(it) / static_cast<double>(iters);  // temperature
+    aff.clear();
+    const bool within = !multi.empty() && (rng.next() & 3) == 0;
+    if (within) {
+      // reorder two entries of one piece
+      Placed& q = pl[multi[rng.uniform_int(multi.size())]];
+      const int32_t i = static_cast<int32_t>(rng.uniform_int(q.len)), j = static_cast<int32_t>(rng.uniform_int(q.len));
+      if (i == j) continue;
+      add_group(q.col, q.off + i);
+      add_group(q.col, q.off + j);
+      const int32_t before = cost_of();
+      auto apply = [&]() {
+        std::swap(q.ents[i], q.ents[j]);
+        grid[static_cast<size_t>(q.col) * E + q.off + i] = q.ents[i];
+        grid[static_cast<size_t>(q.col) * E + q.off + j] = q.ents[j];
+      };
+      apply();
+      const int32_t d = cost_of() - before;
+      if (d > 0 && rng.uniform_01() >= std::exp(-d / (0.6 * T + 1e-9))) apply();
+    } else {
+      // swap two pieces of the same length between chunks
+      const int32_t a = static_cast<int32_t>(rng.uniform_int(pl.size()));
+      const std::vector<int32_t>& same = by_len[pl[a].len];
+      if (same.size() < 2) continue;
+      const int32_t b = same[rng.uniform_int(same.size())];
+      if (a == b || pl[a].col == pl[b].col) continue;
+      for (int32_t t = 0; t <= pl[a].len; ++t) {  // one more step: the next entry's key-change flag
+        add_group(pl[a].col, pl[a].off + t);
+        add_group(pl[b].col, pl[b].off + t);
+      }
+      const int32_t before = cost_of();
+      auto apply = [&]() {
+        std::swap(pl[a].col, pl[b].col);
+        std::swap(pl[a].off, pl[b].off);
+        for (const int32_t k : {a, b})
+          for (int32_t t = 0; t < pl[k].len; ++t) grid[static_cast<size_t>(pl[k].col) * E + pl[k].off + t] = pl[k].ents[t];
+      };
+      apply();
+      const int32_t d = cost_of() - before;
+      if (d > 0 && rng.uniform_01() >= std::exp(-d / (0.6 * T + 1e-9))) apply();
+    }
+  }
+
+  // own / overflow targets: the first piece of a key in chunk order owns the key's slot
+  std::vector<int32_t> order(pl.size());
+  for (size_t k = 0; k < pl.size(); ++k) order[k] = static_cast<int32_t>(k);
+  std::sort(order.begin(), order.end(), [&](int32_t x, int32_t y) {
+    return pl[x].col != pl[y].col ? pl[x].col < pl[y].col : pl[x].off < pl[y].off;
+  });
+  std::vector<int32_t> owner(nkeys, -1), n_ovf(nkeys, 0), first_ovf(nkeys, 0), used(nkeys, 0);
+  for (const int32_t k : order) {
+    const int32_t key = ent[pl[k].ents[0]].key0;
+    if (owner[key] < 0)
+      owner[key] = k;
+    else
+      ++n_ovf[key];
   }
   for (int32_t key = 0; key < nkeys; ++key) {
     if (n_ovf[key] == 0) continue;
@@ -393,10 +520,10 @@ void pack_runs(const std::vector<Entry>& ent, int32_t P, int32_t E, int32_t base
     fix.push_back(0);
     novf += n_ovf[key];
   }
-  std::vector<int32_t> used(nkeys, 0);
-  for (int32_t last : ends) {
+  for (const int32_t k : order) {
+    const int32_t last = pl[k].ents[pl[k].len - 1];
     const int32_t key = ent[last].key0;
-    store[last] = last == first_chunk_end[key] ? key : base + first_ovf[key] + used[key]++;
+    store[last] = owner[key] == k ? key : base + first_ovf[key] + used[key]++;
   }
 }
 
@@ -440,8 +567,25 @@ extern "C" framefb_status framefb_plan_build(const framefb_frame* fin, const fra
 
     std::vector<int32_t> posZ, storeZ, fixZ, posG, storeG, fixG;
     int32_t novfZ = 0, novfG = 0;
-    pack_runs(byrow, P, EZ, m, m, posZ, storeZ, fixZ, novfZ);
-    pack_runs(bycol, P, EG, n, n, posG, storeG, fixG, novfG);
+    // banks of the tensor-core kernel's slots: row path gathers V[b] and
+    // stores Z[a]; column path gathers U[a], reloads V[b] where b changes and
+    // stores G[b]
+    PathBanks bkZ, bkG;
+    bkZ.gather.resize(nz);
+    bkZ.store.resize(nz);
+    for (int32_t q = 0; q < nz; ++q) {
+      bkZ.gather[q] = static_cast<int8_t>(slot_bank(byrow[q].key1, n));
+      bkZ.store[q] = static_cast<int8_t>(slot_bank(byrow[q].key0, m));
+    }
+    bkG.gather.resize(nz);
+    bkG.key.resize(nz);
+    bkG.store.resize(nz);
+    for (int32_t q = 0; q < nz; ++q) {
+      bkG.gather[q] = static_cast<int8_t>(slot_bank(bycol[q].key1, m));
+      bkG.key[q] = bkG.store[q] = static_cast<int8_t>(slot_bank(bycol[q].key0, n));
+    }
+    pack_runs(byrow, P, EZ, m, m, bkZ, posZ, storeZ, fixZ, novfZ);
+    pack_runs(bycol, P, EG, n, n, bkG, posG, storeG, fixG, novfG);
 
     FfbPlanHeader h;
     std::memset(&h, 0, sizeof(h));
