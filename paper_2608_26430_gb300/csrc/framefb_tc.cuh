@@ -336,20 +336,40 @@ __device__ __forceinline__ void tma_row3d(void* dst, const CUtensorMap* map, int
       : "memory");
 }
 
+// Matrix of the units a role walks through in increasing order: the
+// descriptors live in the kernel parameters (constant cache, off the
+// shared-memory request path); j advances when u passes its last unit.
+struct TileTrack {
+  int j;
+  int64_t end;
+  template <typename Args>
+  __device__ __forceinline__ void start(const Args& args, int64_t u) {
+    j = matrix_of(args, 0, u);
+    end = args.m[j].ubeg + args.m[j].ntiles;
+  }
+  // returns true when the matrix changed
+  template <typename Args>
+  __device__ __forceinline__ bool advance(const Args& args, int64_t u) {
+    bool moved = false;
+    while (u >= end) {
+      ++j;
+      end = args.m[j].ubeg + args.m[j].ntiles;
+      moved = true;
+    }
+    return moved;
+  }
+};
+
 template <int MODE>
 __global__ void __launch_bounds__(kTcThreads, 1) tc_tile_kernel(const __grid_constant__ TcLaunchK args) {
   constexpr bool F = MODE & MODE_F, D = MODE & MODE_D, C = MODE & MODE_C;
   constexpr bool NEED_V = F || C, NEED_U = D || C, SYN = F || D;
   extern __shared__ __align__(1024) uint8_t smem[];
-  __shared__ MatK mats_sm[kDescRing];
-  __shared__ int32_t mat_idx[kDescRing];
-  __shared__ int32_t tile_mat[kDescRing];
-  __shared__ uint32_t mat_bits[kDescRing][2][kGroupWords];
   __shared__ uint32_t tmem_slot;
   const int S = args.S;
   uint8_t* stg0 = smem;              // stage b at b * stage: X box, dY box at xbox_u
   float* fset0 = reinterpret_cast<float*>(smem + args.fbase);
-  uint8_t* bops = smem + args.bops;  // B operands: D hi, D lo (bf16), D^T (tf32)
+  uint8_t* bops = smem + args.bops;  // B operands: [D hi | D lo] (bf16), D^T (tf32)
   uint64_t* bar = reinterpret_cast<uint64_t*>(smem + args.mbar);
   uint64_t* mma_bar = bar + S;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -377,77 +397,56 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc_tile_kernel(const __grid_con
                  : "memory");
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
+  __syncthreads();  // barriers initialised before the first copy names them
 
-  // ---- copy issue (thread 32): descriptors, group bitmaps, tensor copies
+  // ---- copy issue (thread 32): tensor copies of tile `issued` into its stage
   constexpr int kIssuer = 32;
-  int jn = 0, jn_end = 0, jn_loaded = -1, nq = -1, issued = 0;
+  TileTrack ti{};
+  int issued = 0;
   auto issue = [&]() {
     const int64_t u = u_begin + issued;
-    while (u >= jn_end) {
-      ++jn;
-      jn_end = args.m[jn].ubeg + args.m[jn].ntiles;
-    }
-    if (jn != jn_loaded) {
-      ++nq;
-      const int q = nq % kDescRing;
-      mats_sm[q] = args.m[jn];
-      mat_idx[q] = jn;
-      jn_loaded = jn;
-      if constexpr (SYN) {
-        const uint8_t* plan = args.m[jn].plan;
-        const FfbPlanHeader& h = hdr(plan);
-        for (int side = 0; side < 2; ++side) {
-          const uint32_t* mask = table<uint32_t>(plan, side ? h.off_gmask : h.off_zmask);
-          const int G = side ? h.Gn : h.Gm;
-          for (int w = 0; w < (G + 31) / 32; ++w) {
-            uint32_t bits = 0;
-#pragma unroll 8
-            for (int i = 0; i < 32; ++i)
-              if (32 * w + i < G && __ldg(mask + 32 * w + i) != 0u) bits |= 1u << i;
-            mat_bits[q][side][w] = bits;
-          }
-        }
-      }
-    }
-    tile_mat[issued % kDescRing] = nq;
-    const MatK& M = args.m[jn];
-    const int32_t t = static_cast<int32_t>(u - M.ubeg);
+    ti.advance(args, u);
+    const int jn = ti.j;
+    const int32_t t = static_cast<int32_t>(u - args.m[jn].ubeg);
     uint8_t* dst = stg0 + (issued % S) * args.stage;
     uint64_t* b = bar + (issued % S);
-    mbar_arrive_expect_tx(b, (NEED_V ? 2u * M.n : 0u) + (NEED_U ? 2u * M.m : 0u));
+    mbar_arrive_expect_tx(b, (NEED_V ? 2u * args.m[jn].n : 0u) + (NEED_U ? 2u * args.m[jn].m : 0u));
     if (NEED_V) tma_row3d(dst, &args.maps[2 * jn], t, b);
     if (NEED_U) tma_row3d(dst + args.xbox_u, &args.maps[2 * jn + 1], t, b);
     ++issued;
   };
   if (tid == kIssuer) {
-    jn = matrix_of(args, 0, u_begin);
-    jn_end = args.m[jn].ubeg + args.m[jn].ntiles;
+    ti.start(args, u_begin);
     while (issued < S - 1 && issued < count) issue();
   }
   tc_fence_before();
-  __syncthreads();  // TMEM address, barriers and the first descriptors are ready
+  __syncthreads();  // TMEM address ready
   tc_fence_after();
   const uint32_t tmem = tmem_slot;
 
   if (warp < 4) {
     // ------------------------------------------------------------ tensor warps
+    TileTrack ta{}, ts{};  // matrices of the analysis (s) and synthesis (s - 2) tiles
+    ta.start(args, u_begin);
+    ts.start(args, u_begin);
     {
       // B operands from the k = 16 group block (the same for every matrix):
       // analysis B[n][k = coordinate], n < 32: D4[k][n] rounded to bf16 (hi),
       // n >= 32: the bf16 remainder D4[k][n - 32] - hi (lo), so that one
       // N = 64 MMA gives both partial products; synthesis B[n = coordinate]
       // [k = coefficient] = D4[n][k] as tf32
-      const MatK& M0 = mats_sm[tile_mat[0] % kDescRing];
+      const float* fv = args.m[ta.j].fval_in;
+      const int rho = args.m[ta.j].rho_in;
       __nv_bfloat16* ban = reinterpret_cast<__nv_bfloat16*>(bops);
       float* bsy = reinterpret_cast<float*>(bops + 4096);
       for (int i = tid; i < 1024; i += 128) {
         const int r = i >> 5, k = i & 31;
-        const float dk = d4(M0.fval_in, M0.rho_in, k, r);  // D4[k][r]
+        const float dk = d4(fv, rho, k, r);  // D4[k][r]
         const __nv_bfloat16 hi = __float2bfloat16_rn(dk);
         const __nv_bfloat16 lo = __float2bfloat16_rn(dk - __bfloat162float(hi));
         ban[can_bf16_off(r, k) / 2] = hi;
         ban[can_bf16_off(32 + r, k) / 2] = lo;
-        bsy[can_f32_off(r, k)] = __uint_as_float(to_tf32(d4(M0.fval_in, M0.rho_in, r, k)));  // D4[r][k]
+        bsy[can_f32_off(r, k)] = __uint_as_float(to_tf32(d4(fv, rho, r, k)));  // D4[r][k]
       }
       fence_async_smem();
       tensor_bar();
@@ -458,6 +457,24 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc_tile_kernel(const __grid_con
     uint32_t mma_phase = 0;
     bool failed = false, mma_pending = false;
     const uint32_t lane_base = static_cast<uint32_t>(32 * warp) << 16;
+    // synthesis matrix, in registers: output rows, sizes, scale, and for this
+    // thread's groups r = 32 warp + lane (+ 128) whether they have entries
+    const int r0 = 32 * warp + lane;
+    bool on_y[kTcMaxTiles] = {}, on_x[kTcMaxTiles] = {};
+    int js = -1;
+    auto load_syn = [&](int j) {
+      js = j;
+      const uint8_t* plan = args.m[j].plan;
+      const FfbPlanHeader& h = hdr(plan);
+      const uint32_t* zm = table<uint32_t>(plan, h.off_zmask);
+      const uint32_t* gm = table<uint32_t>(plan, h.off_gmask);
+#pragma unroll
+      for (int mt = 0; mt < kTcMaxTiles; ++mt) {
+        const int r = r0 + 128 * mt;
+        on_y[mt] = F && r < h.Gm && __ldg(zm + r) != 0u;
+        on_x[mt] = D && r < h.Gn && __ldg(gm + r) != 0u;
+      }
+    };
     for (int s = 0; s < count + 2; ++s) {
       if (tid == kIssuer && issued < count) issue();  // tile s + S - 1 into the stage tile s - 1 used
       const int i2 = s - 2;
@@ -465,40 +482,39 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc_tile_kernel(const __grid_con
       const bool ana = s < count;
       // output rows of tile s-2 for this thread's group of the first tile of
       // each side (read now, used after the MMAs)
-      const MatK* M2 = nullptr;
-      const uint32_t* bits2 = nullptr;
-      int64_t t2 = 0;
+      __nv_bfloat16* yrow = nullptr;
+      __nv_bfloat16* xrow = nullptr;
       int Gm2 = 0, Gn2 = 0;
+      float seff2 = 0.f;
       uint4 yp[2][4];
       if (syn) {
-        const int q2 = tile_mat[i2 % kDescRing] % kDescRing;
-        M2 = &mats_sm[q2];
-        bits2 = mat_bits[q2][0];
-        t2 = u_begin + i2 - M2->ubeg;
-        Gm2 = M2->m / FFB_GROUP;
-        Gn2 = M2->n / FFB_GROUP;
+        const int64_t u2 = u_begin + i2;
+        ts.advance(args, u2);
+        if (ts.j != js) load_syn(ts.j);
+        const MatK& M2 = args.m[ts.j];
+        const int64_t t2 = u2 - M2.ubeg;
+        yrow = static_cast<__nv_bfloat16*>(M2.Y) + t2 * M2.ldy;
+        xrow = static_cast<__nv_bfloat16*>(M2.dX) + t2 * M2.ldx;
+        Gm2 = M2.m / FFB_GROUP;
+        Gn2 = M2.n / FFB_GROUP;
+        seff2 = M2.seff;
+        if (F && on_y[0]) {
+          const uint4* p = reinterpret_cast<const uint4*>(yrow + 32 * r0);
 #pragma unroll
-        for (int side = 0; side < 2; ++side) {
-          const bool on = side == 0 ? F : D;
-          const int G = side == 0 ? Gm2 : Gn2;
-          const int r = 32 * warp + lane;
-          const uint32_t* bits = bits2 + side * kGroupWords;
-          if (on && r < G && ((bits[r >> 5] >> (r & 31)) & 1u)) {
-            const __nv_bfloat16* row = side == 0 ? static_cast<const __nv_bfloat16*>(M2->Y) + t2 * M2->ldy
-                                                 : static_cast<const __nv_bfloat16*>(M2->dX) + t2 * M2->ldx;
-            const uint4* p = reinterpret_cast<const uint4*>(row + 32 * r);
+          for (int j = 0; j < 4; ++j) yp[0][j] = p[j];
+        }
+        if (D && on_x[0]) {
+          const uint4* p = reinterpret_cast<const uint4*>(xrow + 32 * r0);
 #pragma unroll
-            for (int j = 0; j < 4; ++j) yp[side][j] = p[j];
-          }
+          for (int j = 0; j < 4; ++j) yp[1][j] = p[j];
         }
       }
-      const MatK* M0 = nullptr;
       int Gn0 = 0, Gm0 = 0;
       if (ana) {
+        ta.advance(args, u_begin + s);
+        Gn0 = args.m[ta.j].n / FFB_GROUP;
+        Gm0 = args.m[ta.j].m / FFB_GROUP;
         if (!tc_wait_bounded(bar + (s % S), static_cast<uint32_t>((s / S) & 1))) failed = true;
-        M0 = &mats_sm[tile_mat[s % kDescRing] % kDescRing];
-        Gn0 = M0->n / FFB_GROUP;
-        Gm0 = M0->m / FFB_GROUP;
       }
       // four threads issue the MMAs of this step, one per operand side:
       // thread 0 analysis of X, 32 of dY, 64 synthesis of Y, 96 of dX; each
@@ -559,7 +575,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc_tile_kernel(const __grid_con
                 float v[32], w[32];
                 const uint32_t col = tmem + lane_base + (side * kTcMaxTiles + mt) * 64;
                 tmem_ld32x2(col, col + 32, v, w);  // X D_hi, X D_lo
-                const int r = mt * 128 + 32 * warp + lane;
+                const int r = mt * 128 + r0;
                 if (r < G) {
 #pragma unroll
                   for (int c = 0; c < 8; ++c)
@@ -577,20 +593,19 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc_tile_kernel(const __grid_con
           for (int side = 0; side < 2; ++side) {
             const bool on = side == 0 ? F : D;
             const int G = side == 0 ? Gm2 : Gn2;
-            const uint32_t* bits = bits2 + side * kGroupWords;
             if (on) {
-              for (int mt = 0; mt * 128 < G; ++mt) {
+#pragma unroll
+              for (int mt = 0; mt < kTcMaxTiles; ++mt) {
+                if (mt * 128 >= G) break;
                 float v[32];
                 tmem_ld32(tmem + lane_base + kTcColSyn + (side * kTcMaxTiles + mt) * 32, v);
-                const int r = mt * 128 + 32 * warp + lane;
-                if (r < G && ((bits[r >> 5] >> (r & 31)) & 1u)) {
-                  __nv_bfloat16* row = side == 0 ? static_cast<__nv_bfloat16*>(M2->Y) + t2 * M2->ldy
-                                                 : static_cast<__nv_bfloat16*>(M2->dX) + t2 * M2->ldx;
-                  uint4* p = reinterpret_cast<uint4*>(row + 32 * r);
+                const bool has = side == 0 ? on_y[mt] : on_x[mt];
+                if (has) {
+                  uint4* p = reinterpret_cast<uint4*>((side == 0 ? yrow : xrow) + 32 * (r0 + 128 * mt));
 #pragma unroll
                   for (int j = 0; j < 4; ++j) {
                     const uint4 y = mt == 0 ? yp[side][j] : p[j];
-                    p[j] = axpy8(y, v + 8 * j, M2->seff);
+                    p[j] = axpy8(y, v + 8 * j, seff2);
                   }
                 }
               }
@@ -619,28 +634,30 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc_tile_kernel(const __grid_con
     float dc[kEreg];
 #pragma unroll
     for (int e = 0; e < kEreg; ++e) dc[e] = 0.f;
-    int cur = -1, cur_j = -1;
+    TileTrack tp{};
+    tp.start(args, u_begin);
+    int cur = -1;
     const uint8_t* splan = nullptr;
     int4* fixc = reinterpret_cast<int4*>(smem + args.fixc);
-    int nfZ = 0, nfix = 0;
+    int nfZ = 0, nfix = 0, mcur = 0, ncur = 0;
     uint32_t zero_pending = 3u;
     bool failed = false;
     for (int s = 0; s < count + 2; ++s) {
       const int i1 = s - 1;
       if (i1 >= 0 && i1 < count) {
-        const int q = tile_mat[i1 % kDescRing];
-        const MatK& M1 = mats_sm[q % kDescRing];
-        if (q != cur) {
+        tp.advance(args, u_begin + i1);
+        if (tp.j != cur) {
           if constexpr (C) {
             if (cur >= 0) {
-              float* dst = args.partial + static_cast<size_t>(blockIdx.x + cur_j) * args.stride;
+              float* dst = args.partial + static_cast<size_t>(blockIdx.x + cur) * args.stride;
               pipe_flush(splan, dst, dc, st);
             }
           }
-          cur = q;
-          cur_j = mat_idx[q % kDescRing];
-          splan = M1.plan;
-          tc_load_chunk<MODE>(ch, splan, M1.c_val, st);
+          cur = tp.j;
+          splan = args.m[cur].plan;
+          mcur = args.m[cur].m;
+          ncur = args.m[cur].n;
+          tc_load_chunk<MODE>(ch, splan, args.m[cur].c_val, st);
 #pragma unroll
           for (int e = 0; e < kEreg; ++e) dc[e] = 0.f;
           zero_pending = 3u;
@@ -670,7 +687,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc_tile_kernel(const __grid_con
               const int4 it = fixc[i];
               const bool z = i < nfZ;
               float* R = fs1 + (z ? PL.oRZ : PL.oRG);
-              const int dst = tc_slot(it.x, z ? M1.m : M1.n);
+              const int dst = tc_slot(it.x, z ? mcur : ncur);
               float sacc = R[dst];
               for (int c2 = 0; c2 < it.z; ++c2) sacc += R[it.y + c2];
               R[dst] = sacc;
@@ -687,7 +704,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc_tile_kernel(const __grid_con
     if (!failed) {
       if constexpr (C) {
         if (cur >= 0) {
-          float* dst = args.partial + static_cast<size_t>(blockIdx.x + cur_j) * args.stride;
+          float* dst = args.partial + static_cast<size_t>(blockIdx.x + cur) * args.stride;
           pipe_flush(splan, dst, dc, st);
         }
       }
