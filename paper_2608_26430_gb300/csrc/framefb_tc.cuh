@@ -185,6 +185,26 @@ __device__ __forceinline__ void tmem_ld32x2(uint32_t ta, uint32_t tb, float (&v)
   }
 }
 
+// 16 consecutive fp32 columns at each of two TMEM addresses of this lane, one wait.
+__device__ __forceinline__ void tmem_ld16x2(uint32_t ta, uint32_t tb, float (&v)[16], float (&w)[16]) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%32];\n"
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, "
+      "[%33];\n"
+      "tcgen05.wait::ld.sync.aligned;\n"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+        "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+        "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(ta), "r"(tb));
+#pragma unroll
+  for (int i = 0; i < 16; ++i) {
+    v[i] = __uint_as_float(r[i]);
+    w[i] = __uint_as_float(r[16 + i]);
+  }
+}
+
 // y (8 bf16 of one 16-byte chunk) += seff * d[0..7]
 __device__ __forceinline__ uint4 axpy8(uint4 y, const float* d, float seff) {
   uint32_t w[4] = {y.x, y.y, y.z, y.w};
@@ -399,8 +419,9 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc_tile_kernel(const __grid_con
   }
   __syncthreads();  // barriers initialised before the first copy names them
 
-  // ---- copy issue (thread 32): tensor copies of tile `issued` into its stage
-  constexpr int kIssuer = 32;
+  // ---- copy issue (the first SpMM thread): tensor copies of tile `issued`
+  // into its stage
+  constexpr int kIssuer = 128;
   TileTrack ti{};
   int issued = 0;
   auto issue = [&]() {
@@ -476,17 +497,15 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc_tile_kernel(const __grid_con
       }
     };
     for (int s = 0; s < count + 2; ++s) {
-      if (tid == kIssuer && issued < count) issue();  // tile s + S - 1 into the stage tile s - 1 used
       const int i2 = s - 2;
       const bool syn = SYN && i2 >= 0;
       const bool ana = s < count;
-      // output rows of tile s-2 for this thread's group of the first tile of
-      // each side (read now, used after the MMAs)
+      // synthesis of tile s-2: its operands (RZ / RG written last step) are
+      // ready now, so its MMAs go first (threads 64: Y, 96: dX)
       __nv_bfloat16* yrow = nullptr;
       __nv_bfloat16* xrow = nullptr;
       int Gm2 = 0, Gn2 = 0;
       float seff2 = 0.f;
-      uint4 yp[2][4];
       if (syn) {
         const int64_t u2 = u_begin + i2;
         ts.advance(args, u2);
@@ -498,6 +517,30 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc_tile_kernel(const __grid_con
         Gm2 = M2.m / FFB_GROUP;
         Gn2 = M2.n / FFB_GROUP;
         seff2 = M2.seff;
+      }
+      const bool any = (ana || syn) && !failed;  // failed is uniform here (end of the last step)
+      if (lane == 0 && warp >= 2 && any) {
+        const int side = warp & 1;
+        if (syn && (side == 0 ? F : D)) {
+          tc_fence_after();
+          float* fs2 = fset0 + (i2 & 1) * PL.total;
+          const int G = side == 0 ? Gm2 : Gn2;
+          const uint64_t abase = umma_sdesc(smem_u32(fs2 + (side == 0 ? PL.oRZ : PL.oRG)), 128, 1024);
+          for (int mt = 0; mt * 128 < G; ++mt) {
+            const uint32_t d = tmem + kTcColSyn + (side * kTcMaxTiles + mt) * 32;
+#pragma unroll
+            for (int ks = 0; ks < 4; ++ks)
+              umma_tf32(d, abase + ((mt * 16 * 1024 + ks * 256) >> 4), d_bsy + ((ks * 256) >> 4), id_sy, ks > 0);
+          }
+          umma_commit(mma_bar);
+        } else {
+          mbar_arrive(mma_bar);
+        }
+      }
+      // output rows of tile s-2 for this thread's group of the first tile of
+      // each side (read now, used after the MMAs)
+      uint4 yp[2][4];
+      if (syn) {
         if (F && on_y[0]) {
           const uint4* p = reinterpret_cast<const uint4*>(yrow + 32 * r0);
 #pragma unroll
@@ -509,26 +552,17 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc_tile_kernel(const __grid_con
           for (int j = 0; j < 4; ++j) yp[1][j] = p[j];
         }
       }
-      int Gn0 = 0, Gm0 = 0;
-      if (ana) {
-        ta.advance(args, u_begin + s);
-        Gn0 = args.m[ta.j].n / FFB_GROUP;
-        Gm0 = args.m[ta.j].m / FFB_GROUP;
-        if (!tc_wait_bounded(bar + (s % S), static_cast<uint32_t>((s / S) & 1))) failed = true;
-      }
-      // four threads issue the MMAs of this step, one per operand side:
-      // thread 0 analysis of X, 32 of dY, 64 synthesis of Y, 96 of dX; each
-      // commits (or just arrives) on the 4-count MMA barrier
-      failed = tensor_bar_or(failed);
-      const bool any = (ana || syn) && !failed;
-      if (lane == 0 && any) {
-        const int side = warp & 1;
-        const bool is_ana = warp < 2;
-        const bool on = is_ana ? (ana && (side == 0 ? NEED_V : NEED_U)) : (syn && (side == 0 ? F : D));
-        if (on) {
-          tc_fence_after();
-          if (is_ana) {
-            const int G = side == 0 ? Gn0 : Gm0;
+      // analysis of tile s once its rows have landed (threads 0: X, 32: dY)
+      if (any && lane == 0 && warp < 2) {
+        const int side = warp;
+        bool issued_mma = false;
+        if (ana) {
+          ta.advance(args, u_begin + s);
+          const bool landed = tc_wait_bounded(bar + (s % S), static_cast<uint32_t>((s / S) & 1));
+          if (!landed) failed = true;
+          if (landed && (side == 0 ? NEED_V : NEED_U)) {
+            tc_fence_after();
+            const int G = (side == 0 ? args.m[ta.j].n : args.m[ta.j].m) / FFB_GROUP;
             const uint32_t abase = smem_u32(stg0 + (s % S) * args.stage) + (side == 0 ? 0 : args.xbox_u);
             for (int mt = 0; mt * 128 < G; ++mt) {
               const uint32_t d = tmem + (side * kTcMaxTiles + mt) * 64;
@@ -536,21 +570,11 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc_tile_kernel(const __grid_con
               for (int ks = 0; ks < 2; ++ks)
                 umma_f16(d, umma_sdesc_sw64(abase + mt * 8192 + ks * 32), d_ban + ((ks * 256) >> 4), id_an, ks > 0);
             }
-          } else {
-            float* fs2 = fset0 + (i2 & 1) * PL.total;
-            const int G = side == 0 ? Gm2 : Gn2;
-            const uint64_t abase = umma_sdesc(smem_u32(fs2 + (side == 0 ? PL.oRZ : PL.oRG)), 128, 1024);
-            for (int mt = 0; mt * 128 < G; ++mt) {
-              const uint32_t d = tmem + kTcColSyn + (side * kTcMaxTiles + mt) * 32;
-#pragma unroll
-              for (int ks = 0; ks < 4; ++ks)
-                umma_tf32(d, abase + ((mt * 16 * 1024 + ks * 256) >> 4), d_bsy + ((ks * 256) >> 4), id_sy, ks > 0);
-            }
+            umma_commit(mma_bar);
+            issued_mma = true;
           }
-          umma_commit(mma_bar);
-        } else {
-          mbar_arrive(mma_bar);
         }
+        if (!issued_mma) mbar_arrive(mma_bar);  // keeps the phase count; a failure is seen below
       }
       if (any) {
         const bool ok = tc_wait_bounded(mma_bar, mma_phase);
@@ -558,35 +582,10 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc_tile_kernel(const __grid_con
           mma_phase ^= 1u;
         else
           mma_pending = true;
-        failed = tensor_bar_or(!ok);
+        failed = tensor_bar_or(failed || !ok);
         tc_fence_after();
       }
       if (!failed) {
-        // analysis results -> V / U (canonical slots), one group per thread
-        if (ana) {
-          float* fs0 = fset0 + (s & 1) * PL.total;
-#pragma unroll
-          for (int side = 0; side < 2; ++side) {
-            const bool on = side == 0 ? NEED_V : NEED_U;
-            const int G = side == 0 ? Gn0 : Gm0;
-            float* dst = fs0 + (side == 0 ? PL.oV : PL.oU);
-            if (on) {
-              for (int mt = 0; mt * 128 < G; ++mt) {
-                float v[32], w[32];
-                const uint32_t col = tmem + lane_base + (side * kTcMaxTiles + mt) * 64;
-                tmem_ld32x2(col, col + 32, v, w);  // X D_hi, X D_lo
-                const int r = mt * 128 + r0;
-                if (r < G) {
-#pragma unroll
-                  for (int c = 0; c < 8; ++c)
-                    *reinterpret_cast<float4*>(dst + can_f32_off(r, 4 * c)) =
-                        make_float4(v[4 * c] + w[4 * c], v[4 * c + 1] + w[4 * c + 1], v[4 * c + 2] + w[4 * c + 2],
-                                    v[4 * c + 3] + w[4 * c + 3]);
-                }
-              }
-            }
-          }
-        }
         // synthesis results: y += seff * delta for groups with support entries
         if (syn) {
 #pragma unroll
@@ -616,16 +615,9 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc_tile_kernel(const __grid_con
       tc_fence_before();
       if (__syncthreads_or(failed)) break;
     }
-    if (failed) {
-      if (tid == 0) {
-        atomicAdd(&g_wait_timeouts, 1u);
-        if (mma_pending) mbar_wait_bounded(mma_bar, mma_phase);  // MMAs still in flight (bounded)
-      }
-      if (tid == kIssuer) {
-        // the last tile issued into each stage: let its copy land (bounded)
-        for (int i = issued > S ? issued - S : 0; i < issued; ++i)
-          mbar_wait_bounded(bar + (i % S), static_cast<uint32_t>((i / S) & 1));
-      }
+    if (failed && tid == 0) {
+      atomicAdd(&g_wait_timeouts, 1u);
+      if (mma_pending) mbar_wait_bounded(mma_bar, mma_phase);  // MMAs still in flight (bounded)
     }
   } else {
     // ------------------------------------------------------------ SpMM warps
@@ -634,8 +626,13 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc_tile_kernel(const __grid_con
     float dc[kEreg];
 #pragma unroll
     for (int e = 0; e < kEreg; ++e) dc[e] = 0.f;
-    TileTrack tp{};
+    TileTrack tp{}, tq{};  // matrices of the SpMM tile (s - 1) and the analysis tile (s)
     tp.start(args, u_begin);
+    tq.start(args, u_begin);
+    uint32_t mph = 0;  // phase of the MMA barrier
+    const int aside = (warp - 4) >> 2;  // analysis results written: warps 4-7 V (X), 8-11 U (dY)
+    const uint32_t alane = static_cast<uint32_t>(32 * (warp & 3)) << 16;
+    const int ar0 = 32 * (warp & 3) + lane;
     int cur = -1;
     const uint8_t* splan = nullptr;
     int4* fixc = reinterpret_cast<int4*>(smem + args.fixc);
@@ -643,6 +640,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc_tile_kernel(const __grid_con
     uint32_t zero_pending = 3u;
     bool failed = false;
     for (int s = 0; s < count + 2; ++s) {
+      if (tid == kIssuer && issued < count) issue();  // tile s + S - 1 into the stage tile s - 1 used
       const int i1 = s - 1;
       if (i1 >= 0 && i1 < count) {
         tp.advance(args, u_begin + i1);
@@ -696,10 +694,49 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc_tile_kernel(const __grid_con
           fence_async_smem();  // RZ / RG are read by the tensor cores next step
         }
       }
-      if (__syncthreads_or(false)) {
+      // analysis results of tile s (TMEM, [X D_hi | X D_lo] per group) -> V / U
+      // of set s & 1, one group per thread, once the step's MMAs completed
+      const bool ana = s < count;
+      if (ana || (SYN && s >= 2)) {
+        bool ok = tc_wait_bounded(mma_bar, mph);
+        if (ok) mph ^= 1u;
+        failed = !ok;
+        tc_fence_after();
+        const bool on = aside == 0 ? NEED_V : NEED_U;
+        if (ok && ana && on) {
+          tq.advance(args, u_begin + s);
+          const int G = (aside == 0 ? args.m[tq.j].n : args.m[tq.j].m) / FFB_GROUP;
+          float* dst = fset0 + (s & 1) * PL.total + (aside == 0 ? PL.oV : PL.oU);
+#pragma unroll
+          for (int mt = 0; mt < kTcMaxTiles; ++mt) {
+            if (mt * 128 >= G) break;
+            const int r = mt * 128 + ar0;
+#pragma unroll
+            for (int hlf = 0; hlf < 2; ++hlf) {
+              float v[16], w[16];
+              const uint32_t col = tmem + alane + (aside * kTcMaxTiles + mt) * 64 + 16 * hlf;
+              tmem_ld16x2(col, col + 32, v, w);  // coefficients 16 hlf .. +15: hi and lo parts
+              if (r < G) {
+#pragma unroll
+                for (int c = 0; c < 4; ++c)
+                  *reinterpret_cast<float4*>(dst + can_f32_off(r, 16 * hlf + 4 * c)) =
+                      make_float4(v[4 * c] + w[4 * c], v[4 * c + 1] + w[4 * c + 1], v[4 * c + 2] + w[4 * c + 2],
+                                  v[4 * c + 3] + w[4 * c + 3]);
+              }
+            }
+          }
+        }
+      }
+      tc_fence_before();
+      if (__syncthreads_or(failed)) {
         failed = true;
         break;
       }
+    }
+    if (failed && tid == kIssuer) {
+      // the last tile issued into each stage: let its copy land (bounded)
+      for (int i = issued > S ? issued - S : 0; i < issued; ++i)
+        mbar_wait_bounded(bar + (i % S), static_cast<uint32_t>((i / S) & 1));
     }
     if (!failed) {
       if constexpr (C) {
