@@ -36,6 +36,7 @@ def parse():
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu", action="store_true")
     p.add_argument("--cpu-tokens", type=int, default=8192, help="token sample of the CPU oracle baseline")
+    p.add_argument("--cpu-mats", type=int, default=4, help="matrices in the CPU oracle baseline sample")
     p.add_argument("--mats", type=int, default=None, help="first MATS matrices only (small profiling cases)")
     return p.parse_args()
 
@@ -156,27 +157,33 @@ def measured_traffic():
         return None
 
 
-def cpu_oracle_sample(w, tokens: int):
-    """Time the oracle (fp64 numpy) on one matrix of the workload over `tokens` tokens."""
+def cpu_oracle_sample(w, tokens: int, mats: int = 1):
+    """Time the oracle (fp64 numpy) on the first `mats` matrices of the workload
+    over `tokens` tokens each; returns (compute seconds, setup seconds)."""
     import numpy as np
     from oracle import adapter, frames, support
     from paper_2608_26430_gb300 import workloads as wl
-    spec = w.mats[0]
-    X = wl.x_input(w, 0, tokens).float().numpy().astype(np.float64)
-    dY = wl.dy_input(w, 0, tokens).float().numpy().astype(np.float64)
-    c = wl.c_values(w, 0).numpy().astype(np.float64)
-    s = wl.scale_of(w, spec)
-    t0 = time.perf_counter()
-    Pin = frames.real_frame(spec.n, w.k, spec.n // w.k)
-    Pout = Pin if spec.m == spec.n else frames.real_frame(spec.m, w.k, spec.m // w.k)
-    row, col, _, _ = support.sample_support(spec.m, spec.n, w.nnz, w.support_seed, w.support_mode, w.zipf_s, w.k)
-    t1 = time.perf_counter()
-    C = adapter.dense_C(spec.m, spec.n, row, col, c)
-    adapter.forward(X, np.zeros((tokens, spec.m)), Pin, Pout, C, s)
-    adapter.backward_dx(dY, np.zeros((tokens, spec.n)), Pin, Pout, C, s)
-    adapter.grad_coeff(X, dY, Pin, Pout, s, row, col)
-    t2 = time.perf_counter()
-    return t2 - t1, t1 - t0
+    tcomp = tsetup = 0.0
+    for j in range(mats):
+        spec = w.mats[j]
+        X = wl.x_input(w, j, tokens).float().numpy().astype(np.float64)
+        dY = wl.dy_input(w, j, tokens).float().numpy().astype(np.float64)
+        c = wl.c_values(w, j).numpy().astype(np.float64)
+        s = wl.scale_of(w, spec)
+        t0 = time.perf_counter()
+        Pin = frames.real_frame(spec.n, w.k, spec.n // w.k)
+        Pout = Pin if spec.m == spec.n else frames.real_frame(spec.m, w.k, spec.m // w.k)
+        row, col, _, _ = support.sample_support(spec.m, spec.n, w.nnz, w.support_seed, w.support_mode, w.zipf_s,
+                                                w.k)
+        t1 = time.perf_counter()
+        C = adapter.dense_C(spec.m, spec.n, row, col, c)
+        adapter.forward(X, np.zeros((tokens, spec.m)), Pin, Pout, C, s)
+        adapter.backward_dx(dY, np.zeros((tokens, spec.n)), Pin, Pout, C, s)
+        adapter.grad_coeff(X, dY, Pin, Pout, s, row, col)
+        t2 = time.perf_counter()
+        tcomp += t2 - t1
+        tsetup += t1 - t0
+    return tcomp, tsetup
 
 
 def cpu_threads():
@@ -312,11 +319,12 @@ def main():
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu:
-        tcpu, tsetup = cpu_oracle_sample(w, args.cpu_tokens)
-        cpu_tok = args.cpu_tokens / (tcpu * len(w.mats))
+        k = min(args.cpu_mats, len(w.mats))
+        tcpu, tsetup = cpu_oracle_sample(w, args.cpu_tokens, k)
+        cpu_tok = args.cpu_tokens / (tcpu / k * len(w.mats))
         cpu = {"value": cpu_tok, "unit": "tokens/s", "cores": cpu_threads(), "kind": "oracle",
-               "sample": f"dense fp64 oracle on 1 of {len(w.mats)} matrices ({w.mats[0].m}x{w.mats[0].n}) over "
-                         f"{args.cpu_tokens} tokens ({tcpu:.1f} s), scaled to {len(w.mats)} matrices; frame and "
+               "sample": f"dense fp64 oracle on {k} of {len(w.mats)} matrices ({w.mats[0].m}x{w.mats[0].n}) over "
+                         f"{args.cpu_tokens} tokens each ({tcpu:.1f} s), scaled to {len(w.mats)} matrices; frame and "
                          f"support setup ({tsetup:.1f} s) excluded"}
 
     if rank == 0:
