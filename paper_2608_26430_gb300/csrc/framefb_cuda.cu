@@ -15,6 +15,7 @@
 #include "framefb_mma.cuh"
 #include "framefb_pipe.cuh"
 #include "framefb_tc.cuh"
+#include "framefb_tc2.cuh"
 #include "plan_internal.h"
 #include "plan_layout.h"
 
@@ -51,6 +52,7 @@ struct Prepared {
   bool reg;
   bool pipe;  // bf16: pipelined kernel (one token per tile)
   bool tc;    // bf16: pipelined kernel on tcgen05 tensor cores
+  bool tc2;   // bf16: the same, two tokens per unit
   int T;      // tile tokens of the bf16 kernel
   int threads;
 };
@@ -62,6 +64,17 @@ void* tc_kernel_ptr(int mode) {
     case 4: return reinterpret_cast<void*>(ffb::tc_tile_kernel<4>);
     case 6: return reinterpret_cast<void*>(ffb::tc_tile_kernel<6>);
     case 7: return reinterpret_cast<void*>(ffb::tc_tile_kernel<7>);
+    default: return nullptr;
+  }
+}
+
+void* tc2_kernel_ptr(int mode) {
+  switch (mode) {
+    case 1: return reinterpret_cast<void*>(ffb::tc2_tile_kernel<1>);
+    case 2: return reinterpret_cast<void*>(ffb::tc2_tile_kernel<2>);
+    case 4: return reinterpret_cast<void*>(ffb::tc2_tile_kernel<4>);
+    case 6: return reinterpret_cast<void*>(ffb::tc2_tile_kernel<6>);
+    case 7: return reinterpret_cast<void*>(ffb::tc2_tile_kernel<7>);
     default: return nullptr;
   }
 }
@@ -238,6 +251,58 @@ size_t tc_smem_map(const framefb_mat* mats, int32_t nmats, int32_t ops, int S, f
   return mbar + 8 * static_cast<size_t>(S + 1);
 }
 
+// Shared-memory map of the two-token tensor-core kernel: a ring of S stages
+// (two token rows of X, then two of dY, each a swizzled K-major operand of
+// one 128-group tile), B operands (8 KB), one V/U set (float2 per
+// coefficient: both tokens), one RZ/RG set per token in the canonical tf32
+// layout (padded to a whole tile), the fix-up item cache, S + 2 mbarriers.
+// Returns the total bytes, or 0 when a matrix does not fit the shape rules
+// (group counts a multiple of 8 and at most 128).
+size_t tc2_smem_map(const framefb_mat* mats, int32_t nmats, int32_t ops, int S, ffb::TcLaunchK* a) {
+  const bool F = ops & FRAMEFB_OP_FORWARD, D = ops & FRAMEFB_OP_BACKWARD_DX, C = ops & FRAMEFB_OP_GRAD_COEFF;
+  const bool needV = F || C, needU = D || C;
+  size_t nfix = 0;
+  int32_t nmax = 0, mmax = 0, ovfZ = 0, ovfG = 0;
+  for (int32_t j = 0; j < nmats; ++j) {
+    const FfbPlanHeader* h = plan_header(mats[j].plan);
+    if (h->Gn % 8 || h->Gm % 8 || h->Gn > 128 || h->Gm > 128) return 0;
+    nmax = std::max(nmax, h->n);
+    mmax = std::max(mmax, h->m);
+    ovfZ = std::max(ovfZ, h->ovfZ);
+    ovfG = std::max(ovfG, h->ovfG);
+    nfix = std::max<size_t>(nfix, (F ? h->nfixZ : 0) + (D ? h->nfixG : 0));
+  }
+  const size_t tok_x = needV ? 8192 : 0, tok_u = needU ? 8192 : 0;
+  const size_t stage = 2 * tok_x + 2 * tok_u;
+  const size_t bops = S * stage;
+  const size_t vu = bops + 8192;
+  const size_t oU = needV ? nmax : 0;  // float2 units
+  const size_t rzg = vu + round_up((oU + (needU ? mmax : 0)) * 8, 128);
+  const size_t szRZ = F ? round_up(std::max<size_t>(128 * 32, mmax + ovfZ), 32) : 0;
+  const size_t szRG = D ? round_up(std::max<size_t>(128 * 32, nmax + ovfG), 32) : 0;
+  const size_t rzg_tok = szRZ + szRG;  // floats
+  const size_t fixc = rzg + 2 * rzg_tok * 4;
+  const size_t mbar = round_up(fixc + 16 * nfix, 16);
+  if (a) {
+    a->S = S;
+    a->stage = static_cast<int32_t>(stage);
+    a->xbox_u = static_cast<int32_t>(2 * tok_x);
+    a->tok_x = static_cast<int32_t>(tok_x);
+    a->tok_u = static_cast<int32_t>(tok_u);
+    a->bops = static_cast<int32_t>(bops);
+    a->vu = static_cast<int32_t>(vu);
+    a->set_oU = static_cast<int32_t>(oU);
+    a->rzg = static_cast<int32_t>(rzg);
+    a->set_oRZ = 0;
+    a->set_oRG = static_cast<int32_t>(szRZ);
+    a->rzg_tok = static_cast<int32_t>(rzg_tok);
+    a->fixc = static_cast<int32_t>(fixc);
+    a->fixc_items = static_cast<int32_t>(nfix);
+    a->mbar = static_cast<int32_t>(mbar);
+  }
+  return mbar + 8 * static_cast<size_t>(S + 2);
+}
+
 // cuTensorMapEncodeTiled through the runtime's driver entry point (no link
 // against the driver library).
 using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
@@ -271,17 +336,19 @@ bool encode_rows(CUtensorMap* map, const void* base, int32_t d, int32_t N, int64
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// Kernel choice for bf16: the tensor-core pipelined kernel wherever it
+// Kernel choice for bf16: the two-token tensor-core kernel wherever it
 // applies (register-resident plans, group counts a multiple of 8 and at most
-// 256, its shared-memory map fits), else the one-phase-at-a-time tile
-// kernel.  FRAMEFB_KERNEL=tile or =pipe forces the tile kernel or the
-// warp-MMA pipelined kernel instead (for comparison and tests).
+// 128, its shared-memory map fits), else the one-token tensor-core kernel
+// (group counts up to 256), else the one-phase-at-a-time tile kernel.
+// FRAMEFB_KERNEL=tc2, =tc, =pipe or =tile selects one of them where it
+// applies (for comparison and tests).
 bool kernel_is(const char* name) {
   const char* e = std::getenv("FRAMEFB_KERNEL");
   return e && std::strcmp(e, name) == 0;
 }
 bool pipe_allowed() { return kernel_is("pipe"); }
 bool tc_allowed() { return !kernel_is("tile") && !kernel_is("pipe"); }
+bool tc2_allowed() { return tc_allowed() && !kernel_is("tc"); }
 
 // Validate one chunk of matrices and fill the launch parameters.
 framefb_status prepare(const framefb_mat* mats, int32_t nmats, int32_t ops, framefb_dtype dt, Prepared& P) {
@@ -300,8 +367,25 @@ framefb_status prepare(const framefb_mat* mats, int32_t nmats, int32_t ops, fram
   int64_t units = 0;
   size_t smem = 0;
   int T_mma = 0;
-  bool pipe = false, tc = false;
-  if (dt == FRAMEFB_BF16 && reg && tc_allowed() && nmats <= ffb::kTcMaxMats && encode_tiled()) {
+  bool pipe = false, tc = false, tc2 = false;
+  if (dt == FRAMEFB_BF16 && reg && tc2_allowed() && nmats <= ffb::kTcMaxMats && encode_tiled()) {
+    // two-token tensor-core kernel: two stages
+    int dev = 0, optin = 0;
+    cudaFuncAttributes fa{};
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess ||
+        cudaFuncGetAttributes(&fa, tc2_kernel_ptr(ops)) != cudaSuccess)
+      return FRAMEFB_ECUDA;
+    const size_t budget = static_cast<size_t>(optin) - fa.sharedSizeBytes;
+    const size_t need = tc2_smem_map(mats, nmats, ops, 2, nullptr);
+    if (need > 0 && need <= budget) {
+      tc2 = true;
+      T_mma = 2;
+      std::memset(P.tcargs, 0, sizeof(ffb::TcLaunchK));
+      smem = tc2_smem_map(mats, nmats, ops, 2, P.tcargs);
+    }
+  }
+  if (dt == FRAMEFB_BF16 && reg && !tc2 && tc_allowed() && nmats <= ffb::kTcMaxMats && encode_tiled()) {
     // tensor-core pipelined kernel: deepest staging ring (2..4) that fits
     int dev = 0, optin = 0;
     cudaFuncAttributes fa{};
@@ -320,7 +404,7 @@ framefb_status prepare(const framefb_mat* mats, int32_t nmats, int32_t ops, fram
       }
     }
   }
-  if (dt == FRAMEFB_BF16 && reg && !tc && pipe_allowed()) {
+  if (dt == FRAMEFB_BF16 && reg && !tc && !tc2 && pipe_allowed()) {
     // pipelined kernel: deepest staging ring (2..4) that fits next to its
     // static shared memory
     int dev = 0, optin = 0;
@@ -337,7 +421,7 @@ framefb_status prepare(const framefb_mat* mats, int32_t nmats, int32_t ops, fram
         smem = pipe_smem_map(mats, nmats, ops, S, P.args);
       }
   }
-  if (dt == FRAMEFB_BF16 && !pipe && !tc) {
+  if (dt == FRAMEFB_BF16 && !pipe && !tc && !tc2) {
     // one tile size for the launch; stage the output rows too when they fit,
     // else the synthesis reads them from global memory
     bool staged = false;
@@ -413,7 +497,7 @@ framefb_status prepare(const framefb_mat* mats, int32_t nmats, int32_t ops, fram
   P.args->nmats = nmats;
   P.args->total_units = static_cast<int32_t>(units);
   P.args->stride = (nnz_max + 63) & ~63;
-  if (tc) {
+  if (tc || tc2) {
     ffb::TcLaunchK& A = *P.tcargs;
     A.nmats = nmats;
     A.total_units = P.args->total_units;
@@ -432,13 +516,16 @@ framefb_status prepare(const framefb_mat* mats, int32_t nmats, int32_t ops, fram
   P.reg = reg;
   P.pipe = pipe;
   P.tc = tc;
-  P.threads = tc ? ffb::kTcThreads : kThreads;
+  P.tc2 = tc2;
+  P.threads = (tc || tc2) ? ffb::kTcThreads : kThreads;
   P.T = T_mma;
   P.smem = std::max<size_t>(smem, 16);
   P.grid = 0;
   P.ws_bytes = 0;
   if (units == 0) return FRAMEFB_OK;
-  void* fn = tc ? tc_kernel_ptr(ops) : pipe ? pipe_kernel_ptr(ops) : tile_kernel_ptr(dt, ops, reg, T_mma);
+  void* fn = tc2 ? tc2_kernel_ptr(ops)
+             : tc ? tc_kernel_ptr(ops)
+                  : pipe ? pipe_kernel_ptr(ops) : tile_kernel_ptr(dt, ops, reg, T_mma);
   if (!fn) return FRAMEFB_EINVAL;
   int dev = 0, sms = 0, per_sm = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return FRAMEFB_ECUDA;
@@ -543,8 +630,10 @@ extern "C" framefb_status framefb_run(const framefb_mat* mats, int32_t nmats, in
     P.args->partial = static_cast<float*>(ws);
     P.tcargs->partial = static_cast<float*>(ws);
     P.red->partial = static_cast<const float*>(ws);
-    void* fn = P.tc ? tc_kernel_ptr(ops) : P.pipe ? pipe_kernel_ptr(ops) : tile_kernel_ptr(dtype, ops, P.reg, P.T);
-    void* kargs[] = {P.tc ? static_cast<void*>(P.tcargs) : static_cast<void*>(P.args)};
+    void* fn = P.tc2  ? tc2_kernel_ptr(ops)
+               : P.tc ? tc_kernel_ptr(ops)
+                      : P.pipe ? pipe_kernel_ptr(ops) : tile_kernel_ptr(dtype, ops, P.reg, P.T);
+    void* kargs[] = {(P.tc || P.tc2) ? static_cast<void*>(P.tcargs) : static_cast<void*>(P.args)};
     if (cudaLaunchKernel(fn, dim3(P.grid), dim3(P.threads), kargs, P.smem, st) != cudaSuccess)
       return FRAMEFB_ECUDA;
     if (ops & FRAMEFB_OP_GRAD_COEFF) {

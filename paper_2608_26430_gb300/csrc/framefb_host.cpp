@@ -302,15 +302,24 @@ inline int32_t group_major(int32_t c, int32_t rho) {
 
 struct Entry { int32_t key0, key1, q; };
 
-// Bank (4-byte word mod 32) of the fp32 slot of group-major index x in the
-// tensor-core kernel's coefficient buffers (canonical K-major core-matrix
-// layout: group r, coefficient c at 256 (r / 8) + 32 (c / 4) + 4 (r % 8) +
-// c % 4 floats); overflow slots x >= K sit at x.
-inline int32_t slot_bank(int32_t x, int32_t K) { return x >= K ? (x & 31) : (((x >> 5) & 7) * 4 + (x & 3)); }
+// Banks of the default (two-token) tensor-core kernel's coefficient buffers.
+// RZ / RG: 4-byte stores to the canonical K-major core-matrix layout (group
+// r, coefficient c at float 256 (r / 8) + 32 (c / 4) + 4 (r % 8) + c % 4;
+// overflow slots x >= K at x), bank = word mod 32 over a warp.
+inline int32_t store_bank(int32_t x, int32_t K) { return x >= K ? (x & 31) : (((x >> 5) & 7) * 4 + (x & 3)); }
+// V / U: 8-byte gathers (both tokens of a coefficient) from the layout in
+// which group r's 16-byte chunks (two coefficients) are permuted by r mod 8:
+// float2 index 32 r + 2 ((c / 2) xor (r mod 8)) + c mod 2; a half-warp's
+// requests are served together, bank pair = float2 index mod 16.
+inline int32_t gather_bank(int32_t x) {
+  const int32_t r = x >> 5, c = x & 31;
+  return (2 * ((c >> 1) ^ (r & 7)) + (c & 1)) & 15;
+}
 
-// Shared-memory banks one coefficient path touches per entry: the gather of
-// the other index, the reload of the key's own input where the key changes
-// (dC, column path only) and the run-sum store at a piece end.
+// Shared-memory banks one coefficient path touches per entry: the 8-byte
+// gather of the other index and the reload of the key's own input where the
+// key changes (dC, column path only), both per half-warp; the 4-byte run-sum
+// stores at a piece end, per warp.
 struct PathBanks {
   std::vector<int8_t> gather, key, store;  // per entry; key empty: no reload
 };
@@ -416,19 +425,20 @@ void pack_runs(const std::vector<Entry>& ent, int32_t P, int32_t E, int32_t base
     return q.off + q.len - 1 == e;
   };
   auto group_cost = [&](int32_t w, int32_t e) {
-    uint8_t cg[32] = {0}, ck[32] = {0}, cs[32] = {0};
+    uint8_t cg[2][16] = {}, ck[2][16] = {}, cs[32] = {0};
     int32_t ex = 0;
     for (int32_t l = 0; l < 32; ++l) {
       const int32_t p = 32 * w + l;
       if (p >= P) break;
       const int32_t idx = grid[static_cast<size_t>(p) * E + e];
       if (idx < 0) continue;
-      ex += cg[bk.gather[idx]]++ > 0;
+      const int32_t h = l >> 4;
+      ex += cg[h][bk.gather[idx]]++ > 0;
       if (has_key) {
         const int32_t prev = e > 0 ? grid[static_cast<size_t>(p) * E + e - 1] : -1;
-        if (prev < 0 || ent[prev].key0 != ent[idx].key0) ex += ck[bk.key[idx]]++ > 0;
+        if (prev < 0 || ent[prev].key0 != ent[idx].key0) ex += ck[h][bk.key[idx]]++ > 0;
       }
-      if (is_end(idx, e)) ex += cs[bk.store[idx]]++ > 0;
+      if (is_end(idx, e)) ex += 2 * (cs[bk.store[idx]]++ > 0);  // two stores: one per token
     }
     return ex;
   };
@@ -567,22 +577,23 @@ extern "C" framefb_status framefb_plan_build(const framefb_frame* fin, const fra
 
     std::vector<int32_t> posZ, storeZ, fixZ, posG, storeG, fixG;
     int32_t novfZ = 0, novfG = 0;
-    // banks of the tensor-core kernel's slots: row path gathers V[b] and
-    // stores Z[a]; column path gathers U[a], reloads V[b] where b changes and
-    // stores G[b]
+    // banks of the default kernel's slots: row path gathers V[b] and stores
+    // Z[a]; column path gathers U[a], reloads V[b] where b changes and stores
+    // G[b]
     PathBanks bkZ, bkG;
     bkZ.gather.resize(nz);
     bkZ.store.resize(nz);
     for (int32_t q = 0; q < nz; ++q) {
-      bkZ.gather[q] = static_cast<int8_t>(slot_bank(byrow[q].key1, n));
-      bkZ.store[q] = static_cast<int8_t>(slot_bank(byrow[q].key0, m));
+      bkZ.gather[q] = static_cast<int8_t>(gather_bank(byrow[q].key1));
+      bkZ.store[q] = static_cast<int8_t>(store_bank(byrow[q].key0, m));
     }
     bkG.gather.resize(nz);
     bkG.key.resize(nz);
     bkG.store.resize(nz);
     for (int32_t q = 0; q < nz; ++q) {
-      bkG.gather[q] = static_cast<int8_t>(slot_bank(bycol[q].key1, m));
-      bkG.key[q] = bkG.store[q] = static_cast<int8_t>(slot_bank(bycol[q].key0, n));
+      bkG.gather[q] = static_cast<int8_t>(gather_bank(bycol[q].key1));
+      bkG.key[q] = static_cast<int8_t>(gather_bank(bycol[q].key0));
+      bkG.store[q] = static_cast<int8_t>(store_bank(bycol[q].key0, n));
     }
     pack_runs(byrow, P, EZ, m, m, bkZ, posZ, storeZ, fixZ, novfZ);
     pack_runs(bycol, P, EG, n, n, bkG, posG, storeG, fixG, novfG);

@@ -344,6 +344,9 @@ struct TcLaunchK {
   int32_t stage, xbox_u, fbase, mbar;  // staging ring: stage stride, dY box offset (bytes)
   int32_t set_oU, set_oRZ, set_oRG, set_total;
   int32_t fixc, fixc_items, bops, pad;
+  // two-token kernel: stage token strides (bytes), V/U and RZ/RG regions
+  // (bytes offsets), floats of one token's RZ/RG region
+  int32_t tok_x, tok_u, vu, rzg, rzg_tok, pad2;
   MatK m[kTcMaxMats];
   alignas(64) CUtensorMap maps[2 * kTcMaxMats];
 };

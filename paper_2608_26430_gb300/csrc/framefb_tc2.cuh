@@ -1,0 +1,565 @@
+// Pipelined bf16 tile kernel on tcgen05 tensor cores, two tokens per tile.
+// Included by framefb_cuda.cu after framefb_tc.cuh.
+//
+// Same work as tc_tile_kernel (Sec. 3.1 update, Lemma 1 gradient of
+// Appendix A), with units of two tokens of one matrix, so that every
+// coefficient SpMM instruction serves both tokens:
+//   * V and U are held token-minor (a float2 per coefficient), so one 64-bit
+//     gather feeds both tokens; they are not tensor-core operands, their
+//     layout is free: group r's sixteen 16-byte chunks (two coefficients x
+//     two tokens) are permuted by r mod 8 (vu_slot), which makes the
+//     write-back of one group per lane conflict-free;
+//   * RZ and RG stay per token in the canonical tf32 K-major layout (they are
+//     the synthesis A operands);
+//   * shared memory holds one V/U set and one RZ/RG set (two tokens each):
+//     the SpMM warps first compute dC (gathers only), then wait until the
+//     synthesis MMAs of the step have read RZ/RG before the run sums (which
+//     gather again and store), and write the analysis results of the step
+//     into V/U only after all of them finished gathering;
+//   * eight MMA groups per step: analysis (token x side) issued by threads 0
+//     (X) and 32 (dY) on one barrier, synthesis by threads 64 (Y) and 96 (dX)
+//     on another.
+// Shapes: every group count a multiple of 8 and at most 128 (n, m <= 4096).
+// Waits are bounded as in tc_tile_kernel.
+#pragma once
+#include "framefb_tc.cuh"
+
+namespace ffb {
+
+// float2 (two-token) slot of group-major index x in the V / U buffers.
+__host__ __device__ __forceinline__ int32_t vu_slot(int32_t x) {
+  const int32_t r = x >> 5, c = x & 31;
+  return 32 * r + 2 * ((c >> 1) ^ (r & 7)) + (c & 1);
+}
+
+// barrier of the 256 SpMM threads that also ORs a flag over them
+__device__ __forceinline__ bool spmm_bar_or(bool f) {
+  uint32_t out;
+  asm volatile(
+      "{\n .reg .pred p, q;\n setp.ne.u32 p, %1, 0;\n bar.red.or.pred q, 1, 256, p;\n selp.u32 %0, 1, 0, q;\n}\n"
+      : "=r"(out)
+      : "r"(static_cast<uint32_t>(f))
+      : "memory");
+  return out != 0;
+}
+
+// 8 consecutive fp32 columns at each of four TMEM addresses of this lane, one wait.
+__device__ __forceinline__ void tmem_ld8x4(uint32_t t0, uint32_t t1, uint32_t t2, uint32_t t3, float (&a)[8],
+                                           float (&b)[8], float (&c)[8], float (&d)[8]) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%32];\n"
+      "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%8,%9,%10,%11,%12,%13,%14,%15}, [%33];\n"
+      "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%16,%17,%18,%19,%20,%21,%22,%23}, [%34];\n"
+      "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%24,%25,%26,%27,%28,%29,%30,%31}, [%35];\n"
+      "tcgen05.wait::ld.sync.aligned;\n"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+        "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+        "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(t0), "r"(t1), "r"(t2), "r"(t3));
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    a[i] = __uint_as_float(r[i]);
+    b[i] = __uint_as_float(r[8 + i]);
+    c[i] = __uint_as_float(r[16 + i]);
+    d[i] = __uint_as_float(r[24 + i]);
+  }
+}
+
+// Register chunk of plan column `col`: gather slots in the float2 V / U
+// layout, store targets in the canonical RZ / RG layout.
+template <int MODE>
+__device__ __forceinline__ void tc2_load_chunk(Chunk<MODE, true, false>& ch, const uint8_t* plan, const float* c_val,
+                                               int col) {
+  constexpr bool F = MODE & MODE_F, D = MODE & MODE_D, C = MODE & MODE_C;
+  const FfbPlanHeader& h = hdr(plan);
+  ch.EZ = h.EZ;
+  ch.EG = h.EG;
+  ch.n = h.n;
+  ch.m = h.m;
+  const int32_t* tzb = table<int32_t>(plan, h.off_zb);
+  const int32_t* tzq = table<int32_t>(plan, h.off_zq);
+  const int32_t* tga = table<int32_t>(plan, h.off_ga);
+  const int32_t* tgb = table<int32_t>(plan, h.off_gb);
+  const int32_t* tgq = table<int32_t>(plan, h.off_gq);
+  auto slots = [](uint32_t w, int Khi) {
+    const uint32_t lo = w & 0x7FFFu, hi = w >> 16;
+    const uint32_t slo = static_cast<uint32_t>(vu_slot(static_cast<int32_t>(lo)));
+    const uint32_t shi =
+        hi == FFB_NO_STORE ? FFB_NO_STORE : static_cast<uint32_t>(tc_slot(static_cast<int32_t>(hi), Khi));
+    return slo | (shi << 16);
+  };
+#pragma unroll
+  for (int e = 0; e < kEreg; ++e) {
+    ch.zb[e] = FFB_NO_STORE << 16;
+    ch.ga[e] = FFB_NO_STORE << 16;
+    ch.gb[e] = 0;
+    ch.zc[e] = ch.gc[e] = 0.f;
+    if (F && e < ch.EZ) {
+      const uint32_t w = static_cast<uint32_t>(__ldg(tzb + e * kThreads + col));
+      ch.zb[e] = slots(w, ch.m);
+      const int32_t q = __ldg(tzq + e * kThreads + col);
+      ch.zc[e] = q >= 0 ? __ldg(c_val + q) : 0.f;
+    }
+    if ((D || C) && e < ch.EG) {
+      const uint32_t w = static_cast<uint32_t>(__ldg(tga + e * kThreads + col));
+      ch.ga[e] = slots(w, ch.n);
+      ch.gb[e] = static_cast<uint32_t>(vu_slot(__ldg(tgb + e * kThreads + col)));
+      const int32_t q = __ldg(tgq + e * kThreads + col);
+      ch.gc[e] = (D && q >= 0) ? __ldg(c_val + q) : 0.f;
+    }
+  }
+}
+
+template <int MODE>
+__global__ void __launch_bounds__(kTcThreads, 1) tc2_tile_kernel(const __grid_constant__ TcLaunchK args) {
+  constexpr bool F = MODE & MODE_F, D = MODE & MODE_D, C = MODE & MODE_C;
+  constexpr bool NEED_V = F || C, NEED_U = D || C, SYN = F || D;
+  constexpr int B = FFB_ENTRY_BLOCK;
+  extern __shared__ __align__(1024) uint8_t smem[];
+  __shared__ uint32_t tmem_slot;
+  const int S = args.S;
+  uint8_t* stg0 = smem;  // stage b at b * stage: X tokens at k * tok_x, dY tokens at xbox_u + k * tok_u
+  float2* V2 = reinterpret_cast<float2*>(smem + args.vu);
+  float2* U2 = V2 + args.set_oU;
+  float* rzg = reinterpret_cast<float*>(smem + args.rzg);  // token k at k * rzg_tok: RZ at set_oRZ, RG at set_oRG
+  uint8_t* bops = smem + args.bops;
+  uint64_t* bar = reinterpret_cast<uint64_t*>(smem + args.mbar);
+  uint64_t* ana_bar = bar + S;
+  uint64_t* syn_bar = bar + S + 1;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+
+  const int64_t units = args.total_units;
+  const int64_t u_begin = (static_cast<int64_t>(blockIdx.x) * units) / gridDim.x;
+  const int64_t u_end = (static_cast<int64_t>(blockIdx.x + 1) * units) / gridDim.x;
+  const int count = static_cast<int>(u_end - u_begin);
+  if (count <= 0) return;
+
+  if (tid == 0) {
+    for (int b = 0; b < S; ++b) mbar_init(bar + b, 1);
+    mbar_init(ana_bar, 2);  // threads 0 and 32
+    mbar_init(syn_bar, 2);  // threads 64 and 96
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 0) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&tmem_slot)),
+                 "r"(kTcTmemCols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  __syncthreads();  // barriers initialised before the first copy names them
+
+  // ---- copy issue (thread 32, at the start of its step, before it waits for
+  // its own rows): both token rows of unit `issued`
+  constexpr int kIssuer = 32;
+  TileTrack ti{};
+  int issued = 0;
+  auto issue = [&]() {
+    const int64_t u = u_begin + issued;
+    ti.advance(args, u);
+    const int jn = ti.j;
+    const int32_t t0 = static_cast<int32_t>(2 * (u - args.m[jn].ubeg));
+    const int Tc = min(2, args.m[jn].N - t0);
+    uint8_t* dst = stg0 + (issued % S) * args.stage;
+    uint64_t* b = bar + (issued % S);
+    mbar_arrive_expect_tx(b, static_cast<uint32_t>(Tc) * ((NEED_V ? 2u * args.m[jn].n : 0u) +
+                                                         (NEED_U ? 2u * args.m[jn].m : 0u)));
+    for (int k = 0; k < Tc; ++k) {
+      if (NEED_V) tma_row3d(dst + k * args.tok_x, &args.maps[2 * jn], t0 + k, b);
+      if (NEED_U) tma_row3d(dst + args.xbox_u + k * args.tok_u, &args.maps[2 * jn + 1], t0 + k, b);
+    }
+    ++issued;
+  };
+  if (tid == kIssuer) {
+    ti.start(args, u_begin);
+    while (issued < S - 1 && issued < count) issue();
+  }
+  tc_fence_before();
+  __syncthreads();  // TMEM address ready
+  tc_fence_after();
+  const uint32_t tmem = tmem_slot;
+
+  if (warp < 4) {
+    // ------------------------------------------------------------ tensor warps
+    TileTrack ta{}, ts{};
+    ta.start(args, u_begin);
+    ts.start(args, u_begin);
+    {
+      const float* fv = args.m[ta.j].fval_in;
+      const int rho = args.m[ta.j].rho_in;
+      __nv_bfloat16* ban = reinterpret_cast<__nv_bfloat16*>(bops);
+      float* bsy = reinterpret_cast<float*>(bops + 4096);
+      for (int i = tid; i < 1024; i += 128) {
+        const int r = i >> 5, k = i & 31;
+        const float dk = d4(fv, rho, k, r);  // D4[k][r]
+        const __nv_bfloat16 hi = __float2bfloat16_rn(dk);
+        const __nv_bfloat16 lo = __float2bfloat16_rn(dk - __bfloat162float(hi));
+        ban[can_bf16_off(r, k) / 2] = hi;
+        ban[can_bf16_off(32 + r, k) / 2] = lo;
+        bsy[can_f32_off(r, k)] = __uint_as_float(to_tf32(d4(fv, rho, r, k)));  // D4[r][k]
+      }
+      fence_async_smem();
+      tensor_bar();
+    }
+    const uint32_t id_an = umma_idesc(1, 128, 64), id_sy = umma_idesc(2, 128, 32);
+    const uint64_t d_ban = umma_sdesc(smem_u32(bops), 128, 512);
+    const uint64_t d_bsy = umma_sdesc(smem_u32(bops + 4096), 128, 1024);
+    uint32_t syn_ph = 0;
+    bool failed = false, syn_pending = false;
+    const uint32_t lane_base = static_cast<uint32_t>(32 * warp) << 16;
+    const int r0 = 32 * warp + lane;  // this thread's group (one 128-group tile)
+    // synthesis matrix, in registers
+    int js = -1, N2 = 0, Gm2 = 0, Gn2 = 0;
+    bool on_y = false, on_x = false;
+    __nv_bfloat16 *Y2 = nullptr, *X2 = nullptr;
+    int64_t ldy2 = 0, ldx2 = 0, ubeg2 = 0;
+    float seff2 = 0.f;
+    auto load_syn = [&](int j) {
+      js = j;
+      Y2 = static_cast<__nv_bfloat16*>(args.m[j].Y);
+      X2 = static_cast<__nv_bfloat16*>(args.m[j].dX);
+      ldy2 = args.m[j].ldy;
+      ldx2 = args.m[j].ldx;
+      ubeg2 = args.m[j].ubeg;
+      N2 = args.m[j].N;
+      Gm2 = args.m[j].m / FFB_GROUP;
+      Gn2 = args.m[j].n / FFB_GROUP;
+      seff2 = args.m[j].seff;
+      const uint8_t* plan = args.m[j].plan;
+      const FfbPlanHeader& h = hdr(plan);
+      on_y = F && r0 < Gm2 && __ldg(table<uint32_t>(plan, h.off_zmask) + r0) != 0u;
+      on_x = D && r0 < Gn2 && __ldg(table<uint32_t>(plan, h.off_gmask) + r0) != 0u;
+    };
+    for (int s = 0; s < count + 2; ++s) {
+      const int i2 = s - 2;
+      const bool syn = SYN && i2 >= 0;
+      const bool ana = s < count;
+      // both rows of unit s + S - 1 into the stage unit s - 1 used (its MMAs completed last step)
+      if (tid == kIssuer && issued < count) issue();
+      // synthesis of unit s-2 (operands written last step): threads 64 (Y) and 96 (dX)
+      int64_t t2 = 0;
+      int Tc2 = 0;
+      if (syn) {
+        ts.advance(args, u_begin + i2);
+        if (ts.j != js) load_syn(ts.j);
+        t2 = 2 * (u_begin + i2 - ubeg2);
+        Tc2 = min(2, static_cast<int>(N2 - t2));
+        if (lane == 0 && warp >= 2) {
+          const int side = warp & 1;
+          if (side == 0 ? F : D) {
+            tc_fence_after();
+            for (int k = 0; k < Tc2; ++k) {
+              const float* A = rzg + k * args.rzg_tok + (side == 0 ? args.set_oRZ : args.set_oRG);
+              const uint64_t abase = umma_sdesc(smem_u32(A), 128, 1024);
+              const uint32_t d = tmem + kTcColSyn + (2 * k + side) * 32;
+#pragma unroll
+              for (int ks = 0; ks < 4; ++ks)
+                umma_tf32(d, abase + ((ks * 256) >> 4), d_bsy + ((ks * 256) >> 4), id_sy, ks > 0);
+            }
+            umma_commit(syn_bar);
+          } else {
+            mbar_arrive(syn_bar);
+          }
+        }
+      }
+      // output rows of unit s-2 for this thread's group (read now, used after the MMAs)
+      uint4 yp[2][2][4];
+      if (syn) {
+#pragma unroll
+        for (int k = 0; k < 2; ++k) {
+          if (k < Tc2) {
+            if (on_y) {
+              const uint4* p = reinterpret_cast<const uint4*>(Y2 + (t2 + k) * ldy2 + 32 * r0);
+#pragma unroll
+              for (int j = 0; j < 4; ++j) yp[k][0][j] = p[j];
+            }
+            if (on_x) {
+              const uint4* p = reinterpret_cast<const uint4*>(X2 + (t2 + k) * ldx2 + 32 * r0);
+#pragma unroll
+              for (int j = 0; j < 4; ++j) yp[k][1][j] = p[j];
+            }
+          }
+        }
+      }
+      // analysis of unit s once its rows have landed: threads 0 (X) and 32 (dY)
+      if (ana && lane == 0 && warp < 2) {
+        const int side = warp;
+        ta.advance(args, u_begin + s);
+        const int64_t t0 = 2 * (u_begin + s - args.m[ta.j].ubeg);
+        const int Tc0 = min(2, static_cast<int>(args.m[ta.j].N - t0));
+        const bool landed = tc_wait_bounded(bar + (s % S), static_cast<uint32_t>((s / S) & 1));
+        if (!landed) failed = true;
+        if (landed && (side == 0 ? NEED_V : NEED_U)) {
+          tc_fence_after();
+          const uint32_t st0 = smem_u32(stg0 + (s % S) * args.stage);
+          for (int k = 0; k < Tc0; ++k) {
+            const uint32_t abase = st0 + (side == 0 ? k * args.tok_x : args.xbox_u + k * args.tok_u);
+            const uint32_t d = tmem + (2 * k + side) * 64;
+#pragma unroll
+            for (int ks = 0; ks < 2; ++ks)
+              umma_f16(d, umma_sdesc_sw64(abase + ks * 32), d_ban + ((ks * 256) >> 4), id_an, ks > 0);
+          }
+          umma_commit(ana_bar);
+        } else {
+          mbar_arrive(ana_bar);  // keeps the phase count; a failure is seen below
+        }
+      }
+      failed = tensor_bar_or(failed);
+      // synthesis results: y += seff * delta for groups with support entries
+      if (syn && !failed) {
+        const bool ok = tc_wait_bounded(syn_bar, syn_ph);
+        if (ok)
+          syn_ph ^= 1u;
+        else
+          syn_pending = true;
+        failed = tensor_bar_or(!ok);
+        tc_fence_after();
+        if (!failed) {
+#pragma unroll
+          for (int k = 0; k < 2; ++k) {
+            if (k >= Tc2) break;
+#pragma unroll
+            for (int side = 0; side < 2; ++side) {
+              if (!(side == 0 ? F : D)) continue;
+              float v[32];
+              tmem_ld32(tmem + lane_base + kTcColSyn + (2 * k + side) * 32, v);
+              if (side == 0 ? on_y : on_x) {
+                uint4* p = reinterpret_cast<uint4*>(side == 0 ? Y2 + (t2 + k) * ldy2 + 32 * r0
+                                                              : X2 + (t2 + k) * ldx2 + 32 * r0);
+#pragma unroll
+                for (int j = 0; j < 4; ++j) p[j] = axpy8(yp[k][side][j], v + 8 * j, seff2);
+              }
+            }
+          }
+        }
+      }
+      tc_fence_before();
+      if (__syncthreads_or(failed)) break;
+    }
+    if (failed) {
+      if (tid == 0) atomicAdd(&g_wait_timeouts, 1u);
+      if (syn_pending && tid == 64) mbar_wait_bounded(syn_bar, syn_ph);  // synthesis MMAs in flight (bounded)
+      if (tid == kIssuer) {
+        for (int i = issued > S ? issued - S : 0; i < issued; ++i)
+          mbar_wait_bounded(bar + (i % S), static_cast<uint32_t>((i / S) & 1));
+      }
+    }
+  } else {
+    // ------------------------------------------------------------ SpMM warps
+    const int st = tid - 128;
+    Chunk<MODE, true, false> ch;
+    float dc[kEreg];
+#pragma unroll
+    for (int e = 0; e < kEreg; ++e) dc[e] = 0.f;
+    TileTrack tp{}, tq{};
+    tp.start(args, u_begin);
+    tq.start(args, u_begin);
+    uint32_t ana_ph = 0, syn_ph = 0;
+    const int aside = (warp - 4) >> 2;  // analysis results written: warps 4-7 V (X), 8-11 U (dY)
+    const uint32_t alane = static_cast<uint32_t>(32 * (warp & 3)) << 16;
+    const int ar = 32 * (warp & 3) + lane;
+    int cur = -1, mcur = 0, ncur = 0;
+    const uint8_t* splan = nullptr;
+    int4* fixc = reinterpret_cast<int4*>(smem + args.fixc);
+    int nfZ = 0, nfix = 0;
+    bool zero_pending = true;
+    bool failed = false, ana_open = false;  // analysis MMAs of this step not yet waited for
+    for (int s = 0; s < count + 2; ++s) {
+      const int i1 = s - 1;
+      const bool work = i1 >= 0 && i1 < count;
+      const bool syn = SYN && s >= 2;
+      const bool ana = s < count;
+      ana_open = ana;
+      if (work) {
+        tp.advance(args, u_begin + i1);
+        if (tp.j != cur) {
+          if constexpr (C) {
+            if (cur >= 0) {
+              float* dst = args.partial + static_cast<size_t>(blockIdx.x + cur) * args.stride;
+              pipe_flush(splan, dst, dc, st);
+            }
+          }
+          cur = tp.j;
+          splan = args.m[cur].plan;
+          mcur = args.m[cur].m;
+          ncur = args.m[cur].n;
+          tc2_load_chunk<MODE>(ch, splan, args.m[cur].c_val, st);
+#pragma unroll
+          for (int e = 0; e < kEreg; ++e) dc[e] = 0.f;
+          zero_pending = true;
+          if constexpr (SYN) {
+            const FfbPlanHeader& h = hdr(splan);
+            nfZ = F ? h.nfixZ : 0;
+            nfix = nfZ + (D ? h.nfixG : 0);
+            for (int i = st; i < nfix; i += kTcSpmm)
+              fixc[i] = i < nfZ ? __ldg(table<int4>(splan, h.off_fixZ) + i)
+                                : __ldg(table<int4>(splan, h.off_fixG) + (i - nfZ));
+          }
+        }
+        // dC first: column-path gathers only, no stores yet
+        if constexpr (C) {
+          float2 vk = make_float2(0.f, 0.f);
+#pragma unroll
+          for (int e0 = 0; e0 < kEreg; e0 += B) {
+            if (e0 < ch.EG) {
+              float2 ub[B], vb[B];
+#pragma unroll
+              for (int e = 0; e < B; ++e) {
+                ub[e] = U2[ch.ga[e0 + e] & 0xFFFFu];
+                const int ep = e0 + e - 1;
+                vb[e] = (ep < 0 || ch.gb[e0 + e] != ch.gb[ep]) ? V2[ch.gb[e0 + e]] : make_float2(0.f, 0.f);
+              }
+#pragma unroll
+              for (int e = 0; e < B; ++e) {
+                const int ep = e0 + e - 1;
+                if (ep < 0 || ch.gb[e0 + e] != ch.gb[ep]) vk = vb[e];
+                dc[e0 + e] = fmaf(ub[e].x, vk.x, fmaf(ub[e].y, vk.y, dc[e0 + e]));
+              }
+            }
+          }
+        }
+      }
+      // RZ / RG are free once the synthesis MMAs of this step have read them
+      if (syn) {
+        const bool ok = tc_wait_bounded(syn_bar, syn_ph);
+        if (ok) syn_ph ^= 1u;
+        failed = spmm_bar_or(failed || !ok);  // uniform before the barriers below
+      }
+      if (work && !failed) {
+        if constexpr (SYN) {
+          if (zero_pending) {
+            for (int x = st; x < 2 * args.rzg_tok; x += kTcSpmm) rzg[x] = 0.f;
+            zero_pending = false;
+            tc_spmm_bar();
+          }
+          float* RZ0 = rzg + args.set_oRZ;
+          float* RZ1 = RZ0 + args.rzg_tok;
+          float* RG0 = rzg + args.set_oRG;
+          float* RG1 = RG0 + args.rzg_tok;
+          if constexpr (F) {
+            float2 acc = make_float2(0.f, 0.f);
+#pragma unroll
+            for (int e0 = 0; e0 < kEreg; e0 += B) {
+              if (e0 < ch.EZ) {
+                float2 v[B];
+#pragma unroll
+                for (int e = 0; e < B; ++e) v[e] = V2[ch.zb[e0 + e] & 0xFFFFu];
+#pragma unroll
+                for (int e = 0; e < B; ++e) {
+                  acc.x = fmaf(ch.zc[e0 + e], v[e].x, acc.x);
+                  acc.y = fmaf(ch.zc[e0 + e], v[e].y, acc.y);
+                  const uint32_t sz = ch.zb[e0 + e] >> 16;
+                  if (sz != FFB_NO_STORE) {
+                    RZ0[sz] = acc.x;
+                    RZ1[sz] = acc.y;
+                    acc = make_float2(0.f, 0.f);
+                  }
+                }
+              }
+            }
+          }
+          if constexpr (D) {
+            float2 acc = make_float2(0.f, 0.f);
+#pragma unroll
+            for (int e0 = 0; e0 < kEreg; e0 += B) {
+              if (e0 < ch.EG) {
+                float2 ub[B];
+#pragma unroll
+                for (int e = 0; e < B; ++e) ub[e] = U2[ch.ga[e0 + e] & 0xFFFFu];
+#pragma unroll
+                for (int e = 0; e < B; ++e) {
+                  acc.x = fmaf(ch.gc[e0 + e], ub[e].x, acc.x);
+                  acc.y = fmaf(ch.gc[e0 + e], ub[e].y, acc.y);
+                  const uint32_t sg = ch.ga[e0 + e] >> 16;
+                  if (sg != FFB_NO_STORE) {
+                    RG0[sg] = acc.x;
+                    RG1[sg] = acc.y;
+                    acc = make_float2(0.f, 0.f);
+                  }
+                }
+              }
+            }
+          }
+          if (nfix > 0) {
+            // rows (columns) split between chunks: add the overflow pieces
+            tc_spmm_bar();
+            for (int i = st; i < nfix; i += kTcSpmm) {
+              const int4 it = fixc[i];
+              const bool z = i < nfZ;
+              const int dst = tc_slot(it.x, z ? mcur : ncur);
+#pragma unroll
+              for (int k = 0; k < 2; ++k) {
+                float* R = rzg + k * args.rzg_tok + (z ? args.set_oRZ : args.set_oRG);
+                float sacc = R[dst];
+                for (int c2 = 0; c2 < it.z; ++c2) sacc += R[it.y + c2];
+                R[dst] = sacc;
+              }
+            }
+          }
+          fence_async_smem();  // RZ / RG are read by the tensor cores next step
+        }
+      }
+      // analysis results of unit s -> V / U (float2: both tokens), once every
+      // SpMM warp finished gathering from them and the MMAs completed
+      if (ana && !failed) {
+        tc_spmm_bar();
+        const bool ok = tc_wait_bounded(ana_bar, ana_ph);
+        if (ok) {
+          ana_ph ^= 1u;
+          ana_open = false;
+        }
+        failed = !ok;
+        tc_fence_after();
+        const bool on = aside == 0 ? NEED_V : NEED_U;
+        if (ok && on) {
+          tq.advance(args, u_begin + s);
+          const int G = (aside == 0 ? args.m[tq.j].n : args.m[tq.j].m) / FFB_GROUP;
+          const int64_t t0 = 2 * (u_begin + s - args.m[tq.j].ubeg);
+          const bool two = args.m[tq.j].N - t0 >= 2;
+          float2* dst = aside == 0 ? V2 : U2;
+#pragma unroll
+          for (int q8 = 0; q8 < 4; ++q8) {  // coefficients 8 q8 .. 8 q8 + 7
+            float h0[8], l0[8], h1[8], l1[8];
+            const uint32_t c0 = tmem + alane + (0 * 2 + aside) * 64 + 8 * q8;
+            const uint32_t c1 = tmem + alane + (1 * 2 + aside) * 64 + 8 * q8;
+            tmem_ld8x4(c0, c0 + 32, c1, c1 + 32, h0, l0, h1, l1);
+            if (ar < G) {
+#pragma unroll
+              for (int j = 0; j < 4; ++j) {  // chunk q = 4 q8 + j: coefficients 2q, 2q + 1
+                const int q = 4 * q8 + j;
+                const float a0 = h0[2 * j] + l0[2 * j], a1 = h0[2 * j + 1] + l0[2 * j + 1];
+                const float b0 = two ? h1[2 * j] + l1[2 * j] : 0.f, b1 = two ? h1[2 * j + 1] + l1[2 * j + 1] : 0.f;
+                *reinterpret_cast<float4*>(dst + 32 * ar + 2 * (q ^ (ar & 7))) = make_float4(a0, b0, a1, b1);
+              }
+            }
+          }
+        }
+      }
+      tc_fence_before();
+      if (__syncthreads_or(failed)) {
+        failed = true;
+        break;
+      }
+    }
+    if (failed) {
+      // analysis MMAs of the failing step may still be in flight (bounded)
+      if (st == 0 && ana_open) mbar_wait_bounded(ana_bar, ana_ph);
+    } else {
+      if constexpr (C) {
+        if (cur >= 0) {
+          float* dst = args.partial + static_cast<size_t>(blockIdx.x + cur) * args.stride;
+          pipe_flush(splan, dst, dc, st);
+        }
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTcTmemCols) : "memory");
+  }
+}
+
+}  // namespace ffb

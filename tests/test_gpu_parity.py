@@ -68,7 +68,7 @@ def test_single_256_fp32(ops, unit):
     check_batch(b, ops)
 
 
-@pytest.mark.parametrize("kernel", ["tile", "pipe", "tc"])
+@pytest.mark.parametrize("kernel", ["tile", "pipe", "tc", "tc2"])
 @pytest.mark.parametrize("N", [37, 1, 4])
 def test_roberta_base_all_matrices(N, kernel, monkeypatch):
     monkeypatch.setenv("FRAMEFB_KERNEL", kernel)
@@ -77,7 +77,7 @@ def test_roberta_base_all_matrices(N, kernel, monkeypatch):
     check_batch(b, ALL)
 
 
-@pytest.mark.parametrize("kernel", ["tile", "pipe", "tc"])
+@pytest.mark.parametrize("kernel", ["tile", "pipe", "tc", "tc2"])
 def test_vit_b16_mixed_shapes(kernel, monkeypatch):
     # many matrices of three shapes per launch: CTAs cross matrix boundaries
     monkeypatch.setenv("FRAMEFB_KERNEL", kernel)
@@ -94,7 +94,7 @@ def test_llama2_shape_small_n():
     check_batch(b, ALL)
 
 
-@pytest.mark.parametrize("kernel", ["tc", "pipe", "tile"])
+@pytest.mark.parametrize("kernel", ["tc2", "tc", "pipe", "tile"])
 @pytest.mark.parametrize("ops", [ffb.OP_FORWARD, ffb.OP_BACKWARD_DX, ffb.OP_GRAD_COEFF,
                                  ffb.OP_BACKWARD_DX | ffb.OP_GRAD_COEFF, ALL])
 def test_bf16_kernels_every_mode(kernel, ops, monkeypatch):
