@@ -122,19 +122,21 @@ def algorithmic_bytes(batch) -> int:
     return total
 
 
-# sources of the dominant kernel (bf16: the tcgen05 kernel unless FRAMEFB_KERNEL forces another)
-KERNEL_SOURCES = ("framefb_kernels.cuh", "framefb_mma.cuh", "framefb_pipe.cuh", "framefb_tc.cuh", "plan_layout.h")
+# sources of the dominant kernel (bf16: the two-token tcgen05 kernel unless
+# FRAMEFB_KERNEL selects another) and of the plan builder that shapes it
+KERNEL_SOURCES = ("framefb_kernels.cuh", "framefb_mma.cuh", "framefb_pipe.cuh", "framefb_tc.cuh", "framefb_tc2.cuh",
+                  "plan_layout.h", "framefb_host.cpp")
 
 
 def kernel_choice():
-    k = os.environ.get("FRAMEFB_KERNEL", "tc")
-    return k if k in ("tile", "pipe") else "tc"
+    k = os.environ.get("FRAMEFB_KERNEL", "tc2")
+    return k if k in ("tile", "pipe", "tc") else "tc2"
 
 
 def launches_per_step(nmats: int) -> int:
     """Kernel launches of one fused step: a tile kernel and a dC reduction per
-    launch chunk (the tcgen05 kernel takes 64 matrices per launch, the others 256)."""
-    chunk = 64 if kernel_choice() == "tc" else 256
+    launch chunk (the tcgen05 kernels take 64 matrices per launch, the others 256)."""
+    chunk = 64 if kernel_choice() in ("tc", "tc2") else 256
     return 2 * ((nmats + chunk - 1) // chunk)
 
 
@@ -337,7 +339,8 @@ def main():
                "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                             "frac": achieved / peak,
                             "traffic": measured_traffic() if args.mats is None and args.workload is None else None, "peak_kind": peak_kind,
-                            "kernel": {"tc": "tc_tile_kernel<fwd|dx|dc>", "pipe": "pipe_tile_kernel<fwd|dx|dc>",
+                            "kernel": {"tc2": "tc2_tile_kernel<fwd|dx|dc>", "tc": "tc_tile_kernel<fwd|dx|dc>",
+                                       "pipe": "pipe_tile_kernel<fwd|dx|dc>",
                                        "tile": "mma_tile_kernel<fwd|dx|dc>"}[kernel_choice()] + " + dc_reduce",
                             "kernel_ms": kernel_ms,
                             "algorithmic_bytes": alg, "algorithmic_bytes_per_launch": alg / launches,
