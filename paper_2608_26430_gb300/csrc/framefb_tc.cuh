@@ -206,6 +206,20 @@ __device__ __forceinline__ void tmem_ld16x2(uint32_t ta, uint32_t tb, float (&v)
 }
 
 // y (8 bf16 of one 16-byte chunk) += seff * d[0..7]
+// 32 contiguous bytes of global memory (one sector) in one access: a warp whose
+// lanes stride 64 bytes apart (one 32-coordinate bf16 group per lane) then
+// touches each 128-byte line once per instruction instead of twice.
+__device__ __forceinline__ void ld_global_256(const void* p, uint4& a, uint4& b) {
+  asm volatile("ld.global.v8.u32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+               : "=r"(a.x), "=r"(a.y), "=r"(a.z), "=r"(a.w), "=r"(b.x), "=r"(b.y), "=r"(b.z), "=r"(b.w)
+               : "l"(p));
+}
+__device__ __forceinline__ void st_global_256(void* p, const uint4& a, const uint4& b) {
+  asm volatile("st.global.v8.u32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"l"(p), "r"(a.x), "r"(a.y), "r"(a.z), "r"(a.w),
+               "r"(b.x), "r"(b.y), "r"(b.z), "r"(b.w)
+               : "memory");
+}
+
 __device__ __forceinline__ uint4 axpy8(uint4 y, const float* d, float seff) {
   uint32_t w[4] = {y.x, y.y, y.z, y.w};
 #pragma unroll

@@ -211,7 +211,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2_tile_kernel(const __grid_co
     const int r0 = 32 * warp + lane;  // this thread's group (one 128-group tile)
     // synthesis matrix, in registers
     int js = -1, N2 = 0, Gm2 = 0, Gn2 = 0;
-    bool on_y = false, on_x = false;
+    bool on_y = false, on_x = false, wide_y = false, wide_x = false;
     __nv_bfloat16 *Y2 = nullptr, *X2 = nullptr;
     int64_t ldy2 = 0, ldx2 = 0, ubeg2 = 0;
     float seff2 = 0.f;
@@ -226,6 +226,9 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2_tile_kernel(const __grid_co
       Gm2 = args.m[j].m / FFB_GROUP;
       Gn2 = args.m[j].n / FFB_GROUP;
       seff2 = args.m[j].seff;
+      // 256-bit row accesses need 32-byte aligned rows (the interface promises 16)
+      wide_y = (reinterpret_cast<uintptr_t>(Y2) & 31u) == 0 && (ldy2 & 15) == 0;
+      wide_x = (reinterpret_cast<uintptr_t>(X2) & 31u) == 0 && (ldx2 & 15) == 0;
       const uint8_t* plan = args.m[j].plan;
       const FfbPlanHeader& h = hdr(plan);
       on_y = F && r0 < Gm2 && __ldg(table<uint32_t>(plan, h.off_zmask) + r0) != 0u;
@@ -269,15 +272,17 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2_tile_kernel(const __grid_co
 #pragma unroll
         for (int k = 0; k < 2; ++k) {
           if (k < Tc2) {
-            if (on_y) {
-              const uint4* p = reinterpret_cast<const uint4*>(Y2 + (t2 + k) * ldy2 + 32 * r0);
 #pragma unroll
-              for (int j = 0; j < 4; ++j) yp[k][0][j] = p[j];
-            }
-            if (on_x) {
-              const uint4* p = reinterpret_cast<const uint4*>(X2 + (t2 + k) * ldx2 + 32 * r0);
+            for (int side = 0; side < 2; ++side) {
+              if (!(side == 0 ? on_y : on_x)) continue;
+              const __nv_bfloat16* p = side == 0 ? Y2 + (t2 + k) * ldy2 + 32 * r0 : X2 + (t2 + k) * ldx2 + 32 * r0;
+              if (side == 0 ? wide_y : wide_x) {
+                ld_global_256(p, yp[k][side][0], yp[k][side][1]);
+                ld_global_256(p + 16, yp[k][side][2], yp[k][side][3]);
+              } else {
 #pragma unroll
-              for (int j = 0; j < 4; ++j) yp[k][1][j] = p[j];
+                for (int j = 0; j < 4; ++j) yp[k][side][j] = reinterpret_cast<const uint4*>(p)[j];
+              }
             }
           }
         }
@@ -325,10 +330,17 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2_tile_kernel(const __grid_co
               float v[32];
               tmem_ld32(tmem + lane_base + kTcColSyn + (2 * k + side) * 32, v);
               if (side == 0 ? on_y : on_x) {
-                uint4* p = reinterpret_cast<uint4*>(side == 0 ? Y2 + (t2 + k) * ldy2 + 32 * r0
-                                                              : X2 + (t2 + k) * ldx2 + 32 * r0);
+                __nv_bfloat16* p = side == 0 ? Y2 + (t2 + k) * ldy2 + 32 * r0 : X2 + (t2 + k) * ldx2 + 32 * r0;
+                if (side == 0 ? wide_y : wide_x) {
 #pragma unroll
-                for (int j = 0; j < 4; ++j) p[j] = axpy8(yp[k][side][j], v + 8 * j, seff2);
+                  for (int j = 0; j < 2; ++j)
+                    st_global_256(p + 16 * j, axpy8(yp[k][side][2 * j], v + 16 * j, seff2),
+                                  axpy8(yp[k][side][2 * j + 1], v + 16 * j + 8, seff2));
+                } else {
+#pragma unroll
+                  for (int j = 0; j < 4; ++j)
+                    reinterpret_cast<uint4*>(p)[j] = axpy8(yp[k][side][j], v + 8 * j, seff2);
+                }
               }
             }
           }

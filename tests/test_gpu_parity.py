@@ -177,32 +177,36 @@ def test_empty_support_is_a_no_op():
     assert torch.equal(Y, Y0)
 
 
-def test_strided_rows_and_untouched_padding():
+@pytest.mark.parametrize("pad,off", [(64, 0), (8, 8)])
+def test_strided_rows_and_untouched_padding(pad, off):
+    # (64, 0): rows 32-byte aligned; (8, 8): rows only 16-byte aligned (leading
+    # dimension = 8 mod 16 elements, region starting 16 bytes into the row)
     w = wl.WORKLOADS["roberta_base_qv"]
     N, n, m = 19, 768, 768
     src = AdapterBatch(w, DEV, N=N, indices=[0], ops=ALL)
     bb = src.bufs[0]
-    pad = 64
     Xp = torch.zeros(N, n + pad, device=DEV, dtype=torch.bfloat16)
-    Xp[:, :n] = bb.X
+    Xp[:, off:off + n] = bb.X
     dYp = torch.zeros(N + 2, m + pad, device=DEV, dtype=torch.bfloat16)
-    dYp[:N, :m] = bb.dY
+    dYp[:N, off:off + m] = bb.dY
     # padding holds sentinels; the active region starts at zero so that the
     # bf16 result is the delta itself
     Yp = torch.full((N + 2, m + pad), 3.0, device=DEV, dtype=torch.bfloat16)
-    Yp[:N, :m] = 0
+    Yp[:N, off:off + m] = 0
     dXp = torch.full((N, n + pad), 5.0, device=DEV, dtype=torch.bfloat16)
-    dXp[:, :n] = 0
+    dXp[:, off:off + n] = 0
     dC = torch.zeros(w.nnz, device=DEV)
     mat = ffb.make_mat(src.dev_frames[n], src.dev_frames[m], src.plans[(m, n)], src.plan_dev[(m, n)], bb.c_val,
-                       bb.scale, N, X=Xp, dX=dXp, dY=dYp, Y=Yp, dC=dC, ldx=n + pad, ldy=m + pad)
+                       bb.scale, N, X=Xp[:, off:], dX=dXp[:, off:], dY=dYp[:, off:], Y=Yp[:, off:], dC=dC,
+                       ldx=n + pad, ldy=m + pad)
     ws = ffb.workspace([mat], ALL, DEV)
     ffb.framefb_run([mat], ALL, ffb.FRAMEFB_BF16, ws)
     torch.cuda.synchronize()
-    assert torch.all(Yp[:, m:] == 3.0) and torch.all(Yp[N:, :] == 3.0) and torch.all(dXp[:, n:] == 5.0)
+    assert torch.all(Yp[:, off + m:] == 3.0) and torch.all(Yp[:, :off] == 3.0) and torch.all(Yp[N:, :] == 3.0)
+    assert torch.all(dXp[:, off + n:] == 5.0) and torch.all(dXp[:, :off] == 5.0)
     e = Expect(src, 0)
-    assert_bf16(host64(Yp[:N, :m]), e.y(host64(bb.X), np.zeros((N, m))), what="Y strided")
-    assert_bf16(host64(dXp[:, :n]), e.dx(host64(bb.dY), np.zeros((N, n))), what="dX strided")
+    assert_bf16(host64(Yp[:N, off:off + m]), e.y(host64(bb.X), np.zeros((N, m))), what="Y strided")
+    assert_bf16(host64(dXp[:, off:off + n]), e.dx(host64(bb.dY), np.zeros((N, n))), what="dX strided")
     assert_bf16(host64(dC), e.dc(host64(bb.X), host64(bb.dY)), what="dC strided")
 
 
