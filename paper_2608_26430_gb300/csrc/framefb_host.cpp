@@ -8,8 +8,11 @@
 #include <cmath>
 #include <cstdlib>
 #include <cstring>
+#include <exception>
 #include <new>
+#include <system_error>
 #include <unordered_set>
+#include <thread>
 #include <vector>
 
 extern "C" const char* framefb_status_string(int32_t status) {
@@ -331,9 +334,13 @@ struct PathBanks {
 // decreasing); a piece that fits nowhere is split over the roomiest chunks.
 // The pieces are then moved (equal-length pieces swapped between chunks,
 // entries reordered inside a piece) by a deterministic annealing search that
-// lowers shared-memory bank conflicts: for every SpMM instruction (32
-// consecutive chunks at one entry step) it counts the lanes that share a bank
-// with an earlier lane, over the gathers, the key reloads and the stores.
+// lowers shared-memory wavefronts: for every SpMM instruction (32 consecutive
+// chunks at one entry step) it counts the wavefronts of the gathers and key
+// reloads (per half-warp: the largest number of lanes on one bank pair) and
+// of the two run-sum stores (per warp: the largest number on one bank), plus
+// a small sum-of-squares term over the same bank counts that keeps the
+// search moving on plateaus of the wavefront count.  Half of the swaps start
+// from a lane that conflicts in a random instruction.
 // A chunk's pieces are consecutive, so each piece sums in registers and
 // stores once, at its last position: the first piece of a key (in chunk
 // order) writes the key's own slot, later pieces write overflow slots
@@ -424,23 +431,39 @@ void pack_runs(const std::vector<Entry>& ent, int32_t P, int32_t E, int32_t base
     const Placed& q = pl[piece_of[idx]];
     return q.off + q.len - 1 == e;
   };
+  // 16 x wavefronts + 4 x sum of squared bank counts of one instruction
   auto group_cost = [&](int32_t w, int32_t e) {
     uint8_t cg[2][16] = {}, ck[2][16] = {}, cs[32] = {0};
-    int32_t ex = 0;
     for (int32_t l = 0; l < 32; ++l) {
       const int32_t p = 32 * w + l;
       if (p >= P) break;
       const int32_t idx = grid[static_cast<size_t>(p) * E + e];
       if (idx < 0) continue;
       const int32_t h = l >> 4;
-      ex += cg[h][bk.gather[idx]]++ > 0;
+      cg[h][bk.gather[idx]]++;
       if (has_key) {
         const int32_t prev = e > 0 ? grid[static_cast<size_t>(p) * E + e - 1] : -1;
-        if (prev < 0 || ent[prev].key0 != ent[idx].key0) ex += ck[h][bk.key[idx]]++ > 0;
+        if (prev < 0 || ent[prev].key0 != ent[idx].key0) ck[h][bk.key[idx]]++;
       }
-      if (is_end(idx, e)) ex += 2 * (cs[bk.store[idx]]++ > 0);  // two stores: one per token
+      if (is_end(idx, e)) cs[bk.store[idx]]++;
     }
-    return ex;
+    int32_t wf = 0, sq = 0;
+    for (int h = 0; h < 2; ++h) {
+      int32_t mg = 0, mk = 0;
+      for (int b = 0; b < 16; ++b) {
+        mg = std::max<int32_t>(mg, cg[h][b]);
+        mk = std::max<int32_t>(mk, ck[h][b]);
+        sq += cg[h][b] * cg[h][b] + ck[h][b] * ck[h][b];
+      }
+      wf += mg + mk;
+    }
+    int32_t ms = 0;
+    for (int b = 0; b < 32; ++b) {
+      ms = std::max<int32_t>(ms, cs[b]);
+      sq += 2 * cs[b] * cs[b];  // two stores: one per token
+    }
+    wf += 2 * ms;
+    return 16 * wf + 4 * sq;
   };
   std::vector<std::vector<int32_t>> by_len(E + 1);
   std::vector<int32_t> multi;  // pieces of two or more entries
@@ -449,7 +472,7 @@ void pack_runs(const std::vector<Entry>& ent, int32_t P, int32_t E, int32_t base
     if (pl[k].len >= 2) multi.push_back(static_cast<int32_t>(k));
   }
   SplitMix64 rng{0x6A09E667F3BCC909ull ^ static_cast<uint64_t>(nnz)};
-  const int64_t iters = std::min<int64_t>(static_cast<int64_t>(nnz) * 200, 4000000);
+  const int64_t iters = std::min<int64_t>(static_cast<int64_t>(nnz) * 600, 12000000);
   std::vector<std::pair<int32_t, int32_t>> aff;
   auto add_group = [&](int32_t col, int32_t e) {
     if (e < 0 || e >= E) return;
@@ -482,10 +505,26 @@ void pack_runs(const std::vector<Entry>& ent, int32_t P, int32_t E, int32_t base
       };
       apply();
       const int32_t d = cost_of() - before;
-      if (d > 0 && rng.uniform_01() >= std::exp(-d / (0.6 * T + 1e-9))) apply();
+      if (d > 0 && rng.uniform_01() >= std::exp(-d / (3.0 * T + 1e-9))) apply();
     } else {
       // swap two pieces of the same length between chunks
-      const int32_t a = static_cast<int32_t>(rng.uniform_int(pl.size()));
+      int32_t a = static_cast<int32_t>(rng.uniform_int(pl.size()));
+      if (rng.next() & 1) {
+        // a piece holding a lane whose gather shares a bank pair in a random instruction
+        const int32_t w = static_cast<int32_t>(rng.uniform_int(W)), e = static_cast<int32_t>(rng.uniform_int(E));
+        uint8_t cg[2][16] = {};
+        int32_t cand[32], nc = 0;
+        for (int32_t l = 0; l < 32 && 32 * w + l < P; ++l) {
+          const int32_t idx = grid[static_cast<size_t>(32 * w + l) * E + e];
+          if (idx >= 0) cg[l >> 4][bk.gather[idx]]++;
+        }
+        for (int32_t l = 0; l < 32 && 32 * w + l < P; ++l) {
+          const int32_t idx = grid[static_cast<size_t>(32 * w + l) * E + e];
+          if (idx >= 0 && cg[l >> 4][bk.gather[idx]] > 1) cand[nc++] = idx;
+        }
+        if (nc == 0) continue;
+        a = piece_of[cand[rng.uniform_int(nc)]];
+      }
       const std::vector<int32_t>& same = by_len[pl[a].len];
       if (same.size() < 2) continue;
       const int32_t b = same[rng.uniform_int(same.size())];
@@ -503,7 +542,7 @@ void pack_runs(const std::vector<Entry>& ent, int32_t P, int32_t E, int32_t base
       };
       apply();
       const int32_t d = cost_of() - before;
-      if (d > 0 && rng.uniform_01() >= std::exp(-d / (0.6 * T + 1e-9))) apply();
+      if (d > 0 && rng.uniform_01() >= std::exp(-d / (3.0 * T + 1e-9))) apply();
     }
   }
 
@@ -595,8 +634,33 @@ extern "C" framefb_status framefb_plan_build(const framefb_frame* fin, const fra
       bkG.key[q] = static_cast<int8_t>(gather_bank(bycol[q].key0));
       bkG.store[q] = static_cast<int8_t>(store_bank(bycol[q].key0, n));
     }
-    pack_runs(byrow, P, EZ, m, m, bkZ, posZ, storeZ, fixZ, novfZ);
-    pack_runs(bycol, P, EG, n, n, bkG, posG, storeG, fixG, novfG);
+    // the two paths are independent searches: run them side by side (in
+    // sequence if no thread can be started); exceptions reach the caller's
+    // handler after the join
+    {
+      std::exception_ptr ez, eg;
+      auto run_z = [&]() {
+        try {
+          pack_runs(byrow, P, EZ, m, m, bkZ, posZ, storeZ, fixZ, novfZ);
+        } catch (...) {
+          ez = std::current_exception();
+        }
+      };
+      std::thread tz;
+      try {
+        tz = std::thread(run_z);
+      } catch (const std::system_error&) {
+        run_z();
+      }
+      try {
+        pack_runs(bycol, P, EG, n, n, bkG, posG, storeG, fixG, novfG);
+      } catch (...) {
+        eg = std::current_exception();
+      }
+      if (tz.joinable()) tz.join();
+      if (ez) std::rethrow_exception(ez);
+      if (eg) std::rethrow_exception(eg);
+    }
 
     FfbPlanHeader h;
     std::memset(&h, 0, sizeof(h));
