@@ -300,7 +300,7 @@ size_t tc2_smem_map(const framefb_mat* mats, int32_t nmats, int32_t ops, int S, 
     a->fixc_items = static_cast<int32_t>(nfix);
     a->mbar = static_cast<int32_t>(mbar);
   }
-  return mbar + 8 * static_cast<size_t>(S + 2);
+  return mbar + 8 * static_cast<size_t>(S + 3);  // stages, analysis, synthesis, RZ/RG written
 }
 
 // cuTensorMapEncodeTiled through the runtime's driver entry point (no link

@@ -11,14 +11,16 @@
 //     write-back of one group per lane conflict-free;
 //   * RZ and RG stay per token in the canonical tf32 K-major layout (they are
 //     the synthesis A operands);
-//   * shared memory holds one V/U set and one RZ/RG set (two tokens each):
-//     the SpMM warps first compute dC (gathers only), then wait until the
-//     synthesis MMAs of the step have read RZ/RG before the run sums (which
-//     gather again and store), and write the analysis results of the step
-//     into V/U only after all of them finished gathering;
-//   * eight MMA groups per step: analysis (token x side) issued by threads 0
-//     (X) and 32 (dY) on one barrier, synthesis by threads 64 (Y) and 96 (dX)
-//     on another.
+//   * shared memory holds one V/U set and one RZ/RG set (two tokens each).
+//     Step s: the SpMM warps wait until the synthesis MMAs of unit s-2 have
+//     read RZ/RG, run unit s-1 (one pass over the column path gives dC and
+//     G, one over the row path gives Z) and signal RZ/RG complete; the four
+//     tensor warps then issue the synthesis of unit s-1 at once (one
+//     (token, side) each), into the TMEM half of its parity, while the SpMM
+//     warps write the analysis results of unit s into V/U;
+//   * analysis (token x side) of unit s is issued by threads 0 (X) and 32
+//     (dY) at the start of the step; the tensor warps apply the synthesis of
+//     unit s-2 to the output rows.
 // Shapes: every group count a multiple of 8 and at most 128 (n, m <= 4096).
 // Waits are bounded as in tc_tile_kernel.
 #pragma once
@@ -128,6 +130,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2_tile_kernel(const __grid_co
   uint64_t* bar = reinterpret_cast<uint64_t*>(smem + args.mbar);
   uint64_t* ana_bar = bar + S;
   uint64_t* syn_bar = bar + S + 1;
+  uint64_t* rzg_bar = bar + S + 2;  // RZ / RG of the step's SpMM unit written
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
 
   const int64_t units = args.total_units;
@@ -139,7 +142,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2_tile_kernel(const __grid_co
   if (tid == 0) {
     for (int b = 0; b < S; ++b) mbar_init(bar + b, 1);
     mbar_init(ana_bar, 2);  // threads 0 and 32
-    mbar_init(syn_bar, 2);  // threads 64 and 96
+    mbar_init(syn_bar, 4);  // lane 0 of each tensor warp
+    mbar_init(rzg_bar, 1);  // SpMM thread 0
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (warp == 0) {
@@ -182,9 +186,10 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2_tile_kernel(const __grid_co
 
   if (warp < 4) {
     // ------------------------------------------------------------ tensor warps
-    TileTrack ta{}, ts{};
+    TileTrack ta{}, ts{}, tr{};  // units of the analysis (s), the output rows (s-2), the synthesis issue (s-1)
     ta.start(args, u_begin);
     ts.start(args, u_begin);
+    tr.start(args, u_begin);
     {
       const float* fv = args.m[ta.j].fval_in;
       const int rho = args.m[ta.j].rho_in;
@@ -205,8 +210,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2_tile_kernel(const __grid_co
     const uint32_t id_an = umma_idesc(1, 128, 64), id_sy = umma_idesc(2, 128, 32);
     const uint64_t d_ban = umma_sdesc(smem_u32(bops), 128, 512);
     const uint64_t d_bsy = umma_sdesc(smem_u32(bops + 4096), 128, 1024);
-    uint32_t syn_ph = 0;
-    bool failed = false, syn_pending = false;
+    uint32_t syn_ph = 0, rzg_ph = 0;
+    bool failed = false, syn_open = false;  // syn_open: a synthesis issued and not yet waited for
     const uint32_t lane_base = static_cast<uint32_t>(32 * warp) << 16;
     const int r0 = 32 * warp + lane;  // this thread's group (one 128-group tile)
     // synthesis matrix, in registers
@@ -235,40 +240,23 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2_tile_kernel(const __grid_co
       on_x = D && r0 < Gn2 && __ldg(table<uint32_t>(plan, h.off_gmask) + r0) != 0u;
     };
     for (int s = 0; s < count + 2; ++s) {
-      const int i2 = s - 2;
-      const bool syn = SYN && i2 >= 0;
+      const int i2 = s - 2, i1 = s - 1;
+      const bool epi = SYN && i2 >= 0;                // output rows of unit s-2
+      const bool iss = SYN && i1 >= 0 && i1 < count;  // synthesis of unit s-1, after its SpMM
       const bool ana = s < count;
       // both rows of unit s + S - 1 into the stage unit s - 1 used (its MMAs completed last step)
       if (tid == kIssuer && issued < count) issue();
-      // synthesis of unit s-2 (operands written last step): threads 64 (Y) and 96 (dX)
       int64_t t2 = 0;
       int Tc2 = 0;
-      if (syn) {
+      if (epi) {
         ts.advance(args, u_begin + i2);
         if (ts.j != js) load_syn(ts.j);
         t2 = 2 * (u_begin + i2 - ubeg2);
         Tc2 = min(2, static_cast<int>(N2 - t2));
-        if (lane == 0 && warp >= 2) {
-          const int side = warp & 1;
-          if (side == 0 ? F : D) {
-            tc_fence_after();
-            for (int k = 0; k < Tc2; ++k) {
-              const float* A = rzg + k * args.rzg_tok + (side == 0 ? args.set_oRZ : args.set_oRG);
-              const uint64_t abase = umma_sdesc(smem_u32(A), 128, 1024);
-              const uint32_t d = tmem + kTcColSyn + (2 * k + side) * 32;
-#pragma unroll
-              for (int ks = 0; ks < 4; ++ks)
-                umma_tf32(d, abase + ((ks * 256) >> 4), d_bsy + ((ks * 256) >> 4), id_sy, ks > 0);
-            }
-            umma_commit(syn_bar);
-          } else {
-            mbar_arrive(syn_bar);
-          }
-        }
       }
-      // output rows of unit s-2 for this thread's group (read now, used after the MMAs)
+      // output rows of unit s-2 for this thread's group (read now, used after the wait)
       uint4 yp[2][2][4];
-      if (syn) {
+      if (epi) {
 #pragma unroll
         for (int k = 0; k < 2; ++k) {
           if (k < Tc2) {
@@ -311,16 +299,17 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2_tile_kernel(const __grid_co
         }
       }
       failed = tensor_bar_or(failed);
-      // synthesis results: y += seff * delta for groups with support entries
-      if (syn && !failed) {
+      // synthesis results of unit s-2: y += seff * delta for groups with support entries
+      if (epi && !failed) {
         const bool ok = tc_wait_bounded(syn_bar, syn_ph);
-        if (ok)
+        if (ok) {
           syn_ph ^= 1u;
-        else
-          syn_pending = true;
+          syn_open = false;
+        }
         failed = tensor_bar_or(!ok);
         tc_fence_after();
         if (!failed) {
+          const uint32_t col0 = tmem + lane_base + kTcColSyn + 128 * static_cast<uint32_t>(i2 & 1);
 #pragma unroll
           for (int k = 0; k < 2; ++k) {
             if (k >= Tc2) break;
@@ -328,7 +317,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2_tile_kernel(const __grid_co
             for (int side = 0; side < 2; ++side) {
               if (!(side == 0 ? F : D)) continue;
               float v[32];
-              tmem_ld32(tmem + lane_base + kTcColSyn + (2 * k + side) * 32, v);
+              tmem_ld32(col0 + (2 * k + side) * 32, v);
               if (side == 0 ? on_y : on_x) {
                 __nv_bfloat16* p = side == 0 ? Y2 + (t2 + k) * ldy2 + 32 * r0 : X2 + (t2 + k) * ldx2 + 32 * r0;
                 if (side == 0 ? wide_y : wide_x) {
@@ -346,12 +335,41 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2_tile_kernel(const __grid_co
           }
         }
       }
+      // synthesis of unit s-1 once the SpMM warps have written its RZ / RG:
+      // lane 0 of tensor warp w issues (token w / 2, side w % 2) into the TMEM
+      // half of the unit's parity
+      if (iss && !failed && lane == 0) {
+        tr.advance(args, u_begin + i1);
+        const int64_t t1 = 2 * (u_begin + i1 - args.m[tr.j].ubeg);
+        const int Tc1 = min(2, static_cast<int>(args.m[tr.j].N - t1));
+        const int k = warp >> 1, side = warp & 1;
+        const bool ok = tc_wait_bounded(rzg_bar, rzg_ph);
+        if (ok)
+          rzg_ph ^= 1u;
+        else
+          failed = true;
+        if (ok && k < Tc1 && (side == 0 ? F : D)) {
+          tc_fence_after();
+          const float* A = rzg + k * args.rzg_tok + (side == 0 ? args.set_oRZ : args.set_oRG);
+          const uint64_t abase = umma_sdesc(smem_u32(A), 128, 1024);
+          const uint32_t d = tmem + kTcColSyn + 128 * static_cast<uint32_t>(i1 & 1) + (2 * k + side) * 32;
+#pragma unroll
+          for (int ks = 0; ks < 4; ++ks)
+            umma_tf32(d, abase + ((ks * 256) >> 4), d_bsy + ((ks * 256) >> 4), id_sy, ks > 0);
+          umma_commit(syn_bar);
+        } else {
+          mbar_arrive(syn_bar);  // keeps the phase count
+        }
+        syn_open = true;
+      }
       tc_fence_before();
       if (__syncthreads_or(failed)) break;
     }
     if (failed) {
-      if (tid == 0) atomicAdd(&g_wait_timeouts, 1u);
-      if (syn_pending && tid == 64) mbar_wait_bounded(syn_bar, syn_ph);  // synthesis MMAs in flight (bounded)
+      if (tid == 0) {
+        atomicAdd(&g_wait_timeouts, 1u);
+        if (syn_open) mbar_wait_bounded(syn_bar, syn_ph);  // synthesis MMAs in flight (bounded)
+      }
       if (tid == kIssuer) {
         for (int i = issued > S ? issued - S : 0; i < issued; ++i)
           mbar_wait_bounded(bar + (i % S), static_cast<uint32_t>((i / S) & 1));
@@ -380,7 +398,6 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2_tile_kernel(const __grid_co
     for (int s = 0; s < count + 2; ++s) {
       const int i1 = s - 1;
       const bool work = i1 >= 0 && i1 < count;
-      const bool syn = SYN && s >= 2;
       const bool ana = s < count;
       ana_open = ana;
       if (work) {
@@ -409,31 +426,9 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2_tile_kernel(const __grid_co
                                 : __ldg(table<int4>(splan, h.off_fixG) + (i - nfZ));
           }
         }
-        // dC first: column-path gathers only, no stores yet
-        if constexpr (C) {
-          float2 vk = make_float2(0.f, 0.f);
-#pragma unroll
-          for (int e0 = 0; e0 < kEreg; e0 += B) {
-            if (e0 < ch.EG) {
-              float2 ub[B], vb[B];
-#pragma unroll
-              for (int e = 0; e < B; ++e) {
-                ub[e] = U2[ch.ga[e0 + e] & 0xFFFFu];
-                const int ep = e0 + e - 1;
-                vb[e] = (ep < 0 || ch.gb[e0 + e] != ch.gb[ep]) ? V2[ch.gb[e0 + e]] : make_float2(0.f, 0.f);
-              }
-#pragma unroll
-              for (int e = 0; e < B; ++e) {
-                const int ep = e0 + e - 1;
-                if (ep < 0 || ch.gb[e0 + e] != ch.gb[ep]) vk = vb[e];
-                dc[e0 + e] = fmaf(ub[e].x, vk.x, fmaf(ub[e].y, vk.y, dc[e0 + e]));
-              }
-            }
-          }
-        }
       }
-      // RZ / RG are free once the synthesis MMAs of this step have read them
-      if (syn) {
+      // RZ / RG are free once the synthesis MMAs of unit s-2 have read them
+      if (SYN && work && i1 >= 1) {
         const bool ok = tc_wait_bounded(syn_bar, syn_ph);
         if (ok) syn_ph ^= 1u;
         failed = spmm_bar_or(failed || !ok);  // uniform before the barriers below
@@ -445,42 +440,35 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2_tile_kernel(const __grid_co
             zero_pending = false;
             tc_spmm_bar();
           }
-          float* RZ0 = rzg + args.set_oRZ;
-          float* RZ1 = RZ0 + args.rzg_tok;
-          float* RG0 = rzg + args.set_oRG;
-          float* RG1 = RG0 + args.rzg_tok;
-          if constexpr (F) {
-            float2 acc = make_float2(0.f, 0.f);
+        }
+        float* RZ0 = rzg + args.set_oRZ;
+        float* RZ1 = RZ0 + args.rzg_tok;
+        float* RG0 = rzg + args.set_oRG;
+        float* RG1 = RG0 + args.rzg_tok;
+        // column path: one gather of U[a] per entry serves dC (with V[b],
+        // reloaded where b changes) and the run sums of G
+        if constexpr (NEED_U) {
+          float2 vk = make_float2(0.f, 0.f), acc = make_float2(0.f, 0.f);
 #pragma unroll
-            for (int e0 = 0; e0 < kEreg; e0 += B) {
-              if (e0 < ch.EZ) {
-                float2 v[B];
+          for (int e0 = 0; e0 < kEreg; e0 += B) {
+            if (e0 < ch.EG) {
+              float2 ub[B], vb[B];
 #pragma unroll
-                for (int e = 0; e < B; ++e) v[e] = V2[ch.zb[e0 + e] & 0xFFFFu];
-#pragma unroll
-                for (int e = 0; e < B; ++e) {
-                  acc.x = fmaf(ch.zc[e0 + e], v[e].x, acc.x);
-                  acc.y = fmaf(ch.zc[e0 + e], v[e].y, acc.y);
-                  const uint32_t sz = ch.zb[e0 + e] >> 16;
-                  if (sz != FFB_NO_STORE) {
-                    RZ0[sz] = acc.x;
-                    RZ1[sz] = acc.y;
-                    acc = make_float2(0.f, 0.f);
-                  }
+              for (int e = 0; e < B; ++e) {
+                ub[e] = U2[ch.ga[e0 + e] & 0xFFFFu];
+                if constexpr (C) {
+                  const int ep = e0 + e - 1;
+                  vb[e] = (ep < 0 || ch.gb[e0 + e] != ch.gb[ep]) ? V2[ch.gb[e0 + e]] : make_float2(0.f, 0.f);
                 }
               }
-            }
-          }
-          if constexpr (D) {
-            float2 acc = make_float2(0.f, 0.f);
 #pragma unroll
-            for (int e0 = 0; e0 < kEreg; e0 += B) {
-              if (e0 < ch.EG) {
-                float2 ub[B];
-#pragma unroll
-                for (int e = 0; e < B; ++e) ub[e] = U2[ch.ga[e0 + e] & 0xFFFFu];
-#pragma unroll
-                for (int e = 0; e < B; ++e) {
+              for (int e = 0; e < B; ++e) {
+                if constexpr (C) {
+                  const int ep = e0 + e - 1;
+                  if (ep < 0 || ch.gb[e0 + e] != ch.gb[ep]) vk = vb[e];
+                  dc[e0 + e] = fmaf(ub[e].x, vk.x, fmaf(ub[e].y, vk.y, dc[e0 + e]));
+                }
+                if constexpr (D) {
                   acc.x = fmaf(ch.gc[e0 + e], ub[e].x, acc.x);
                   acc.y = fmaf(ch.gc[e0 + e], ub[e].y, acc.y);
                   const uint32_t sg = ch.ga[e0 + e] >> 16;
@@ -493,6 +481,31 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2_tile_kernel(const __grid_co
               }
             }
           }
+        }
+        // row path: run sums of Z
+        if constexpr (F) {
+          float2 acc = make_float2(0.f, 0.f);
+#pragma unroll
+          for (int e0 = 0; e0 < kEreg; e0 += B) {
+            if (e0 < ch.EZ) {
+              float2 v[B];
+#pragma unroll
+              for (int e = 0; e < B; ++e) v[e] = V2[ch.zb[e0 + e] & 0xFFFFu];
+#pragma unroll
+              for (int e = 0; e < B; ++e) {
+                acc.x = fmaf(ch.zc[e0 + e], v[e].x, acc.x);
+                acc.y = fmaf(ch.zc[e0 + e], v[e].y, acc.y);
+                const uint32_t sz = ch.zb[e0 + e] >> 16;
+                if (sz != FFB_NO_STORE) {
+                  RZ0[sz] = acc.x;
+                  RZ1[sz] = acc.y;
+                  acc = make_float2(0.f, 0.f);
+                }
+              }
+            }
+          }
+        }
+        if constexpr (SYN) {
           if (nfix > 0) {
             // rows (columns) split between chunks: add the overflow pieces
             tc_spmm_bar();
@@ -509,13 +522,19 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2_tile_kernel(const __grid_co
               }
             }
           }
-          fence_async_smem();  // RZ / RG are read by the tensor cores next step
+          fence_async_smem();  // RZ / RG are read by the tensor cores next
         }
+      }
+      // RZ / RG of unit s-1 complete (also on a failure: the tensor warps'
+      // wait keeps its phase count)
+      if (SYN && work) {
+        tc_spmm_bar();
+        if (st == 0) mbar_arrive(rzg_bar);
       }
       // analysis results of unit s -> V / U (float2: both tokens), once every
       // SpMM warp finished gathering from them and the MMAs completed
       if (ana && !failed) {
-        tc_spmm_bar();
+        if (!(SYN && work)) tc_spmm_bar();  // (else the barrier above): all gathers done
         const bool ok = tc_wait_bounded(ana_bar, ana_ph);
         if (ok) {
           ana_ph ^= 1u;
