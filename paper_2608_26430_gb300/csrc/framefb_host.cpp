@@ -424,47 +424,57 @@ void pack_runs(const std::vector<Entry>& ent, int32_t P, int32_t E, int32_t base
     }
   }
 
-  // bank-conflict search (groups of 32 chunks at one step)
+  // bank-conflict search.  An instruction is a group of 32 chunks at one
+  // step; its bank counts (gathers and key reloads per half-warp, stores per
+  // warp) are kept per instruction and updated cell by cell as pieces move.
   const bool has_key = !bk.key.empty();
   const int32_t W = (P + 31) / 32;
+  struct Counts {
+    uint8_t g[2][16], k[2][16], s[32];
+  };
+  std::vector<Counts> cnt(static_cast<size_t>(W) * E);
+  std::memset(cnt.data(), 0, cnt.size() * sizeof(Counts));
   auto is_end = [&](int32_t idx, int32_t e) {
     const Placed& q = pl[piece_of[idx]];
     return q.off + q.len - 1 == e;
   };
+  // add (d = 1) or remove (d = -1) what the entry at chunk p, step e puts in
+  // its instruction; the key reload counts on every lane (the kernel loads it
+  // on all lanes and keeps it where the key changes)
+  auto cell = [&](int32_t p, int32_t e, int d) {
+    const int32_t idx = grid[static_cast<size_t>(p) * E + e];
+    if (idx < 0) return;
+    Counts& c = cnt[static_cast<size_t>(p >> 5) * E + e];
+    const int h = (p >> 4) & 1;
+    c.g[h][bk.gather[idx]] = static_cast<uint8_t>(c.g[h][bk.gather[idx]] + d);
+    if (has_key) c.k[h][bk.key[idx]] = static_cast<uint8_t>(c.k[h][bk.key[idx]] + d);
+    if (is_end(idx, e)) c.s[bk.store[idx]] = static_cast<uint8_t>(c.s[bk.store[idx]] + d);
+  };
   // 16 x wavefronts + 4 x sum of squared bank counts of one instruction
-  auto group_cost = [&](int32_t w, int32_t e) {
-    uint8_t cg[2][16] = {}, ck[2][16] = {}, cs[32] = {0};
-    for (int32_t l = 0; l < 32; ++l) {
-      const int32_t p = 32 * w + l;
-      if (p >= P) break;
-      const int32_t idx = grid[static_cast<size_t>(p) * E + e];
-      if (idx < 0) continue;
-      const int32_t h = l >> 4;
-      cg[h][bk.gather[idx]]++;
-      if (has_key) {
-        const int32_t prev = e > 0 ? grid[static_cast<size_t>(p) * E + e - 1] : -1;
-        if (prev < 0 || ent[prev].key0 != ent[idx].key0) ck[h][bk.key[idx]]++;
-      }
-      if (is_end(idx, e)) cs[bk.store[idx]]++;
-    }
+  auto cost_of = [](const Counts& c) {
     int32_t wf = 0, sq = 0;
     for (int h = 0; h < 2; ++h) {
       int32_t mg = 0, mk = 0;
       for (int b = 0; b < 16; ++b) {
-        mg = std::max<int32_t>(mg, cg[h][b]);
-        mk = std::max<int32_t>(mk, ck[h][b]);
-        sq += cg[h][b] * cg[h][b] + ck[h][b] * ck[h][b];
+        mg = std::max<int32_t>(mg, c.g[h][b]);
+        mk = std::max<int32_t>(mk, c.k[h][b]);
+        sq += c.g[h][b] * c.g[h][b] + c.k[h][b] * c.k[h][b];
       }
       wf += mg + mk;
     }
     int32_t ms = 0;
     for (int b = 0; b < 32; ++b) {
-      ms = std::max<int32_t>(ms, cs[b]);
-      sq += 2 * cs[b] * cs[b];  // two stores: one per token
+      ms = std::max<int32_t>(ms, c.s[b]);
+      sq += 2 * c.s[b] * c.s[b];  // two stores: one per token
     }
     wf += 2 * ms;
     return 16 * wf + 4 * sq;
   };
+  for (int32_t p = 0; p < P; ++p)
+    for (int32_t e = 0; e < E; ++e) cell(p, e, 1);
+  std::vector<int32_t> gcost(cnt.size());
+  for (size_t g = 0; g < cnt.size(); ++g) gcost[g] = cost_of(cnt[g]);
+
   std::vector<std::vector<int32_t>> by_len(E + 1);
   std::vector<int32_t> multi;  // pieces of two or more entries
   for (size_t k = 0; k < pl.size(); ++k) {
@@ -472,55 +482,64 @@ void pack_runs(const std::vector<Entry>& ent, int32_t P, int32_t E, int32_t base
     if (pl[k].len >= 2) multi.push_back(static_cast<int32_t>(k));
   }
   SplitMix64 rng{0x6A09E667F3BCC909ull ^ static_cast<uint64_t>(nnz)};
-  const int64_t iters = std::min<int64_t>(static_cast<int64_t>(nnz) * 600, 12000000);
-  std::vector<std::pair<int32_t, int32_t>> aff;
-  auto add_group = [&](int32_t col, int32_t e) {
-    if (e < 0 || e >= E) return;
-    const std::pair<int32_t, int32_t> g{col / 32, e};
-    for (const auto& x : aff)
-      if (x == g) return;
-    aff.push_back(g);
+  const int64_t iters = std::min<int64_t>(static_cast<int64_t>(nnz) * 4000, 60000000);
+  std::vector<std::pair<int32_t, int32_t>> cells;
+  std::vector<int32_t> groups, newcost;
+  auto add_cell = [&](int32_t p, int32_t e) {
+    cells.emplace_back(p, e);
+    const int32_t g = (p >> 5) * E + e;
+    if (std::find(groups.begin(), groups.end(), g) == groups.end()) groups.push_back(g);
   };
-  auto cost_of = [&]() {
-    int32_t c = 0;
-    for (const auto& g : aff) c += group_cost(g.first, g.second);
-    return c;
+  // tries a move: `apply` performs it and, called again, undoes it
+  auto attempt = [&](double T, auto&& apply) {
+    int32_t before = 0;
+    for (const int32_t g : groups) before += gcost[g];
+    for (const auto& c : cells) cell(c.first, c.second, -1);
+    apply();
+    for (const auto& c : cells) cell(c.first, c.second, 1);
+    int32_t after = 0;
+    newcost.clear();
+    for (const int32_t g : groups) {
+      newcost.push_back(cost_of(cnt[g]));
+      after += newcost.back();
+    }
+    const int32_t d = after - before;
+    if (d > 0 && rng.uniform_01() >= std::exp(-d / (3.0 * T + 1e-9))) {
+      for (const auto& c : cells) cell(c.first, c.second, -1);
+      apply();
+      for (const auto& c : cells) cell(c.first, c.second, 1);
+      return;
+    }
+    for (size_t k = 0; k < groups.size(); ++k) gcost[groups[k]] = newcost[k];
   };
   for (int64_t it = 0; it < iters; ++it) {
     const double T = 1.0 - static_cast<double>(it) / static_cast<double>(iters);  // temperature
-    aff.clear();
+    cells.clear();
+    groups.clear();
     const bool within = !multi.empty() && (rng.next() & 3) == 0;
     if (within) {
-      // reorder two entries of one piece
+      // reorder two entries of one piece (one run: the key reloads stay)
       Placed& q = pl[multi[rng.uniform_int(multi.size())]];
       const int32_t i = static_cast<int32_t>(rng.uniform_int(q.len)), j = static_cast<int32_t>(rng.uniform_int(q.len));
       if (i == j) continue;
-      add_group(q.col, q.off + i);
-      add_group(q.col, q.off + j);
-      const int32_t before = cost_of();
-      auto apply = [&]() {
+      add_cell(q.col, q.off + i);
+      add_cell(q.col, q.off + j);
+      attempt(T, [&]() {
         std::swap(q.ents[i], q.ents[j]);
         grid[static_cast<size_t>(q.col) * E + q.off + i] = q.ents[i];
         grid[static_cast<size_t>(q.col) * E + q.off + j] = q.ents[j];
-      };
-      apply();
-      const int32_t d = cost_of() - before;
-      if (d > 0 && rng.uniform_01() >= std::exp(-d / (3.0 * T + 1e-9))) apply();
+      });
     } else {
       // swap two pieces of the same length between chunks
       int32_t a = static_cast<int32_t>(rng.uniform_int(pl.size()));
       if (rng.next() & 1) {
         // a piece holding a lane whose gather shares a bank pair in a random instruction
         const int32_t w = static_cast<int32_t>(rng.uniform_int(W)), e = static_cast<int32_t>(rng.uniform_int(E));
-        uint8_t cg[2][16] = {};
+        const Counts& c = cnt[static_cast<size_t>(w) * E + e];
         int32_t cand[32], nc = 0;
         for (int32_t l = 0; l < 32 && 32 * w + l < P; ++l) {
           const int32_t idx = grid[static_cast<size_t>(32 * w + l) * E + e];
-          if (idx >= 0) cg[l >> 4][bk.gather[idx]]++;
-        }
-        for (int32_t l = 0; l < 32 && 32 * w + l < P; ++l) {
-          const int32_t idx = grid[static_cast<size_t>(32 * w + l) * E + e];
-          if (idx >= 0 && cg[l >> 4][bk.gather[idx]] > 1) cand[nc++] = idx;
+          if (idx >= 0 && c.g[l >> 4][bk.gather[idx]] > 1) cand[nc++] = idx;
         }
         if (nc == 0) continue;
         a = piece_of[cand[rng.uniform_int(nc)]];
@@ -529,20 +548,16 @@ void pack_runs(const std::vector<Entry>& ent, int32_t P, int32_t E, int32_t base
       if (same.size() < 2) continue;
       const int32_t b = same[rng.uniform_int(same.size())];
       if (a == b || pl[a].col == pl[b].col) continue;
-      for (int32_t t = 0; t <= pl[a].len; ++t) {  // one more step: the next entry's key-change flag
-        add_group(pl[a].col, pl[a].off + t);
-        add_group(pl[b].col, pl[b].off + t);
+      for (int32_t t = 0; t < pl[a].len; ++t) {
+        add_cell(pl[a].col, pl[a].off + t);
+        add_cell(pl[b].col, pl[b].off + t);
       }
-      const int32_t before = cost_of();
-      auto apply = [&]() {
+      attempt(T, [&]() {
         std::swap(pl[a].col, pl[b].col);
         std::swap(pl[a].off, pl[b].off);
         for (const int32_t k : {a, b})
           for (int32_t t = 0; t < pl[k].len; ++t) grid[static_cast<size_t>(pl[k].col) * E + pl[k].off + t] = pl[k].ents[t];
-      };
-      apply();
-      const int32_t d = cost_of() - before;
-      if (d > 0 && rng.uniform_01() >= std::exp(-d / (3.0 * T + 1e-9))) apply();
+      });
     }
   }
 
