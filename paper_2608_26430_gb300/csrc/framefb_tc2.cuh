@@ -45,30 +45,6 @@ __device__ __forceinline__ bool spmm_bar_or(bool f) {
   return out != 0;
 }
 
-// 8 consecutive fp32 columns at each of four TMEM addresses of this lane, one wait.
-__device__ __forceinline__ void tmem_ld8x4(uint32_t t0, uint32_t t1, uint32_t t2, uint32_t t3, float (&a)[8],
-                                           float (&b)[8], float (&c)[8], float (&d)[8]) {
-  uint32_t r[32];
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%32];\n"
-      "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%8,%9,%10,%11,%12,%13,%14,%15}, [%33];\n"
-      "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%16,%17,%18,%19,%20,%21,%22,%23}, [%34];\n"
-      "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%24,%25,%26,%27,%28,%29,%30,%31}, [%35];\n"
-      "tcgen05.wait::ld.sync.aligned;\n"
-      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
-        "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
-        "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
-      : "r"(t0), "r"(t1), "r"(t2), "r"(t3));
-#pragma unroll
-  for (int i = 0; i < 8; ++i) {
-    a[i] = __uint_as_float(r[i]);
-    b[i] = __uint_as_float(r[8 + i]);
-    c[i] = __uint_as_float(r[16 + i]);
-    d[i] = __uint_as_float(r[24 + i]);
-  }
-}
-
 // Register chunk of plan column `col`: gather slots in the float2 V / U
 // layout, store targets in the canonical RZ / RG layout.
 template <int MODE>
@@ -200,8 +176,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2_tile_kernel(const __grid_co
         const float dk = d4(fv, rho, k, r);  // D4[k][r]
         const __nv_bfloat16 hi = __float2bfloat16_rn(dk);
         const __nv_bfloat16 lo = __float2bfloat16_rn(dk - __bfloat162float(hi));
-        ban[can_bf16_off(r, k) / 2] = hi;
-        ban[can_bf16_off(32 + r, k) / 2] = lo;
+        ban[can_bf16_off(16 * (r >> 3) + (r & 7), k) / 2] = hi;      // output column 16 (c / 8) + c % 8
+        ban[can_bf16_off(16 * (r >> 3) + 8 + (r & 7), k) / 2] = lo;  // output column 16 (c / 8) + 8 + c % 8
         bsy[can_f32_off(r, k)] = __uint_as_float(to_tf32(d4(fv, rho, r, k)));  // D4[r][k]
       }
       fence_async_smem();
@@ -550,17 +526,17 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2_tile_kernel(const __grid_co
           const bool two = args.m[tq.j].N - t0 >= 2;
           float2* dst = aside == 0 ? V2 : U2;
 #pragma unroll
-          for (int q8 = 0; q8 < 4; ++q8) {  // coefficients 8 q8 .. 8 q8 + 7
-            float h0[8], l0[8], h1[8], l1[8];
-            const uint32_t c0 = tmem + alane + (0 * 2 + aside) * 64 + 8 * q8;
-            const uint32_t c1 = tmem + alane + (1 * 2 + aside) * 64 + 8 * q8;
-            tmem_ld8x4(c0, c0 + 32, c1, c1 + 32, h0, l0, h1, l1);
+          for (int q8 = 0; q8 < 4; ++q8) {  // coefficients 8 q8 .. 8 q8 + 7: hi and lo in 16 columns
+            float x0[16], x1[16];
+            const uint32_t c0 = tmem + alane + (0 * 2 + aside) * 64 + 16 * q8;
+            const uint32_t c1 = tmem + alane + (1 * 2 + aside) * 64 + 16 * q8;
+            tmem_ld16x2(c0, c1, x0, x1);
             if (ar < G) {
 #pragma unroll
               for (int j = 0; j < 4; ++j) {  // chunk q = 4 q8 + j: coefficients 2q, 2q + 1
                 const int q = 4 * q8 + j;
-                const float a0 = h0[2 * j] + l0[2 * j], a1 = h0[2 * j + 1] + l0[2 * j + 1];
-                const float b0 = two ? h1[2 * j] + l1[2 * j] : 0.f, b1 = two ? h1[2 * j + 1] + l1[2 * j + 1] : 0.f;
+                const float a0 = x0[2 * j] + x0[8 + 2 * j], a1 = x0[2 * j + 1] + x0[8 + 2 * j + 1];
+                const float b0 = two ? x1[2 * j] + x1[8 + 2 * j] : 0.f, b1 = two ? x1[2 * j + 1] + x1[8 + 2 * j + 1] : 0.f;
                 *reinterpret_cast<float4*>(dst + 32 * ar + 2 * (q ^ (ar & 7))) = make_float4(a0, b0, a1, b1);
               }
             }
