@@ -16,8 +16,12 @@ Everything is written from the paper (FrameFT, arxiv 2608.26430):
 * ``adapter`` -- dense C, the update dW = alpha/sqrt(mn) P_m C P_n^T
   (Sec. 3.1, Algorithm 1 steps 5-6), Y, dX, the coefficient gradient
   P_m^T grad_W P_n (Lemma 1 proof, Appendix A) and the multi-tenant merge.
+* ``optim``   -- the AdamW step on the coefficient values and the linear
+  learning-rate schedule with warmup (Appendix "Hyperparameters used for
+  the experiments").
 
 Parity status: every function is pinned by a ``-m "not gpu"`` test against
 the printed worked example, closed forms (numpy FFT), invariants (tightness,
-isometry, adjoint identities, linearity), finite differences or brute force.
+isometry, adjoint identities, linearity), finite differences, brute force,
+or the library optimiser of PyTorch on the CPU (``optim``).
 """
