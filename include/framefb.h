@@ -293,6 +293,45 @@ framefb_status framefb_merge(const void* W0, framefb_dtype dtype, int32_t m, int
                              const framefb_plan* plan, const void* plan_dev, const float* c_vals,
                              int32_t T, float scale, void* Wout, void* stream);
 
+/* ------------------------------------------------------------------------ */
+/* Optimiser step on the coefficient values (device)                         */
+/* ------------------------------------------------------------------------ */
+
+/* AdamW hyperparameters (the paper's runs use AdamW with the stock defaults
+ * beta1 0.9, beta2 0.999, eps 1e-8, weight decay 0.01 and the adapter
+ * learning rates of its hyperparameter tables). */
+typedef struct {
+  float lr;            /* this step's learning rate, >= 0 */
+  float beta1, beta2;  /* moment decay rates, in [0, 1) */
+  float eps;           /* > 0 */
+  float weight_decay;  /* decoupled weight decay, >= 0 */
+} framefb_adamw_params;
+
+/*
+ * One AdamW step (Adam with decoupled weight decay; Appendix "Hyperparameters
+ * used for the experiments": AdamW with a linear schedule with warmup) on n
+ * fp32 coefficient values, elementwise and in place:
+ *   p <- p (1 - lr wd);  m <- b1 m + (1 - b1) g;  v <- b2 v + (1 - b2) g^2;
+ *   p <- p - lr (m / (1 - b1^step)) / (sqrt(v / (1 - b2^step)) + eps).
+ * param, m, v: device fp32 [n], read and written; grad: device fp32 [n], read
+ * (typically the dC of framefb_run, so n = matrices x nnz when the matrices'
+ * C and dC are contiguous).  m and v are zero before step 1.  Pointers 4-byte
+ * aligned (16-byte alignment of all four takes the vector path); the four
+ * arrays must not overlap.  step: 1-based count of this step (bias
+ * corrections, computed on the host in double precision).  n == 0 is a no-op.
+ * Errors: FRAMEFB_EINVAL for n < 0, step < 1, a null or misaligned pointer or
+ * hyperparameters outside the ranges above; FRAMEFB_ECUDA if the launch fails.
+ * Asynchronous on `stream`.
+ */
+framefb_status framefb_adamw(float* param, const float* grad, float* m, float* v, int64_t n,
+                             const framefb_adamw_params* hp, int64_t step, void* stream);
+
+/* Learning rate of the step with 0-based index i under the linear schedule
+ * with warmup over `total` steps, `warmup` of them warming up:
+ * lr_max i / warmup for i < warmup, else lr_max max(0, (total - i) /
+ * (total - warmup)); 0 for negative arguments.  Host only. */
+double framefb_linear_warmup_lr(int64_t i, int64_t total, int64_t warmup, double lr_max);
+
 #ifdef __cplusplus
 }
 #endif

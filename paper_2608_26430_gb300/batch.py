@@ -33,6 +33,9 @@ class AdapterBatch:
     workload's matrices to include (defaults to all); alias_inputs: share X by
     input dimension and dY by output dimension (read-only inputs of a model
     whose layers see the same shapes); y_init / dx_init: "zeros" or "random".
+    The coefficient values of all matrices are rows of one [matrices x nnz]
+    tensor ``C`` (and their gradients rows of ``dC``), so that one optimiser
+    call covers them all.
     """
 
     def __init__(self, w: wl.Workload, device, N: int | None = None, indices=None, alias_inputs: bool = False,
@@ -53,11 +56,14 @@ class AdapterBatch:
             self.plans[(m, n)] = ffb.Plan(self.frames[n], self.frames[m], row, col)
             self.plan_dev[(m, n)] = self.plans[(m, n)].to_device(device)
         shared_x, shared_dy = {}, {}
+        self.C = torch.stack([wl.c_values(w, i, device) for i in self.indices]) if self.indices else None
+        self.dC = (torch.full((len(self.indices), w.nnz), float("nan"), dtype=torch.float32, device=device)
+                   if ops & ffb.OP_GRAD_COEFF and self.indices else None)
         self.bufs = []
-        for i in self.indices:
+        for r, i in enumerate(self.indices):
             spec = w.mats[i]
             s = 1.0 if unit_scale else wl.scale_of(w, spec)
-            b = MatBuffers(spec, s, wl.c_values(w, i, device))
+            b = MatBuffers(spec, s, self.C[r])
             if ops & (ffb.OP_FORWARD | ffb.OP_GRAD_COEFF):
                 if alias_inputs:
                     if spec.n not in shared_x:
@@ -77,7 +83,7 @@ class AdapterBatch:
             if ops & ffb.OP_BACKWARD_DX:
                 b.dX = self._init((self.N, spec.n), y_init, i, 8)
             if ops & ffb.OP_GRAD_COEFF:
-                b.dC = torch.full((w.nnz,), float("nan"), dtype=torch.float32, device=device)
+                b.dC = self.dC[r]
             self.bufs.append(b)
         self.mats = [self._mat(b) for b in self.bufs]
 

@@ -714,6 +714,52 @@ extern "C" framefb_status framefb_merge(const void* W0, framefb_dtype dtype, int
   return FRAMEFB_OK;
 }
 
+extern "C" framefb_status framefb_adamw(float* param, const float* grad, float* m, float* v, int64_t n,
+                                        const framefb_adamw_params* hp, int64_t step, void* stream) {
+  if (n < 0 || step < 1 || !hp) return FRAMEFB_EINVAL;
+  const double lr = hp->lr, b1 = hp->beta1, b2 = hp->beta2, eps = hp->eps, wd = hp->weight_decay;
+  if (!(lr >= 0) || !(b1 >= 0 && b1 < 1) || !(b2 >= 0 && b2 < 1) || !(eps > 0) || !(wd >= 0) || !std::isfinite(lr) ||
+      !std::isfinite(eps) || !std::isfinite(wd))
+    return FRAMEFB_EINVAL;
+  if (n == 0) return FRAMEFB_OK;
+  const float* ptrs[4] = {param, grad, m, v};
+  bool vec = true;
+  for (const float* q : ptrs) {
+    if (!q || reinterpret_cast<uintptr_t>(q) % 4) return FRAMEFB_EINVAL;
+    vec = vec && aligned16(q);
+  }
+  ffb::AdamWK a{};
+  a.p = param;
+  a.g = grad;
+  a.m = m;
+  a.v = v;
+  a.n = n;
+  a.decay = static_cast<float>(1.0 - lr * wd);
+  a.beta1 = hp->beta1;
+  a.beta2 = hp->beta2;
+  a.step_size = static_cast<float>(lr / (1.0 - std::pow(b1, static_cast<double>(step))));
+  a.inv_sqrt_bc2 = static_cast<float>(1.0 / std::sqrt(1.0 - std::pow(b2, static_cast<double>(step))));
+  a.eps = hp->eps;
+  const int64_t work = vec ? (n + 3) / 4 : n;
+  int dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    return FRAMEFB_ECUDA;
+  const int64_t blocks = std::max<int64_t>(1, std::min<int64_t>((work + 255) / 256, static_cast<int64_t>(sms) * 8));
+  void* kargs[] = {&a};
+  void* fn = vec ? reinterpret_cast<void*>(ffb::adamw_kernel<true>) : reinterpret_cast<void*>(ffb::adamw_kernel<false>);
+  if (cudaLaunchKernel(fn, dim3(static_cast<unsigned>(blocks)), dim3(256), kargs, 0, static_cast<cudaStream_t>(stream)) !=
+      cudaSuccess)
+    return FRAMEFB_ECUDA;
+  return FRAMEFB_OK;
+}
+
+extern "C" double framefb_linear_warmup_lr(int64_t i, int64_t total, int64_t warmup, double lr_max) {
+  if (i < 0 || total < 0 || warmup < 0) return 0.0;
+  if (i < warmup) return lr_max * static_cast<double>(i) / static_cast<double>(warmup);
+  if (total <= warmup) return 0.0;
+  return lr_max * std::max(0.0, static_cast<double>(total - i) / static_cast<double>(total - warmup));
+}
+
 // ---------------------------------------------------------------------------
 // Workspace-free variant of framefb_run for callers that cannot allocate
 // device memory: the dC partial sums live in this file-scope device array.

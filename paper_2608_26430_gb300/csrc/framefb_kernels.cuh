@@ -789,4 +789,54 @@ __global__ void __launch_bounds__(256) merge_kernel(const __grid_constant__ Merg
   }
 }
 
+// ---------------------------------------------------------------------------
+// AdamW step on coefficient values (Appendix, hyperparameter tables: AdamW):
+// elementwise over n fp32 values, 16 B read + 12 B written per element; a
+// grid-stride loop over float4 chunks (VEC, all four arrays 16-byte aligned)
+// or single values.  Bias corrections arrive as step_size = lr / (1 - b1^t)
+// and inv_sqrt_bc2 = 1 / sqrt(1 - b2^t).
+// ---------------------------------------------------------------------------
+struct AdamWK {
+  float* p;
+  const float* g;
+  float* m;
+  float* v;
+  int64_t n;
+  float decay;  // 1 - lr * weight_decay
+  float beta1, beta2, step_size, inv_sqrt_bc2, eps;
+};
+
+__device__ __forceinline__ void adamw_one(float& p, float g, float& m, float& v, const AdamWK& a) {
+  p *= a.decay;
+  m = fmaf(a.beta1, m, (1.f - a.beta1) * g);
+  v = fmaf(a.beta2, v, (1.f - a.beta2) * g * g);
+  const float denom = fmaf(sqrtf(v), a.inv_sqrt_bc2, a.eps);
+  p -= a.step_size * (m / denom);
+}
+
+template <bool VEC>
+__global__ void __launch_bounds__(256) adamw_kernel(const AdamWK a) {
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  const int64_t i0 = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if constexpr (VEC) {
+    const int64_t n4 = a.n >> 2;
+    for (int64_t i = i0; i < n4; i += stride) {
+      float4 p = reinterpret_cast<const float4*>(a.p)[i];
+      const float4 g = __ldg(reinterpret_cast<const float4*>(a.g) + i);
+      float4 m = reinterpret_cast<const float4*>(a.m)[i];
+      float4 v = reinterpret_cast<const float4*>(a.v)[i];
+      adamw_one(p.x, g.x, m.x, v.x, a);
+      adamw_one(p.y, g.y, m.y, v.y, a);
+      adamw_one(p.z, g.z, m.z, v.z, a);
+      adamw_one(p.w, g.w, m.w, v.w, a);
+      reinterpret_cast<float4*>(a.p)[i] = p;
+      reinterpret_cast<float4*>(a.m)[i] = m;
+      reinterpret_cast<float4*>(a.v)[i] = v;
+    }
+    for (int64_t i = (n4 << 2) + i0; i < a.n; i += stride) adamw_one(a.p[i], __ldg(a.g + i), a.m[i], a.v[i], a);
+  } else {
+    for (int64_t i = i0; i < a.n; i += stride) adamw_one(a.p[i], __ldg(a.g + i), a.m[i], a.v[i], a);
+  }
+}
+
 }  // namespace ffb

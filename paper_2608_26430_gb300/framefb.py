@@ -27,7 +27,7 @@ EXPORTED = [
     "framefb_support_build", "framefb_plan_build", "framefb_plan_bytes", "framefb_plan_data", "framefb_plan_free",
     "framefb_workspace_size", "framefb_run", "framefb_forward", "framefb_backward_dx", "framefb_grad_coeff",
     "framefb_backward", "framefb_fused_fwd_bwd", "framefb_merge", "framefb_run_static_ws",
-    "framefb_wait_timeouts",
+    "framefb_wait_timeouts", "framefb_adamw", "framefb_linear_warmup_lr",
 ]
 STATIC_WS_BYTES = 8 << 20
 
@@ -66,6 +66,11 @@ class framefb_mat(ct.Structure):
                 ("fin", ct.POINTER(framefb_dev_frame)), ("fout", ct.POINTER(framefb_dev_frame)),
                 ("plan", ct.c_void_p), ("plan_dev", ct.c_void_p),
                 ("c_val", ct.c_void_p), ("dC", ct.c_void_p), ("scale", ct.c_float), ("pad2_", ct.c_int32)]
+
+
+class framefb_adamw_params(ct.Structure):
+    _fields_ = [("lr", ct.c_float), ("beta1", ct.c_float), ("beta2", ct.c_float), ("eps", ct.c_float),
+                ("weight_decay", ct.c_float)]
 
 
 _lib = None
@@ -113,6 +118,10 @@ def lib() -> ct.CDLL:
         L.framefb_merge.restype = i32
         L.framefb_merge.argtypes = [vp, i32, i32, i32, i64, ct.POINTER(framefb_dev_frame),
                                     ct.POINTER(framefb_dev_frame), vp, vp, vp, i32, ct.c_float, vp, vp]
+        L.framefb_adamw.restype = i32
+        L.framefb_adamw.argtypes = [vp, vp, vp, vp, i64, ct.POINTER(framefb_adamw_params), i64, vp]
+        L.framefb_linear_warmup_lr.restype = ct.c_double
+        L.framefb_linear_warmup_lr.argtypes = [i64, i64, i64, ct.c_double]
         _lib = L
     return _lib
 
@@ -326,6 +335,20 @@ def framefb_merge(W0, fin: DevFrame, fout: DevFrame, plan: Plan, plan_dev, c_val
     _check(lib().framefb_merge(_ptr(W0), _dtype_code(W0), m, n, W0.stride(0), ct.byref(fin.struct),
                                ct.byref(fout.struct), plan.handle.value, _ptr(plan_dev), _ptr(c_vals), T,
                                float(scale), _ptr(Wout), _stream(stream)), "framefb_merge")
+
+
+def framefb_adamw(param, grad, m, v, step: int, lr: float, beta1: float = 0.9, beta2: float = 0.999,
+                  eps: float = 1e-8, weight_decay: float = 0.01, n: int | None = None, stream=None) -> None:
+    """One AdamW step on fp32 device tensors (param, m, v updated in place)."""
+    if n is None:
+        n = param.numel()
+    hp = framefb_adamw_params(float(lr), float(beta1), float(beta2), float(eps), float(weight_decay))
+    _check(lib().framefb_adamw(_ptr(param), _ptr(grad), _ptr(m), _ptr(v), int(n), ct.byref(hp), int(step),
+                               _stream(stream)), "framefb_adamw")
+
+
+def framefb_linear_warmup_lr(i: int, total: int, warmup: int, lr_max: float) -> float:
+    return float(lib().framefb_linear_warmup_lr(int(i), int(total), int(warmup), float(lr_max)))
 
 
 def framefb_wait_timeouts() -> int:
