@@ -49,12 +49,19 @@ class AdapterBatch:
         self.dtype_code = ffb.FRAMEFB_F32 if w.dtype == "f32" else ffb.FRAMEFB_BF16
         self.frames = {d: ffb.Frame(d, w.k, d // w.k, parseval=True) for d in w.dims()}
         self.dev_frames = {d: f.to_device(device) for d, f in self.frames.items()}
+        # one support and plan per shape (shared across layers, Sec. 3.3), or
+        # per matrix for per-layer supports
         self.supports, self.plans, self.plan_dev = {}, {}, {}
-        for (m, n) in w.shapes():
-            row, col, _, _ = ffb.framefb_support_build(m, n, w.nnz, w.support_seed, w.support_mode, w.zipf_s, w.k)
-            self.supports[(m, n)] = (row, col)
-            self.plans[(m, n)] = ffb.Plan(self.frames[n], self.frames[m], row, col)
-            self.plan_dev[(m, n)] = self.plans[(m, n)].to_device(device)
+        self.keys = [wl.support_key(w, i) for i in self.indices]
+        for key, i in zip(self.keys, self.indices):
+            if key in self.plans:
+                continue
+            m, n = key[0], key[1]
+            row, col, _, _ = ffb.framefb_support_build(m, n, w.nnz, wl.support_seed_of(w, i), w.support_mode,
+                                                       w.zipf_s, w.k)
+            self.supports[key] = (row, col)
+            self.plans[key] = ffb.Plan(self.frames[n], self.frames[m], row, col)
+            self.plan_dev[key] = self.plans[key].to_device(device)
         shared_x, shared_dy = {}, {}
         self.C = torch.stack([wl.c_values(w, i, device) for i in self.indices]) if self.indices else None
         self.dC = (torch.full((len(self.indices), w.nnz), float("nan"), dtype=torch.float32, device=device)
@@ -85,7 +92,7 @@ class AdapterBatch:
             if ops & ffb.OP_GRAD_COEFF:
                 b.dC = self.dC[r]
             self.bufs.append(b)
-        self.mats = [self._mat(b) for b in self.bufs]
+        self.mats = [self._mat(b, key) for b, key in zip(self.bufs, self.keys)]
 
     def _init(self, shape, kind, i, salt):
         import torch
@@ -93,11 +100,10 @@ class AdapterBatch:
             return torch.zeros(shape, dtype=self.dtype, device=self.device)
         return wl.normal(shape, 10000 * salt + i, 1.0, self.dtype, self.device)
 
-    def _mat(self, b: MatBuffers):
+    def _mat(self, b: MatBuffers, key):
         spec = b.spec
-        return ffb.make_mat(self.dev_frames[spec.n], self.dev_frames[spec.m], self.plans[(spec.m, spec.n)],
-                            self.plan_dev[(spec.m, spec.n)], b.c_val, b.scale, self.N, X=b.X, dX=b.dX, dY=b.dY,
-                            Y=b.Y, dC=b.dC, ldx=spec.n, ldy=spec.m)
+        return ffb.make_mat(self.dev_frames[spec.n], self.dev_frames[spec.m], self.plans[key], self.plan_dev[key],
+                            b.c_val, b.scale, self.N, X=b.X, dX=b.dX, dY=b.dY, Y=b.Y, dC=b.dC, ldx=spec.n, ldy=spec.m)
 
     def workspace(self, ops: int):
         return ffb.workspace(self.mats, ops, self.device)

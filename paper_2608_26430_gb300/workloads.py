@@ -39,6 +39,7 @@ class Workload:
     merge_shape: tuple = ()      # (m, n) of the merged W0
     w0_std: float = 0.02
     support_seed: int = 1
+    per_layer_support: bool = False  # one support per matrix instead of one per shape
     notes: str = ""
 
     def shapes(self):
@@ -86,8 +87,30 @@ WORKLOADS = {
         notes="ViT-B/16 blocks, 64 images x 197 tokens; merge of 64 tenants over a 768x768 W0"),
 }
 
+# Support variants of the scope table's next rows, at RoBERTa shapes: supports
+# restricted to the k diagonal blocks (Sec. 3.3), and one support per layer
+# instead of one per shape.
+WORKLOADS["roberta_blockdiag"] = Workload(
+    "roberta_blockdiag", _layers(2, [("q", 768, 768), ("v", 768, 768), ("fc1", 768, 3072)]), N=4096, nnz=1000,
+    dtype="bf16", c_std=0.02, support_mode=BLOCKDIAG,
+    notes="supports uniform inside the 16 diagonal blocks of C")
+WORKLOADS["roberta_per_layer"] = Workload(
+    "roberta_per_layer", _layers(3, [("q", 768, 768), ("v", 768, 768)]), N=4096, nnz=1000, dtype="bf16",
+    c_std=0.02, per_layer_support=True, notes="a distinct uniform support for every matrix")
+
 # The configuration the headline metric is quoted on.
 HEADLINE = "llama2_7b_qkvo"
+
+
+def support_key(w: Workload, mat_index: int):
+    """Key of the support (and plan) matrix `mat_index` uses: its shape, or
+    the matrix itself with per-layer supports."""
+    spec = w.mats[mat_index]
+    return (spec.m, spec.n, mat_index) if w.per_layer_support else (spec.m, spec.n)
+
+
+def support_seed_of(w: Workload, mat_index: int) -> int:
+    return w.support_seed + (100 + mat_index if w.per_layer_support else 0)
 
 
 def scale_of(w: Workload, spec: MatSpec) -> float:

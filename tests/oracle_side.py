@@ -10,6 +10,7 @@ from functools import lru_cache
 import numpy as np
 
 from oracle import adapter, frames, support
+from paper_2608_26430_gb300 import workloads as wl
 
 
 @lru_cache(maxsize=8)
@@ -33,8 +34,9 @@ class Expect:
         w, b = batch.w, batch.bufs[j]
         spec = b.spec
         self.spec, self.scale = spec, b.scale
-        row, col, _, _ = oracle_support(spec.m, spec.n, w.nnz, w.support_seed, w.support_mode, w.zipf_s, w.k)
-        lrow, lcol = batch.supports[(spec.m, spec.n)]
+        seed = wl.support_seed_of(w, batch.indices[j])
+        row, col, _, _ = oracle_support(spec.m, spec.n, w.nnz, seed, w.support_mode, w.zipf_s, w.k)
+        lrow, lcol = batch.supports[batch.keys[j]]
         assert np.array_equal(row, lrow) and np.array_equal(col, lcol), "support differs from the oracle's"
         self.row, self.col = row, col
         self.Pin, self.Pout = frame(spec.n, w.k), frame(spec.m, w.k)

@@ -108,6 +108,17 @@ def test_bf16_kernels_every_mode(kernel, ops, monkeypatch):
     check_batch(b, ops)
 
 
+@pytest.mark.parametrize("kernel", ["tc2", "tile"])
+@pytest.mark.parametrize("wname", ["roberta_blockdiag", "roberta_per_layer"])
+def test_blockdiag_and_per_layer_supports(wname, kernel, monkeypatch):
+    # supports inside the diagonal blocks of C, and a distinct support (and
+    # plan) for every matrix of one launch
+    monkeypatch.setenv("FRAMEFB_KERNEL", kernel)
+    b = AdapterBatch(wl.WORKLOADS[wname], DEV, N=37, ops=ALL)
+    run(b, ALL)
+    check_batch(b, ALL)
+
+
 def test_llama3_zipf_nonsquare():
     # nnz = 8192 exceeds the register-resident chunk: exercises the streamed-plan path
     w = wl.WORKLOADS["llama3_8b_all"]

@@ -165,13 +165,14 @@ def test_slot_map_is_a_pair_preserving_bijection_and_bank_spread():
 
 
 PLAN_CASES = [(256, 256, 128, 0), (768, 768, 1000, 0), (768, 3072, 2000, 0), (4096, 1024, 8192, 1),
-              (1024, 256, 6000, 1), (256, 768, 4000, 0), (512, 512, 7, 0), (256, 256, 256 * 17, 0)]
+              (1024, 256, 6000, 1), (256, 768, 4000, 0), (512, 512, 7, 0), (256, 256, 256 * 17, 0),
+              (768, 768, 1000, 2), (3072, 768, 2000, 2)]
 
 
 @pytest.mark.parametrize("n,m,nnz,mode", PLAN_CASES)
 def test_plan_replays_coefficient_products(n, m, nnz, mode):
     fin, fout = ffb.Frame(n, 16, n // 16), ffb.Frame(m, 16, m // 16)
-    row, col, _, _ = support.sample_support(m, n, nnz, 1, mode, 1.1)
+    row, col, _, _ = support.sample_support(m, n, nnz, 1, mode, 1.1, 16)  # k: the diagonal blocks of mode 2
     t = decode(ffb.Plan(fin, fout, row, col).image())
     h = t["h"]
     assert h["magic"] == 0x50424646 and h["P"] == ffb.THREADS and h["nnz"] == nnz
