@@ -36,6 +36,8 @@ def parse():
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu", action="store_true")
     p.add_argument("--no-optimizer", action="store_true", help="skip the timing of the AdamW step")
+    p.add_argument("--serving", action="store_true",
+                   help="also time the mixed-tenant forward on ViT-B/16 shapes (64 images, one tenant each)")
     p.add_argument("--cpu-tokens", type=int, default=8192, help="token sample of the CPU oracle baseline")
     p.add_argument("--cpu-mats", type=int, default=4, help="matrices in the CPU oracle baseline sample")
     p.add_argument("--mats", type=int, default=None, help="first MATS matrices only (small profiling cases)")
@@ -223,6 +225,44 @@ def reference_arm(args, w, rank, world):
     print(json.dumps(out), flush=True)
 
 
+def serving_timing(dev, stream, reps: int = 10):
+    """Forward-only ViT-B/16 step (72 matrices, 64 images x 197 tokens) with
+    one tenant per image through framefb_forward_tenants, against the same
+    step with one tenant for all tokens (framefb_forward)."""
+    import torch
+    from paper_2608_26430_gb300 import framefb as ffb
+    from paper_2608_26430_gb300 import workloads as wl
+    from paper_2608_26430_gb300.batch import AdapterBatch
+    w = wl.WORKLOADS["vit_b16_merge"]
+    T, per = 64, 197
+    b = AdapterBatch(w, dev, ops=ffb.OP_FORWARD)
+    cv = [wl.normal((T, w.nnz), 900 + i, w.c_std, device=dev) for i in range(len(b.mats))]
+    mats = []
+    for mat, c in zip(b.mats, cv):
+        m2 = ffb.framefb_mat.from_buffer_copy(mat)
+        m2.c_val = c.data_ptr()
+        mats.append(m2)
+    starts, tenants = [per * i for i in range(T + 1)], list(range(T))
+
+    def timed(fn):
+        for _ in range(3):
+            fn()
+        torch.cuda.synchronize()
+        a, z = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(reps):
+            fn()
+        z.record(stream)
+        torch.cuda.synchronize()
+        return a.elapsed_time(z) / reps
+
+    ms_t = timed(lambda: ffb.framefb_forward_tenants(mats, b.dtype_code, starts, tenants, T, stream))
+    ms_1 = timed(lambda: ffb.framefb_forward(b.mats, b.dtype_code, None, stream))
+    return {"workload": "vit_b16 forward, 72 matrices, 64 images x 197 tokens", "tenants": T,
+            "ms_mixed_tenants": ms_t, "ms_one_tenant": ms_1, "tokens_per_s_mixed": w.N / (ms_t / 1e3),
+            "tokens_per_s_one_tenant": w.N / (ms_1 / 1e3)}
+
+
 def main():
     args = parse()
     rank = int(os.environ.get("RANK", "0"))
@@ -342,6 +382,8 @@ def main():
                "achieved_gbs": nb / (us * 1e-6) / 1e9, "note": "arrays L2-resident between calls; launch-bound"}
         del mo, vo
 
+    serving = serving_timing(dev, stream) if args.serving else None
+
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu:
         k = min(args.cpu_mats, len(w.mats))
@@ -368,7 +410,7 @@ def main():
                             "kernel_ms": kernel_ms,
                             "algorithmic_bytes": alg, "algorithmic_bytes_per_launch": alg / launches,
                             "launches_per_step": launches, "frac_of_8tbs": achieved / 8000.0},
-               "cpu_baseline": cpu, "e2e": e2e, "optimizer": opt,
+               "cpu_baseline": cpu, "e2e": e2e, "optimizer": opt, "serving": serving,
                "gpu_launches": launches_per_step(len(batch.bufs)) * args.steps,
                "clocks": clk.summary()}
         print(json.dumps(out), flush=True)

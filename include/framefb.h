@@ -268,6 +268,27 @@ framefb_status framefb_backward(const framefb_mat* mats, int32_t nmats, framefb_
 framefb_status framefb_fused_fwd_bwd(const framefb_mat* mats, int32_t nmats, framefb_dtype dtype,
                                      void* ws, size_t ws_bytes, void* stream);
 
+/*
+ * Mixed-tenant forward without merge (Sec. 3.4, multi-tenant serving): the
+ * tokens of one batch belong to requests of different tenants, each with its
+ * own coefficient values on the shared support:
+ *   Y[t] += X[t] dW(C_{tenant(t)})^T  for every token t and matrix.
+ * Tokens are grouped in nseg segments: segment i holds tokens
+ * [seg_start[i], seg_start[i+1]) of tenant seg_tenant[i] (host arrays;
+ * seg_start non-decreasing from 0 to N, empty segments allowed; tenants in
+ * [0, ntenants)).  Each framefb_mat describes the whole batch (N = seg_start[nseg],
+ * X and Y as for framefb_forward) and its c_val points to the tenants'
+ * values, tenant-major: [ntenants][nnz] fp32 on the device.  Every segment
+ * of every matrix is run as its own matrix of framefb_forward (rows offset
+ * into X and Y, the tenant's row of c_val), so the coefficient SpMM loads a
+ * tenant's values once per segment.  dX and dC are not touched.
+ * Errors as framefb_forward, and FRAMEFB_EINVAL for an inconsistent segment
+ * table.
+ */
+framefb_status framefb_forward_tenants(const framefb_mat* mats, int32_t nmats, framefb_dtype dtype,
+                                       const int32_t* seg_start, const int32_t* seg_tenant, int32_t nseg,
+                                       int32_t ntenants, void* stream);
+
 /* Number of waits on asynchronous row copies, since the library was loaded
  * on the current device, that gave up after their time limit (about one
  * second) instead of hanging; the CTA concerned stopped without finishing its

@@ -561,7 +561,9 @@ struct Buffers {
 // kTcMaxMats; the chunk is that short only when the kernel applies to it.
 int32_t chunk_len(const framefb_mat* mats, int32_t rest, framefb_dtype dt) {
   if (dt == FRAMEFB_BF16 && tc_allowed()) {
-    const int32_t k = std::min(rest, ffb::kTcMaxMats);
+    // launches of equal size (at most 64 matrices each): no small tail launch
+    const int32_t launches = (rest + ffb::kTcMaxMats - 1) / ffb::kTcMaxMats;
+    const int32_t k = (rest + launches - 1) / launches;
     bool ok = true;
     for (int32_t j = 0; j < k && ok; ++j) {
       const FfbPlanHeader* h = plan_header(mats[j].plan);
@@ -712,6 +714,43 @@ extern "C" framefb_status framefb_merge(const void* W0, framefb_dtype dtype, int
   if (cudaLaunchKernel(fn, dim3(h->Gm, T), dim3(256), kargs, 0, static_cast<cudaStream_t>(stream)) != cudaSuccess)
     return FRAMEFB_ECUDA;
   return FRAMEFB_OK;
+}
+
+extern "C" framefb_status framefb_forward_tenants(const framefb_mat* mats, int32_t nmats, framefb_dtype dtype,
+                                                  const int32_t* seg_start, const int32_t* seg_tenant, int32_t nseg,
+                                                  int32_t ntenants, void* stream) {
+  if (nmats < 0 || (nmats > 0 && !mats) || nseg < 0 || ntenants <= 0 || !seg_start || (nseg > 0 && !seg_tenant))
+    return FRAMEFB_EINVAL;
+  if (seg_start[0] != 0) return FRAMEFB_EINVAL;
+  for (int32_t i = 0; i < nseg; ++i)
+    if (seg_start[i + 1] < seg_start[i] || seg_tenant[i] < 0 || seg_tenant[i] >= ntenants) return FRAMEFB_EINVAL;
+  const int32_t N = seg_start[nseg];
+  std::vector<framefb_mat> seg;
+  try {
+    seg.reserve(static_cast<size_t>(nmats) * static_cast<size_t>(nseg));
+  } catch (const std::bad_alloc&) {
+    return FRAMEFB_ENOMEM;
+  }
+  const size_t esz = dtype == FRAMEFB_BF16 ? 2 : 4;
+  for (int32_t j = 0; j < nmats; ++j) {
+    const framefb_mat& M = mats[j];
+    const FfbPlanHeader* h = plan_header(M.plan);
+    if (!h || M.N != N) return FRAMEFB_EINVAL;
+    for (int32_t i = 0; i < nseg; ++i) {
+      const int32_t t0 = seg_start[i], len = seg_start[i + 1] - seg_start[i];
+      if (len == 0) continue;
+      framefb_mat S = M;
+      S.N = len;
+      S.X = M.X ? static_cast<const uint8_t*>(M.X) + static_cast<size_t>(t0) * M.ldx * esz : nullptr;
+      S.Y = M.Y ? static_cast<uint8_t*>(M.Y) + static_cast<size_t>(t0) * M.ldy * esz : nullptr;
+      S.dX = nullptr;
+      S.dY = nullptr;
+      S.dC = nullptr;
+      S.c_val = M.c_val ? M.c_val + static_cast<size_t>(seg_tenant[i]) * h->nnz : nullptr;
+      seg.push_back(S);
+    }
+  }
+  return framefb_run(seg.data(), static_cast<int32_t>(seg.size()), FRAMEFB_OP_FORWARD, dtype, nullptr, 0, stream);
 }
 
 extern "C" framefb_status framefb_adamw(float* param, const float* grad, float* m, float* v, int64_t n,

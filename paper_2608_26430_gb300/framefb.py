@@ -27,7 +27,7 @@ EXPORTED = [
     "framefb_support_build", "framefb_plan_build", "framefb_plan_bytes", "framefb_plan_data", "framefb_plan_free",
     "framefb_workspace_size", "framefb_run", "framefb_forward", "framefb_backward_dx", "framefb_grad_coeff",
     "framefb_backward", "framefb_fused_fwd_bwd", "framefb_merge", "framefb_run_static_ws",
-    "framefb_wait_timeouts", "framefb_adamw", "framefb_linear_warmup_lr",
+    "framefb_wait_timeouts", "framefb_adamw", "framefb_linear_warmup_lr", "framefb_forward_tenants",
 ]
 STATIC_WS_BYTES = 8 << 20
 
@@ -118,6 +118,8 @@ def lib() -> ct.CDLL:
         L.framefb_merge.restype = i32
         L.framefb_merge.argtypes = [vp, i32, i32, i32, i64, ct.POINTER(framefb_dev_frame),
                                     ct.POINTER(framefb_dev_frame), vp, vp, vp, i32, ct.c_float, vp, vp]
+        L.framefb_forward_tenants.restype = i32
+        L.framefb_forward_tenants.argtypes = [ct.POINTER(framefb_mat), i32, i32, vp, vp, i32, i32, vp]
         L.framefb_adamw.restype = i32
         L.framefb_adamw.argtypes = [vp, vp, vp, vp, i64, ct.POINTER(framefb_adamw_params), i64, vp]
         L.framefb_linear_warmup_lr.restype = ct.c_double
@@ -311,6 +313,20 @@ def framefb_run_static_ws(mats: Sequence[framefb_mat], ops: int, dtype: int, str
 
 def framefb_forward(mats, dtype, ws=None, stream=None):
     framefb_run(mats, OP_FORWARD, dtype, ws, stream)
+
+
+def framefb_forward_tenants(mats: Sequence[framefb_mat], dtype: int, seg_start, seg_tenant, ntenants: int,
+                            stream=None) -> None:
+    """Mixed-tenant forward: tokens [seg_start[i], seg_start[i+1]) use tenant
+    seg_tenant[i]'s coefficient values (each mat's c_val is [ntenants][nnz])."""
+    nseg = len(seg_tenant)
+    if len(seg_start) != nseg + 1:
+        raise ValueError("seg_start needs one more entry than seg_tenant")
+    starts = (ct.c_int32 * (nseg + 1))(*[int(x) for x in seg_start])
+    tenants = (ct.c_int32 * max(nseg, 1))(*[int(x) for x in seg_tenant])
+    arr = _mats_array(mats)
+    _check(lib().framefb_forward_tenants(arr, len(mats), dtype, starts, tenants, nseg, int(ntenants),
+                                         _stream(stream)), "framefb_forward_tenants")
 
 
 def framefb_backward_dx(mats, dtype, ws=None, stream=None):
