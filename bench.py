@@ -202,6 +202,16 @@ def cpu_threads():
     return os.cpu_count() or 1
 
 
+def max_over_ranks(ms: float, world: int, device) -> float:
+    """The slowest rank's time (every rank's timed region counts)."""
+    import torch
+    t = torch.tensor([float(ms)], dtype=torch.float64, device=device)
+    if world > 1:
+        import torch.distributed as dist
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
 def reference_arm(args, w, rank, world):
     if rank != 0:
         return
@@ -315,10 +325,7 @@ def main():
     barrier()
     total_ms = t_start.elapsed_time(t_end)
     kern_ms = [a.elapsed_time(b) for a, b in evs]
-    t = torch.tensor([total_ms], device=dev)
-    if world > 1:
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-    ms_step = float(t.item()) / args.steps
+    ms_step = max_over_ranks(total_ms, world, dev) / args.steps
     value = w.N * world / (ms_step / 1e3)
     kernel_ms = statistics.mean(kern_ms)
     peak, peak_kind = peaks()
@@ -353,10 +360,8 @@ def main():
             e2e_step()
         s1.record(stream)
         torch.cuda.synchronize()
-        te = torch.tensor([s0.elapsed_time(s1) / e2e_steps], device=dev)
-        if world > 1:
-            dist.all_reduce(te, op=dist.ReduceOp.MAX)
-        e2e = {"value": w.N * world / (float(te.item()) / 1e3), "unit": "tokens/s", "h2d_bytes_per_step": h2d,
+        te = max_over_ranks(s0.elapsed_time(s1) / e2e_steps, world, dev)
+        e2e = {"value": w.N * world / (te / 1e3), "unit": "tokens/s", "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": d2h, "steps": e2e_steps}
         del hx, hdy
 
