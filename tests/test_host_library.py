@@ -34,7 +34,8 @@ def test_library_exports_every_declared_function():
 
 @pytest.mark.parametrize("d,k,rho,parseval", [(256, 16, 16, True), (768, 16, 48, True), (22, 6, 6, False),
                                               (22, 6, 6, True), (40, 7, 8, True), (64, 8, 8, False),
-                                              (1024, 16, 64, True), (46, 10, 10, True)])
+                                              (1024, 16, 64, True), (46, 10, 10, True),
+                                              (64, 32, 2, True), (768, 384, 2, True)])  # rho = 2: dense DFT
 def test_frame_build_matches_oracle(d, k, rho, parseval):
     fr = ffb.Frame(d, k, rho, parseval)
     P = frames.real_frame(d, k, rho, parseval)

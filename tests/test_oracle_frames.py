@@ -68,7 +68,8 @@ def test_worked_example_real_bound():
     np.testing.assert_allclose(P @ P.T, (18.0 / 11.0) * np.eye(22), atol=1e-13)
 
 
-@pytest.mark.parametrize("d,k", [(256, 16), (64, 8), (96, 16), (48, 4), (40, 2)])
+# rho = d / k; the last three are the paper's own regime rho = 2 (one dense DFT_{d/2})
+@pytest.mark.parametrize("d,k", [(256, 16), (64, 8), (96, 16), (48, 4), (40, 2), (64, 32), (256, 128), (12, 6)])
 def test_closed_form_analysis_is_inverse_dft(d, k):
     rho = d // k
     P = frames.real_frame(d, k, rho, parseval=True)
@@ -84,7 +85,7 @@ def test_closed_form_analysis_is_inverse_dft(d, k):
             np.testing.assert_allclose(V[:, i * rho + 2 * r + 1], f[:, i].imag, atol=1e-13)
 
 
-@pytest.mark.parametrize("d,k", [(256, 16), (64, 8)])
+@pytest.mark.parametrize("d,k", [(256, 16), (64, 8), (64, 32)])
 def test_closed_form_synthesis_is_forward_dft(d, k):
     rho = d // k
     P = frames.real_frame(d, k, rho, parseval=True)
