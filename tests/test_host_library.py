@@ -262,5 +262,9 @@ def test_plan_rejects_unsorted_and_unsupported():
     with pytest.raises(ffb.FramefbError) as e:
         ffb.Plan(red, red, np.array([0], np.int32), np.array([0], np.int32))
     assert e.value.status == ffb.FRAMEFB_EUNSUPPORTED
+    dense = ffb.Frame(64, 32, 2)  # rho = 2: one dense DFT, no 32-wide groups (no device path yet)
+    with pytest.raises(ffb.FramefbError) as e:
+        ffb.Plan(dense, dense, np.array([0], np.int32), np.array([0], np.int32))
+    assert e.value.status == ffb.FRAMEFB_EUNSUPPORTED
     p = ffb.Plan(f256, f256, np.zeros(0, np.int32), np.zeros(0, np.int32))
     assert decode(p.image())["h"]["nnz"] == 0
