@@ -6,8 +6,9 @@ The shapes follow the five evaluation configurations of the adapter hot path;
 the paper's GLUE / Alpaca / ImageNet data are replaced by N(0, 1) activations
 of the same shapes (Sec. 4: RoBERTa q/v adapters, Llama q/v/k/o, ViT blocks).
 
-Seeds: support seed 1 per (m, n) shape; C values seed 2 + matrix index;
-X seed 3 (+ matrix index); dY seed 4 (+ matrix index); W0 seed 5.
+Seeds: support seed 1 per (m, n) shape (101 + matrix index with per-layer
+supports); C values seed 2 + matrix index; X seed 3 (+ matrix index); dY
+seed 4 (+ matrix index); W0 seed 5.
 """
 from __future__ import annotations
 
