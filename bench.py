@@ -7,7 +7,10 @@ pass of the whole path over one batch.
 
 Prints one JSON line (rank 0).  Under torchrun every rank runs its own
 replica of the workload (the path needs no exchange between GPUs; weak
-scaling) and the timing is the max over ranks.
+scaling) and the timing is the max over ranks.  Besides the headline, the
+line carries ``per_config``: the same fused step timed on each of the five
+evaluation workloads and the 64-tenant merge, each against its algorithmic
+bytes, with the fp64 oracle sampled beside it.
 """
 from __future__ import annotations
 
@@ -24,6 +27,11 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 METRIC = "adapter fwd+bwd tokens/sec at LLaMA-7B shape; achieved HBM GB/s vs 8 TB/s"
+NOMINAL_GBS = 8000.0
+L2_BYTES = 126 * 1024 * 1024
+
+# evaluation workloads reported in per_config, in the order of their configs
+PER_CONFIG = ("single_256_fp32", "roberta_base_qv", "llama2_7b_qkvo", "llama3_8b_all", "vit_b16_merge")
 
 
 def parse():
@@ -36,6 +44,8 @@ def parse():
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu", action="store_true")
     p.add_argument("--no-optimizer", action="store_true", help="skip the timing of the AdamW step")
+    p.add_argument("--no-per-config", action="store_true", help="skip the per-config timings")
+    p.add_argument("--configs", default=",".join(PER_CONFIG), help="comma-separated workloads for per_config")
     p.add_argument("--serving", action="store_true",
                    help="also time the mixed-tenant forward on ViT-B/16 shapes (64 images, one tenant each)")
     p.add_argument("--cpu-tokens", type=int, default=8192, help="token sample of the CPU oracle baseline")
@@ -114,8 +124,8 @@ def algorithmic_bytes(batch) -> int:
     import numpy as np
     total = 0
     esz = 2 if batch.w.dtype == "bf16" else 4
-    for b in batch.bufs:
-        img = batch.plans[(b.spec.m, b.spec.n)].image()
+    for b, key in zip(batch.bufs, batch.keys):
+        img = batch.plans[key].image()
         hdr = np.frombuffer(img[:128].tobytes(), dtype=np.int32)
         Gn, Gm, nnz = int(hdr[4]), int(hdr[5]), int(hdr[6])
         zmask = np.frombuffer(img[hdr[21]:hdr[21] + 4 * Gm].tobytes(), dtype=np.uint32)
@@ -125,22 +135,21 @@ def algorithmic_bytes(batch) -> int:
     return total
 
 
+def merge_bytes(m: int, n: int, T: int, nnz: int, esz: int) -> int:
+    """Minimum HBM bytes of a T-tenant merge: W0 read once, every W_t written,
+    the tenants' C values and the support indices read."""
+    return esz * m * n * (T + 1) + T * nnz * 4 + nnz * 8
+
+
 # sources of the dominant kernel (bf16: the two-token tcgen05 kernel unless
 # FRAMEFB_KERNEL selects another) and of the plan builder that shapes it
-KERNEL_SOURCES = ("framefb_kernels.cuh", "framefb_mma.cuh", "framefb_pipe.cuh", "framefb_tc.cuh", "framefb_tc2.cuh",
+KERNEL_SOURCES = ("framefb_kernels.cuh", "framefb_mma.cuh", "framefb_tc.cuh", "framefb_tc2.cuh",
                   "plan_layout.h", "framefb_host.cpp")
 
 
 def kernel_choice():
     k = os.environ.get("FRAMEFB_KERNEL", "tc2")
-    return k if k in ("tile", "pipe", "tc") else "tc2"
-
-
-def launches_per_step(nmats: int) -> int:
-    """Kernel launches of one fused step: a tile kernel and a dC reduction per
-    launch chunk (the tcgen05 kernels take 64 matrices per launch, the others 256)."""
-    chunk = 64 if kernel_choice() in ("tc", "tc2") else 256
-    return 2 * ((nmats + chunk - 1) // chunk)
+    return k if k in ("tile", "tc") else "tc2"
 
 
 def measured_traffic():
@@ -162,14 +171,51 @@ def measured_traffic():
         return None
 
 
-def cpu_oracle_sample(w, tokens: int, mats: int = 1):
-    """Time the oracle (fp64 numpy) on the first `mats` matrices of the workload
-    over `tokens` tokens each; returns (compute seconds, setup seconds)."""
+# ---------------------------------------------------------------------------
+# CPU side: the oracle as it stands, and what the host is
+# ---------------------------------------------------------------------------
+def cpu_threads():
+    try:
+        from threadpoolctl import threadpool_info
+        info = threadpool_info()
+        if info:
+            return max(int(i.get("num_threads", 1)) for i in info)
+    except Exception:
+        pass
+    return os.cpu_count() or 1
+
+
+def cpu_model() -> str:
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for ln in out.splitlines():
+            if ln.strip().lower().startswith("model name"):
+                return ln.split(":", 1)[1].strip()
+    except Exception:
+        pass
+    return "unknown"
+
+
+def host_info() -> dict:
+    return {"nproc": os.cpu_count(), "cpu_model": cpu_model(), "blas_threads": cpu_threads()}
+
+
+def oracle_flops(m: int, n: int, N: int) -> float:
+    """Dense fp64 flops of the oracle for one matrix over N tokens (k*rho = d
+    frames, so K_m = m and K_n = n): dW = P_m C P_n^T twice (forward and dX),
+    X dW^T, dY dW, and dY^T X followed by P_m^T (.) P_n for dC."""
+    dw = 2.0 * (m * m * n + m * n * n)
+    return 2 * dw + 2.0 * N * m * n * 3 + dw
+
+
+def cpu_oracle_sample(w, tokens: int, mats=(0,)):
+    """Time the oracle (fp64 numpy) on the given matrices of the workload over
+    `tokens` tokens each; returns (compute seconds, setup seconds)."""
     import numpy as np
     from oracle import adapter, frames, support
     from paper_2608_26430_gb300 import workloads as wl
     tcomp = tsetup = 0.0
-    for j in range(mats):
+    for j in mats:
         spec = w.mats[j]
         X = wl.x_input(w, j, tokens).float().numpy().astype(np.float64)
         dY = wl.dy_input(w, j, tokens).float().numpy().astype(np.float64)
@@ -178,8 +224,8 @@ def cpu_oracle_sample(w, tokens: int, mats: int = 1):
         t0 = time.perf_counter()
         Pin = frames.real_frame(spec.n, w.k, spec.n // w.k)
         Pout = Pin if spec.m == spec.n else frames.real_frame(spec.m, w.k, spec.m // w.k)
-        row, col, _, _ = support.sample_support(spec.m, spec.n, w.nnz, w.support_seed, w.support_mode, w.zipf_s,
-                                                w.k)
+        row, col, _, _ = support.sample_support(spec.m, spec.n, w.nnz, wl.support_seed_of(w, j), w.support_mode,
+                                                w.zipf_s, w.k)
         t1 = time.perf_counter()
         C = adapter.dense_C(spec.m, spec.n, row, col, c)
         adapter.forward(X, np.zeros((tokens, spec.m)), Pin, Pout, C, s)
@@ -191,15 +237,25 @@ def cpu_oracle_sample(w, tokens: int, mats: int = 1):
     return tcomp, tsetup
 
 
-def cpu_threads():
-    try:
-        from threadpoolctl import threadpool_info
-        info = threadpool_info()
-        if info:
-            return max(int(i.get("num_threads", 1)) for i in info)
-    except Exception:
-        pass
-    return os.cpu_count() or 1
+def oracle_step_estimate(w, tokens: int, mats=(0,)):
+    """The oracle timed on a sample (the given matrices over `tokens` tokens),
+    scaled to a full step of the workload by the dense oracle's flop count:
+    returns (tokens/s, sample seconds, sample description)."""
+    t, _ = cpu_oracle_sample(w, tokens, mats)
+    f_sample = sum(oracle_flops(w.mats[j].m, w.mats[j].n, tokens) for j in mats)
+    f_step = sum(oracle_flops(s.m, s.n, w.N) for s in w.mats)
+    step_s = t * f_step / f_sample
+    shapes = ", ".join(f"{w.mats[j].m}x{w.mats[j].n}" for j in mats)
+    desc = (f"dense fp64 oracle on {len(mats)} of {len(w.mats)} matrices ({shapes}) over {tokens} of {w.N} tokens "
+            f"({t:.2f} s), scaled to the full step by the oracle's flop count")
+    return w.N / step_s, t, desc
+
+
+def config_of(w, nmats: int, world: int) -> dict:
+    """The workload description both arms print."""
+    return {"workload": w.name, "matrices": nmats, "tokens": w.N, "nnz": w.nnz,
+            "shape": f"{w.mats[0].m}x{w.mats[0].n}", "k": w.k, "parallelism": "replicas" if world > 1 else "single",
+            "l2": "inputs larger than L2 (32 GB per step)"}
 
 
 def max_over_ranks(ms: float, world: int, device) -> float:
@@ -213,6 +269,9 @@ def max_over_ranks(ms: float, world: int, device) -> float:
 
 
 def reference_arm(args, w, rank, world):
+    """The oracle as it stands on the host cores (the paper ships no code):
+    each step is one matrix of the workload over cpu_tokens tokens, scaled to
+    the full step."""
     if rank != 0:
         return
     per = []
@@ -227,12 +286,116 @@ def reference_arm(args, w, rank, world):
     out = {"impl": "reference", "metric": METRIC, "value": tok_s, "unit": "tokens/s", "n_gpus": args.gpus,
            "steps": args.steps, "warmup": args.warmup, "ms_per_step": step * 1e3 * len(w.mats) * w.N / args.cpu_tokens,
            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-           "config": {"workload": w.name, "matrices": len(w.mats), "tokens": w.N, "nnz": w.nnz},
+           "config": config_of(w, len(w.mats), world),
            "cpu_baseline": {"value": tok_s, "unit": "tokens/s", "cores": cpu_threads(), "kind": "oracle",
                             "sample": f"dense fp64 oracle, 1 of {len(w.mats)} matrices ({w.mats[0].m}x{w.mats[0].n}), "
-                                      f"{args.cpu_tokens} of {w.N} tokens per step, scaled to the full step"},
+                                      f"{args.cpu_tokens} of {w.N} tokens per step, scaled to the full step",
+                            **host_info()},
            "e2e": {"value": tok_s, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(out), flush=True)
+
+
+# ---------------------------------------------------------------------------
+# GPU side
+# ---------------------------------------------------------------------------
+class L2Flush:
+    """Writes a buffer larger than L2 between timed iterations."""
+
+    def __init__(self, dev):
+        import torch
+        self.buf = torch.empty(2 * L2_BYTES // 4, dtype=torch.float32, device=dev)
+
+    def __call__(self):
+        self.buf.fill_(1.0)
+
+
+def time_steps(fn, stream, steps: int, warmup: int, flush=None):
+    """Mean CUDA-event time (ms) of `fn` over `steps` calls on `stream`, each
+    call timed on its own; `flush` (outside the events) runs before each."""
+    import torch
+    for _ in range(warmup):
+        if flush:
+            flush()
+        fn()
+    torch.cuda.synchronize()
+    ms = []
+    for _ in range(steps):
+        if flush:
+            flush()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        fn()
+        b.record(stream)
+        ms.append((a, b))
+    torch.cuda.synchronize()
+    return statistics.mean(a.elapsed_time(b) for a, b in ms)
+
+
+def time_config(name, dev, stream, steps, warmup, flush, with_cpu, headline=None):
+    """One fused fwd + dX + dC step over every matrix of workload `name`."""
+    import torch
+    from paper_2608_26430_gb300 import framefb as ffb
+    from paper_2608_26430_gb300 import workloads as wl
+    from paper_2608_26430_gb300.batch import AdapterBatch
+    w = wl.WORKLOADS[name]
+    ops = ffb.OP_FORWARD | ffb.OP_BACKWARD_DX | ffb.OP_GRAD_COEFF
+    peak, _ = peaks()
+    if headline is not None:
+        ms, alg, kernels = headline
+    else:
+        batch = AdapterBatch(w, dev, ops=ops)
+        ws = batch.workspace(ops)
+        alg = algorithmic_bytes(batch)
+        kernels = ffb.framefb_kernel_names(batch.mats, ops, batch.dtype_code)
+        small = alg < 2 * L2_BYTES
+        ms = time_steps(lambda: batch.run(ops, ws, stream), stream, steps, warmup, flush if small else None)
+        del batch, ws
+        torch.cuda.empty_cache()
+    gbs = alg / (ms / 1e3) / 1e9
+    rec = {"ms_per_step": ms, "tokens_per_s": w.N / (ms / 1e3), "matrices": len(w.mats), "tokens": w.N,
+           "dtype": w.dtype, "algorithmic_bytes": alg, "achieved_gbs": gbs, "frac_of_measured": gbs / peak,
+           "frac_of_8tbs": gbs / NOMINAL_GBS, "kernels": kernels + ["dc_reduce_kernel"],
+           "l2": "L2 flushed between steps" if alg < 2 * L2_BYTES else "step moves more than L2"}
+    if with_cpu:
+        shapes = []
+        for j, s in enumerate(w.mats):
+            if (s.m, s.n) not in [(w.mats[i].m, w.mats[i].n) for i in shapes]:
+                shapes.append(j)
+        # fp64 BLAS on the largest shapes takes minutes per matrix: the sample
+        # keeps the shapes up to 4096 and fewer tokens for the large workloads
+        big = max(max(w.mats[j].m, w.mats[j].n) for j in shapes)
+        tokens = min(w.N, 2048 if big <= 4096 else 512)
+        shapes = [j for j in shapes if max(w.mats[j].m, w.mats[j].n) <= 4096]
+        tok_s, t, desc = oracle_step_estimate(w, tokens, tuple(shapes))
+        rec["cpu_oracle"] = {"value": tok_s, "unit": "tokens/s", "sample_s": t, "sample": desc,
+                             "cores": cpu_threads()}
+    return rec
+
+
+def time_merge(dev, stream, steps, warmup, flush):
+    """The 64-tenant merge of the ViT-B/16 workload (768 x 768 bf16 W0)."""
+    import torch
+    from paper_2608_26430_gb300 import framefb as ffb
+    from paper_2608_26430_gb300 import workloads as wl
+    w = wl.WORKLOADS["vit_b16_merge"]
+    m, n = w.merge_shape
+    T = w.merge_tenants
+    fin, fout = ffb.Frame(n, w.k, n // w.k), ffb.Frame(m, w.k, m // w.k)
+    row, col, _, _ = ffb.framefb_support_build(m, n, w.nnz, w.support_seed, w.support_mode, w.zipf_s, w.k)
+    plan = ffb.Plan(fin, fout, row, col)
+    pd, dfin, dfout = plan.to_device(dev), fin.to_device(dev), fout.to_device(dev)
+    W0 = wl.w0_input(w, dev)
+    cv = wl.merge_c_values(w, dev)
+    Wout = torch.empty((T, m, n), device=dev, dtype=W0.dtype)
+    s = w.alpha / (m * n) ** 0.5
+    ms = time_steps(lambda: ffb.framefb_merge(W0, dfin, dfout, plan, pd, cv, T, s, Wout, stream), stream,
+                    steps, warmup, flush)
+    nb = merge_bytes(m, n, T, w.nnz, 2)
+    peak, _ = peaks()
+    gbs = nb / (ms / 1e3) / 1e9
+    return {"ms_per_call": ms, "tenants": T, "shape": f"{m}x{n}", "dtype": "bf16", "algorithmic_bytes": nb,
+            "achieved_gbs": gbs, "frac_of_measured": gbs / peak, "frac_of_8tbs": gbs / NOMINAL_GBS,
+            "kernels": ["merge_kernel<bf16>"], "l2": "L2 flushed between calls"}
 
 
 def serving_timing(dev, stream, reps: int = 10):
@@ -273,6 +436,47 @@ def serving_timing(dev, stream, reps: int = 10):
             "tokens_per_s_one_tenant": w.N / (ms_1 / 1e3)}
 
 
+def e2e_timing(batch, ops, ws, stream, steps, world, dev, barrier):
+    """The same step through the same C-ABI call with host buffers: per step
+    X, dY, Y and dX (Y and dX are read-modify-written) are copied in from
+    pinned host memory and Y, dX and dC read back."""
+    import torch
+    w = batch.w
+    hin = []
+    for b in batch.bufs:
+        for t in (b.X, b.dY, b.Y, b.dX):
+            hin.append((torch.empty(t.shape, dtype=t.dtype, pin_memory=True), t))
+    for h, t in hin:
+        h.copy_(t)
+    hout = []
+    for b in batch.bufs:
+        for t in (b.Y, b.dX, b.dC):
+            hout.append((torch.empty(t.shape, dtype=t.dtype, pin_memory=True), t))
+    h2d = sum(h.numel() * h.element_size() for h, _ in hin)
+    d2h = sum(h.numel() * h.element_size() for h, _ in hout)
+
+    def step():
+        for h, t in hin:
+            t.copy_(h, non_blocking=True)
+        batch.run(ops, ws, stream)
+        for h, t in hout:
+            h.copy_(t, non_blocking=True)
+    step()
+    torch.cuda.synchronize()
+    barrier()
+    s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    s0.record(stream)
+    for _ in range(steps):
+        step()
+    s1.record(stream)
+    torch.cuda.synchronize()
+    te = max_over_ranks(s0.elapsed_time(s1) / steps, world, dev)
+    del hin, hout
+    return {"value": w.N * world / (te / 1e3), "unit": "tokens/s", "h2d_bytes_per_step": h2d,
+            "d2h_bytes_per_step": d2h, "steps": steps,
+            "moves": "X, dY, Y, dX host to device; Y, dX, dC device to host"}
+
+
 def main():
     args = parse()
     rank = int(os.environ.get("RANK", "0"))
@@ -300,10 +504,12 @@ def main():
     from paper_2608_26430_gb300.batch import AdapterBatch
 
     ops = ffb.OP_FORWARD | ffb.OP_BACKWARD_DX | ffb.OP_GRAD_COEFF
+    timeouts0 = ffb.framefb_wait_timeouts()
     batch = AdapterBatch(w, dev, ops=ops, indices=None if args.mats is None else range(args.mats))
     ws = batch.workspace(ops)
     stream = torch.cuda.current_stream()
     alg = algorithmic_bytes(batch)
+    kernels = ffb.framefb_kernel_names(batch.mats, ops, batch.dtype_code)
 
     for _ in range(args.warmup):
         batch.run(ops, ws, stream)
@@ -330,40 +536,12 @@ def main():
     kernel_ms = statistics.mean(kern_ms)
     peak, peak_kind = peaks()
     achieved = alg / (kernel_ms / 1e3) / 1e9  # = bytes per launch / time per launch (equal launches)
-    launches = launches_per_step(len(batch.bufs)) // 2
+    chunk = 64 if kernel_choice() in ("tc", "tc2") else 256
+    launches = (len(batch.bufs) + chunk - 1) // chunk  # tile-kernel launches per step (each with a dC reduction)
 
-    # end to end through the same C-ABI call with host buffers: per step the
-    # inputs X and dY are copied from pinned host memory and dC read back
     e2e = None
     if not args.no_e2e:
-        hx = [b.X.cpu().pin_memory() for b in batch.bufs]
-        hdy = [b.dY.cpu().pin_memory() for b in batch.bufs]
-        hdc = torch.empty(len(batch.bufs), w.nnz, dtype=torch.float32).pin_memory()
-        h2d = sum(x.numel() * x.element_size() for x in hx + hdy)
-        d2h = hdc.numel() * hdc.element_size()
-        e2e_steps = max(2, min(args.steps, 5))
-
-        def e2e_step():
-            for b, x, y in zip(batch.bufs, hx, hdy):
-                b.X.copy_(x, non_blocking=True)
-                b.dY.copy_(y, non_blocking=True)
-            batch.run(ops, ws, stream)
-            for i, b in enumerate(batch.bufs):
-                hdc[i].copy_(b.dC, non_blocking=True)
-        e2e_step()
-        torch.cuda.synchronize()
-        barrier()
-        s0 = torch.cuda.Event(enable_timing=True)
-        s1 = torch.cuda.Event(enable_timing=True)
-        s0.record(stream)
-        for _ in range(e2e_steps):
-            e2e_step()
-        s1.record(stream)
-        torch.cuda.synchronize()
-        te = max_over_ranks(s0.elapsed_time(s1) / e2e_steps, world, dev)
-        e2e = {"value": w.N * world / (te / 1e3), "unit": "tokens/s", "h2d_bytes_per_step": h2d,
-               "d2h_bytes_per_step": d2h, "steps": e2e_steps}
-        del hx, hdy
+        e2e = e2e_timing(batch, ops, ws, stream, max(2, min(args.steps, 4)), world, dev, barrier)
 
     # the optimiser step on the coefficients of all matrices (one framefb_adamw
     # call over the contiguous [matrices x nnz] values), timed on its own after
@@ -387,36 +565,51 @@ def main():
                "achieved_gbs": nb / (us * 1e-6) / 1e9, "note": "arrays L2-resident between calls; launch-bound"}
         del mo, vo
 
-    serving = serving_timing(dev, stream) if args.serving else None
-
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu:
         k = min(args.cpu_mats, len(w.mats))
-        tcpu, tsetup = cpu_oracle_sample(w, args.cpu_tokens, k)
+        tcpu, tsetup = cpu_oracle_sample(w, args.cpu_tokens, tuple(range(k)))
         cpu_tok = args.cpu_tokens / (tcpu / k * len(w.mats))
         cpu = {"value": cpu_tok, "unit": "tokens/s", "cores": cpu_threads(), "kind": "oracle",
                "sample": f"dense fp64 oracle on {k} of {len(w.mats)} matrices ({w.mats[0].m}x{w.mats[0].n}) over "
                          f"{args.cpu_tokens} tokens each ({tcpu:.1f} s), scaled to {len(w.mats)} matrices; frame and "
-                         f"support setup ({tsetup:.1f} s) excluded"}
+                         f"support setup ({tsetup:.1f} s) excluded", **host_info()}
+
+    headline = (kernel_ms, alg, kernels)
+    del batch, ws
+    torch.cuda.empty_cache()
+
+    serving = serving_timing(dev, stream) if args.serving else None
+
+    per_config = None
+    if rank == 0 and not args.no_per_config and args.mats is None:
+        flush = L2Flush(dev)
+        per_config = {}
+        with_cpu = world == 1 and not args.no_cpu
+        for name in [c for c in args.configs.split(",") if c]:
+            per_config[name] = time_config(name, dev, stream, 5, 3, flush, with_cpu,
+                                           headline if name == w.name else None)
+        per_config["vit_b16_merge.merge"] = time_merge(dev, stream, 20, 3, flush)
+        del flush
+        torch.cuda.empty_cache()
+
+    timeouts = ffb.framefb_wait_timeouts() - timeouts0
 
     if rank == 0:
+        cfg = config_of(w, len(w.mats) if args.mats is None else args.mats, world)
         out = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
                "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
-               "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
-               "config": {"workload": w.name, "matrices": len(batch.bufs), "tokens": w.N, "nnz": w.nnz,
-                          "shape": f"{w.mats[0].m}x{w.mats[0].n}", "k": w.k, "parallelism": "replicas" if world > 1 else "single",
-                          "l2": "inputs larger than L2 (32 GB per step)"},
+               "vs_baseline": None, "dtype": w.dtype, "data": "synthetic", "config": cfg,
                "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                             "frac": achieved / peak,
-                            "traffic": measured_traffic() if args.mats is None and args.workload is None else None, "peak_kind": peak_kind,
-                            "kernel": {"tc2": "tc2_tile_kernel<fwd|dx|dc>", "tc": "tc_tile_kernel<fwd|dx|dc>",
-                                       "pipe": "pipe_tile_kernel<fwd|dx|dc>",
-                                       "tile": "mma_tile_kernel<fwd|dx|dc>"}[kernel_choice()] + " + dc_reduce",
+                            "traffic": measured_traffic() if args.mats is None and args.workload is None else None,
+                            "peak_kind": peak_kind,
+                            "kernel": ",".join(kernels) + " + dc_reduce_kernel",
                             "kernel_ms": kernel_ms,
                             "algorithmic_bytes": alg, "algorithmic_bytes_per_launch": alg / launches,
-                            "launches_per_step": launches, "frac_of_8tbs": achieved / 8000.0},
-               "cpu_baseline": cpu, "e2e": e2e, "optimizer": opt, "serving": serving,
-               "gpu_launches": launches_per_step(len(batch.bufs)) * args.steps,
+                            "launches_per_step": launches, "frac_of_8tbs": achieved / NOMINAL_GBS},
+               "cpu_baseline": cpu, "e2e": e2e, "optimizer": opt, "serving": serving, "per_config": per_config,
+               "gpu_launches": 2 * launches * args.steps, "wait_timeouts": timeouts,
                "clocks": clk.summary()}
         print(json.dumps(out), flush=True)
     if world > 1:

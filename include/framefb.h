@@ -241,8 +241,10 @@ framefb_status framefb_run(const framefb_mat* mats, int32_t nmats, int32_t ops, 
  * holds until the process exits; nothing is allocated per call.  A call whose
  * workspace need (framefb_workspace_size) exceeds that size returns
  * FRAMEFB_EWORKSPACE and queues nothing.  The first call on a device looks up
- * the array's device address with cudaGetSymbolAddress and caches it: make
- * that first call outside any stream capture.  All calls on one device share
+ * the array's device address with cudaGetSymbolAddress and caches it with the
+ * device's current context (a device reset or a new primary context makes
+ * the next call look it up again): make that first call outside any stream
+ * capture.  All calls on one device share
  * the array: calls whose kernels can overlap on the GPU (e.g. on unordered
  * streams) race on it and must be ordered by the caller.  Each call writes
  * every partial sum it reads, so no state carries over between calls.
@@ -251,6 +253,18 @@ framefb_status framefb_run(const framefb_mat* mats, int32_t nmats, int32_t ops, 
 #define FRAMEFB_STATIC_WS_BYTES (8u << 20)
 framefb_status framefb_run_static_ws(const framefb_mat* mats, int32_t nmats, int32_t ops, framefb_dtype dtype,
                                      void* stream);
+
+/*
+ * Names of the kernels framefb_run would launch for these arguments (no
+ * launch, no device work beyond attribute queries): the distinct tile
+ * kernels of its launch chunks, comma-separated, each with its op mask, e.g.
+ * "tc2_tile_kernel<7>"; empty when no tile kernel runs (N = 0).  buf: host,
+ * len bytes, always NUL-terminated.  The paper has no counterpart: this is a
+ * query for benchmarks and tests.  Errors as framefb_run, and FRAMEFB_EINVAL
+ * when buf is NULL or too short.
+ */
+framefb_status framefb_kernel_names(const framefb_mat* mats, int32_t nmats, int32_t ops, framefb_dtype dtype,
+                                    char* buf, size_t len);
 
 /* S3 -> S4 -> S5: Y += ((X Phi_in) C^T) Phi_out^T * s  (forward of Y = X W'^T). */
 framefb_status framefb_forward(const framefb_mat* mats, int32_t nmats, framefb_dtype dtype,

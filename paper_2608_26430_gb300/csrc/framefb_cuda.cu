@@ -8,12 +8,12 @@
 #include <cstdlib>
 #include <cstring>
 #include <mutex>
+#include <string>
 #include <vector>
 
 #include "framefb.h"
 #include "framefb_kernels.cuh"
 #include "framefb_mma.cuh"
-#include "framefb_pipe.cuh"
 #include "framefb_tc.cuh"
 #include "framefb_tc2.cuh"
 #include "plan_internal.h"
@@ -50,7 +50,6 @@ struct Prepared {
   size_t smem;
   size_t ws_bytes;
   bool reg;
-  bool pipe;  // bf16: pipelined kernel (one token per tile)
   bool tc;    // bf16: pipelined kernel on tcgen05 tensor cores
   bool tc2;   // bf16: the same, two tokens per unit
   int T;      // tile tokens of the bf16 kernel
@@ -75,17 +74,6 @@ void* tc2_kernel_ptr(int mode) {
     case 4: return reinterpret_cast<void*>(ffb::tc2_tile_kernel<4>);
     case 6: return reinterpret_cast<void*>(ffb::tc2_tile_kernel<6>);
     case 7: return reinterpret_cast<void*>(ffb::tc2_tile_kernel<7>);
-    default: return nullptr;
-  }
-}
-
-void* pipe_kernel_ptr(int mode) {
-  switch (mode) {
-    case 1: return reinterpret_cast<void*>(ffb::pipe_tile_kernel<1>);
-    case 2: return reinterpret_cast<void*>(ffb::pipe_tile_kernel<2>);
-    case 4: return reinterpret_cast<void*>(ffb::pipe_tile_kernel<4>);
-    case 6: return reinterpret_cast<void*>(ffb::pipe_tile_kernel<6>);
-    case 7: return reinterpret_cast<void*>(ffb::pipe_tile_kernel<7>);
     default: return nullptr;
   }
 }
@@ -153,51 +141,6 @@ size_t mma_smem_map(const framefb_mat* mats, int32_t nmats, int32_t ops, bool re
     a->mbar = static_cast<int32_t>(mbar);
   }
   return mbar + 16;
-}
-
-// Shared-memory map of the pipelined kernel: a ring of S staging buffers
-// (one token of X and dY each), two fp32 sets (V, U, RZ, RG of one token),
-// S mbarriers.  Returns the total bytes.
-size_t pipe_smem_map(const framefb_mat* mats, int32_t nmats, int32_t ops, int S, ffb::LaunchK* a) {
-  const bool F = ops & FRAMEFB_OP_FORWARD, D = ops & FRAMEFB_OP_BACKWARD_DX, C = ops & FRAMEFB_OP_GRAD_COEFF;
-  size_t stage = 0;
-  // one set layout for all matrices: the largest n, m and overflow counts
-  FfbPlanHeader hmax;
-  std::memset(&hmax, 0, sizeof(hmax));
-  for (int32_t j = 0; j < nmats; ++j) {
-    const FfbPlanHeader* h = plan_header(mats[j].plan);
-    const size_t rx = round_up(2 * static_cast<size_t>(h->n), 128), ry = round_up(2 * static_cast<size_t>(h->m), 128);
-    stage = std::max(stage, ((F || C) ? rx : 0) + ((D || C) ? ry : 0));
-    hmax.n = std::max(hmax.n, h->n);
-    hmax.m = std::max(hmax.m, h->m);
-    hmax.ovfZ = std::max(hmax.ovfZ, h->ovfZ);
-    hmax.ovfG = std::max(hmax.ovfG, h->ovfG);
-  }
-  const FfbTileLayout L = ffb_tile_layout(hmax, ops, 1, false);
-  const size_t set = round_up(static_cast<size_t>(L.total), 32);
-  size_t nfix = 0;  // fix-up items of the largest list
-  for (int32_t j = 0; j < nmats; ++j) {
-    const FfbPlanHeader* h = plan_header(mats[j].plan);
-    nfix = std::max<size_t>(nfix, (F ? h->nfixZ : 0) + (D ? h->nfixG : 0));
-  }
-  const size_t fbase = round_up(S * stage, 128);
-  const size_t fixc = round_up(fbase + 2 * set * 4, 16);
-  const size_t mbar = round_up(fixc + 16 * nfix, 16);
-  if (a) {
-    a->stg_in = 0;
-    a->stg_out = static_cast<int32_t>(stage);
-    a->stage_out = S;
-    a->fbase = static_cast<int32_t>(fbase);
-    a->mbar = static_cast<int32_t>(mbar);
-    a->set_oU = L.oU;
-    a->set_oRZ = L.oRZ;
-    a->set_oRG = L.oRG;
-    a->set_total = static_cast<int32_t>(set);
-    a->fixc = static_cast<int32_t>(fixc);
-    a->fixc_items = static_cast<int32_t>(nfix);
-    a->pad = kThreads - ffb::kPipeSpmm;  // first SpMM thread issues the copies
-  }
-  return mbar + 8 * static_cast<size_t>(S);
 }
 
 // Shared-memory map of the tensor-core pipelined kernel: a ring of S stages
@@ -340,14 +283,13 @@ bool encode_rows(CUtensorMap* map, const void* base, int32_t d, int32_t N, int64
 // applies (register-resident plans, group counts a multiple of 8 and at most
 // 128, its shared-memory map fits), else the one-token tensor-core kernel
 // (group counts up to 256), else the one-phase-at-a-time tile kernel.
-// FRAMEFB_KERNEL=tc2, =tc, =pipe or =tile selects one of them where it
-// applies (for comparison and tests).
+// FRAMEFB_KERNEL=tc2, =tc or =tile selects one of them where it applies
+// (for comparison and tests).
 bool kernel_is(const char* name) {
   const char* e = std::getenv("FRAMEFB_KERNEL");
   return e && std::strcmp(e, name) == 0;
 }
-bool pipe_allowed() { return kernel_is("pipe"); }
-bool tc_allowed() { return !kernel_is("tile") && !kernel_is("pipe"); }
+bool tc_allowed() { return !kernel_is("tile"); }
 bool tc2_allowed() { return tc_allowed() && !kernel_is("tc"); }
 
 // Validate one chunk of matrices and fill the launch parameters.
@@ -367,7 +309,7 @@ framefb_status prepare(const framefb_mat* mats, int32_t nmats, int32_t ops, fram
   int64_t units = 0;
   size_t smem = 0;
   int T_mma = 0;
-  bool pipe = false, tc = false, tc2 = false;
+  bool tc = false, tc2 = false;
   if (dt == FRAMEFB_BF16 && reg && tc2_allowed() && nmats <= ffb::kTcMaxMats && encode_tiled()) {
     // two-token tensor-core kernel: two stages
     int dev = 0, optin = 0;
@@ -404,24 +346,7 @@ framefb_status prepare(const framefb_mat* mats, int32_t nmats, int32_t ops, fram
       }
     }
   }
-  if (dt == FRAMEFB_BF16 && reg && !tc && !tc2 && pipe_allowed()) {
-    // pipelined kernel: deepest staging ring (2..4) that fits next to its
-    // static shared memory
-    int dev = 0, optin = 0;
-    cudaFuncAttributes fa{};
-    if (cudaGetDevice(&dev) != cudaSuccess ||
-        cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess ||
-        cudaFuncGetAttributes(&fa, pipe_kernel_ptr(ops)) != cudaSuccess)
-      return FRAMEFB_ECUDA;
-    const size_t budget = static_cast<size_t>(optin) - fa.sharedSizeBytes;
-    for (int S = 4; S >= 2 && !pipe; --S)
-      if (pipe_smem_map(mats, nmats, ops, S, nullptr) <= budget) {
-        pipe = true;
-        T_mma = 1;
-        smem = pipe_smem_map(mats, nmats, ops, S, P.args);
-      }
-  }
-  if (dt == FRAMEFB_BF16 && !pipe && !tc && !tc2) {
+  if (dt == FRAMEFB_BF16 && !tc && !tc2) {
     // one tile size for the launch; stage the output rows too when they fit,
     // else the synthesis reads them from global memory
     bool staged = false;
@@ -514,7 +439,6 @@ framefb_status prepare(const framefb_mat* mats, int32_t nmats, int32_t ops, fram
   P.red->total_units = static_cast<int32_t>(units);
   P.red->stride = P.args->stride;
   P.reg = reg;
-  P.pipe = pipe;
   P.tc = tc;
   P.tc2 = tc2;
   P.threads = (tc || tc2) ? ffb::kTcThreads : kThreads;
@@ -523,9 +447,7 @@ framefb_status prepare(const framefb_mat* mats, int32_t nmats, int32_t ops, fram
   P.grid = 0;
   P.ws_bytes = 0;
   if (units == 0) return FRAMEFB_OK;
-  void* fn = tc2 ? tc2_kernel_ptr(ops)
-             : tc ? tc_kernel_ptr(ops)
-                  : pipe ? pipe_kernel_ptr(ops) : tile_kernel_ptr(dt, ops, reg, T_mma);
+  void* fn = tc2 ? tc2_kernel_ptr(ops) : tc ? tc_kernel_ptr(ops) : tile_kernel_ptr(dt, ops, reg, T_mma);
   if (!fn) return FRAMEFB_EINVAL;
   int dev = 0, sms = 0, per_sm = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return FRAMEFB_ECUDA;
@@ -583,18 +505,25 @@ extern "C" size_t framefb_workspace_size(const framefb_mat* mats, int32_t nmats,
   if (!mats || nmats <= 0 || !ops_ok(ops)) return 0;
   Buffers b;
   size_t need = 0;
-  // the workspace depends on the launch chunking, which depends on the dtype:
-  // the larger of the two (bf16 is used for the occupancy query, the fp32
-  // kernels run with the same grid bound)
+  // the workspace depends on the launch chunking, the kernel and its grid,
+  // all of which depend on the dtype: the larger need of the two dtypes the
+  // matrices are valid for (the descriptors carry no dtype)
+  bool any = false;
   for (const framefb_dtype dt : {FRAMEFB_BF16, FRAMEFB_F32}) {
-    for (int32_t j0 = 0, nm = 0; j0 < nmats; j0 += nm) {
+    size_t need_dt = 0;
+    bool ok = true;
+    for (int32_t j0 = 0, nm = 0; j0 < nmats && ok; j0 += nm) {
       nm = chunk_len(mats + j0, nmats - j0, dt);
       Prepared P = b.prep();
-      if (prepare(mats + j0, nm, ops, FRAMEFB_BF16, P) != FRAMEFB_OK) return 0;
-      need = std::max(need, P.ws_bytes);
+      ok = prepare(mats + j0, nm, ops, dt, P) == FRAMEFB_OK;
+      need_dt = std::max(need_dt, P.ws_bytes);
+    }
+    if (ok) {
+      any = true;
+      need = std::max(need, need_dt);
     }
   }
-  return need;
+  return any ? need : 0;
 }
 
 extern "C" framefb_status framefb_run(const framefb_mat* mats, int32_t nmats, int32_t ops, framefb_dtype dtype,
@@ -632,9 +561,7 @@ extern "C" framefb_status framefb_run(const framefb_mat* mats, int32_t nmats, in
     P.args->partial = static_cast<float*>(ws);
     P.tcargs->partial = static_cast<float*>(ws);
     P.red->partial = static_cast<const float*>(ws);
-    void* fn = P.tc2  ? tc2_kernel_ptr(ops)
-               : P.tc ? tc_kernel_ptr(ops)
-                      : P.pipe ? pipe_kernel_ptr(ops) : tile_kernel_ptr(dtype, ops, P.reg, P.T);
+    void* fn = P.tc2 ? tc2_kernel_ptr(ops) : P.tc ? tc_kernel_ptr(ops) : tile_kernel_ptr(dtype, ops, P.reg, P.T);
     void* kargs[] = {(P.tc || P.tc2) ? static_cast<void*>(P.tcargs) : static_cast<void*>(P.args)};
     if (cudaLaunchKernel(fn, dim3(P.grid), dim3(P.threads), kargs, P.smem, st) != cudaSuccess)
       return FRAMEFB_ECUDA;
@@ -650,6 +577,33 @@ extern "C" framefb_status framefb_run(const framefb_mat* mats, int32_t nmats, in
       }
     }
   }
+  return FRAMEFB_OK;
+}
+
+extern "C" framefb_status framefb_kernel_names(const framefb_mat* mats, int32_t nmats, int32_t ops,
+                                               framefb_dtype dtype, char* buf, size_t len) {
+  if (!buf || len == 0) return FRAMEFB_EINVAL;
+  buf[0] = '\0';
+  if (nmats < 0 || (nmats > 0 && !mats) || !ops_ok(ops)) return FRAMEFB_EINVAL;
+  if (dtype != FRAMEFB_F32 && dtype != FRAMEFB_BF16) return FRAMEFB_EINVAL;
+  Buffers b;
+  std::vector<std::string> names;
+  for (int32_t j0 = 0, nm = 0; j0 < nmats; j0 += nm) {
+    nm = chunk_len(mats + j0, nmats - j0, dtype);
+    Prepared P = b.prep();
+    const framefb_status s = prepare(mats + j0, nm, ops, dtype, P);
+    if (s != FRAMEFB_OK) return s;
+    if (P.grid == 0) continue;
+    std::string k = P.tc2  ? "tc2_tile_kernel"
+                    : P.tc ? "tc_tile_kernel"
+                           : (dtype == FRAMEFB_BF16 ? "mma_tile_kernel" : "fft_tile_kernel");
+    k += "<" + std::to_string(ops) + ">";
+    if (std::find(names.begin(), names.end(), k) == names.end()) names.push_back(k);
+  }
+  std::string out;
+  for (const std::string& k : names) out += (out.empty() ? "" : ",") + k;
+  if (out.size() + 1 > len) return FRAMEFB_EINVAL;
+  std::memcpy(buf, out.c_str(), out.size() + 1);
   return FRAMEFB_OK;
 }
 
@@ -711,7 +665,15 @@ extern "C" framefb_status framefb_merge(const void* W0, framefb_dtype dtype, int
   void* kargs[] = {&a};
   void* fn = dtype == FRAMEFB_BF16 ? reinterpret_cast<void*>(ffb::merge_kernel<__nv_bfloat16>)
                                    : reinterpret_cast<void*>(ffb::merge_kernel<float>);
-  if (cudaLaunchKernel(fn, dim3(h->Gm, T), dim3(256), kargs, 0, static_cast<cudaStream_t>(stream)) != cudaSuccess)
+  // grid-stride over (out group, tenant) items: as many CTAs as are resident
+  int dev = 0, sms = 0, per_sm = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, ffb::kMergeThreads, 0) != cudaSuccess)
+    return FRAMEFB_ECUDA;
+  const int64_t items = static_cast<int64_t>(h->Gm) * T;
+  const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(items, static_cast<int64_t>(sms) * std::max(per_sm, 1)));
+  if (cudaLaunchKernel(fn, dim3(static_cast<unsigned>(grid)), dim3(ffb::kMergeThreads), kargs, 0,
+                       static_cast<cudaStream_t>(stream)) != cudaSuccess)
     return FRAMEFB_ECUDA;
   return FRAMEFB_OK;
 }
@@ -725,6 +687,8 @@ extern "C" framefb_status framefb_forward_tenants(const framefb_mat* mats, int32
   for (int32_t i = 0; i < nseg; ++i)
     if (seg_start[i + 1] < seg_start[i] || seg_tenant[i] < 0 || seg_tenant[i] >= ntenants) return FRAMEFB_EINVAL;
   const int32_t N = seg_start[nseg];
+  // the segments of all matrices run as the matrices of one framefb_run call
+  if (static_cast<int64_t>(nmats) * nseg > INT32_MAX) return FRAMEFB_EINVAL;
   std::vector<framefb_mat> seg;
   try {
     seg.reserve(static_cast<size_t>(nmats) * static_cast<size_t>(nseg));
@@ -810,19 +774,46 @@ static __device__ __align__(256) unsigned char g_static_ws[FRAMEFB_STATIC_WS_BYT
 namespace {
 constexpr int kMaxDevices = 64;
 std::mutex g_static_ws_mu;
-void* g_static_ws_ptr[kMaxDevices] = {};
+struct StaticWsEntry {
+  CUcontext ctx;  // context the address was looked up in
+  void* ptr;
+};
+StaticWsEntry g_static_ws_cache[kMaxDevices] = {};
 
-// Device address of g_static_ws on the current device (looked up on first use).
+using CtxGetCurrentFn = CUresult (*)(CUcontext*);
+CtxGetCurrentFn ctx_get_current() {
+  static const CtxGetCurrentFn fn = [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q{};
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess)
+      return static_cast<CtxGetCurrentFn>(nullptr);
+    return reinterpret_cast<CtxGetCurrentFn>(p);
+  }();
+  return fn;
+}
+
+// Device address of g_static_ws in the current context of the current
+// device.  It is looked up on the first call in a context and cached with
+// that context: after a device reset or a new primary context the module is
+// loaded again, the array may move, and the next call looks it up afresh.
 framefb_status static_ws_address(void** out) {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return FRAMEFB_ECUDA;
+  const CtxGetCurrentFn get = ctx_get_current();
+  CUcontext ctx = nullptr;
+  if (!get || get(&ctx) != CUDA_SUCCESS) return FRAMEFB_ECUDA;
   std::lock_guard<std::mutex> lock(g_static_ws_mu);
-  if (!g_static_ws_ptr[dev]) {
+  StaticWsEntry& e = g_static_ws_cache[dev];
+  if (!ctx || !e.ptr || e.ctx != ctx) {
+    // the lookup also makes the runtime's context current when none is yet
     void* p = nullptr;
     if (cudaGetSymbolAddress(&p, g_static_ws) != cudaSuccess || !p) return FRAMEFB_ECUDA;
-    g_static_ws_ptr[dev] = p;
+    if (get(&ctx) != CUDA_SUCCESS || !ctx) return FRAMEFB_ECUDA;
+    e.ctx = ctx;
+    e.ptr = p;
   }
-  *out = g_static_ws_ptr[dev];
+  *out = e.ptr;
   return FRAMEFB_OK;
 }
 }  // namespace

@@ -746,45 +746,120 @@ __global__ void __launch_bounds__(256) dc_reduce_kernel(const __grid_constant__ 
 }
 
 // ---------------------------------------------------------------------------
-// Merge: W_t[32g + i][32h + jl] = W0 + (s/16) sum_{e in block (g,h)} c_e
-// Dout[i][a_e] Din[jl][b_e], D = 4 x the group-0 block of each frame staged in
-// shared memory.  One CTA per (out group g, tenant t); a thread owns a column.
+// Merge (Sec. 3.4 "Storage efficiency", Alg. 1 step 6 per tenant):
+//   W_t[32g + i][32h + j] = W0[..] + (s/16) sum_{e in block (g,h)} c_{t,e} Dout[i][a_e] Din[j][b_e],
+// D = 4 x the group-0 block of each frame (k = 16, k*rho = d frames), staged
+// once per CTA.  Work items are (out group g, tenant t), taken grid-stride
+// (any number of tenants); inside an item warp w owns the 32 x 32 blocks
+// h = w, w + 8, ...  A lane owns one 16-byte chunk of one row per row pass:
+// lanes (row l / CPR, chunk l % CPR), CPR = 16-byte chunks per 32-element
+// row (4 bf16, 8 fp32), so a warp's store covers whole 64- or 128-byte row
+// segments.  The block's entries are uniform over the warp: no divergence.
+// Bound: HBM (W_t written once; W0 and the plan are L2-resident across
+// tenants).
 // ---------------------------------------------------------------------------
 template <typename Elem>
-__global__ void __launch_bounds__(256) merge_kernel(const __grid_constant__ MergeK a) {
-  __shared__ float Din[32][33];
-  __shared__ float Dout[32][33];
+struct MergeIO;
+template <>
+struct MergeIO<__nv_bfloat16> {
+  static constexpr int kPer = 8;  // elements per 16-byte chunk
+  static __device__ __forceinline__ void unpack(const uint4& q, float (&x)[8]) {
+    const uint32_t w[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      x[2 * i] = __uint_as_float(w[i] << 16);
+      x[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
+    }
+  }
+  static __device__ __forceinline__ uint4 pack(const float (&x)[8]) {
+    uint32_t w[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const __nv_bfloat162 h = __floats2bfloat162_rn(x[2 * i], x[2 * i + 1]);
+      w[i] = *reinterpret_cast<const uint32_t*>(&h);
+    }
+    return make_uint4(w[0], w[1], w[2], w[3]);
+  }
+};
+template <>
+struct MergeIO<float> {
+  static constexpr int kPer = 4;
+  static __device__ __forceinline__ void unpack(const uint4& q, float (&x)[4]) {
+    x[0] = __uint_as_float(q.x);
+    x[1] = __uint_as_float(q.y);
+    x[2] = __uint_as_float(q.z);
+    x[3] = __uint_as_float(q.w);
+  }
+  static __device__ __forceinline__ uint4 pack(const float (&x)[4]) {
+    return make_uint4(__float_as_uint(x[0]), __float_as_uint(x[1]), __float_as_uint(x[2]), __float_as_uint(x[3]));
+  }
+};
+
+constexpr int kMergeThreads = 256;
+
+template <typename Elem>
+__global__ void __launch_bounds__(kMergeThreads) merge_kernel(const __grid_constant__ MergeK a) {
+  using IO = MergeIO<Elem>;
+  constexpr int PER = IO::kPer;             // elements per lane chunk
+  constexpr int CPR = 32 / PER;             // chunks per 32-element block row
+  constexpr int RPP = 32 / CPR;             // rows per warp pass
+  constexpr int PASSES = 32 / RPP;          // passes over the block's 32 rows
+  __shared__ float DoutT[32][33];           // [a][i] = Dout[i][a]
+  __shared__ __align__(16) float DinT[32][32];  // [b][j] = Din[j][b]
   for (int idx = threadIdx.x; idx < 1024; idx += blockDim.x) {
-    const int w = idx & 31, x = idx >> 5, i = x >> 1, s = x & 1;
-    Dout[w][x] = 4.f * __ldg(a.fout_val + 32 * (i * a.rho_out + s) + w);
-    Din[w][x] = 4.f * __ldg(a.fin_val + 32 * (i * a.rho_in + s) + w);
+    const int w = idx & 31, x = idx >> 5, i = x >> 1, s = x & 1;  // column x = 2i + s of the group block, row w
+    DoutT[x][w] = 4.f * __ldg(a.fout_val + 32 * (i * a.rho_out + s) + w);
+    DinT[x][w] = 4.f * __ldg(a.fin_val + 32 * (i * a.rho_in + s) + w);
   }
   __syncthreads();
-  const int g = blockIdx.x, t = blockIdx.y;
   const FfbPlanHeader& h = hdr(a.plan);
   const int32_t* blkptr = table<int32_t>(a.plan, h.off_blkptr);
   const int2* blkent = table<int2>(a.plan, h.off_blkent);
-  const float* cv = a.c_vals + static_cast<size_t>(t) * a.nnz;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int rl = lane / CPR, cl = lane % CPR;  // row in the pass, chunk in the row
   const Elem* W0 = static_cast<const Elem*>(a.W0);
-  Elem* Wt = static_cast<Elem*>(a.Wout) + static_cast<size_t>(t) * a.m * a.ldw;
-  for (int jc = threadIdx.x; jc < a.n; jc += blockDim.x) {
-    const int hh = jc >> 5, jl = jc & 31;
-    float acc[32];
+  const int64_t items = static_cast<int64_t>(h.Gm) * a.T;
+  for (int64_t it = blockIdx.x; it < items; it += gridDim.x) {
+    const int g = static_cast<int>(it % h.Gm);
+    const int64_t t = it / h.Gm;
+    const float* cv = a.c_vals + t * a.nnz;
+    Elem* Wt = static_cast<Elem*>(a.Wout) + t * static_cast<int64_t>(a.m) * a.ldw;
+    for (int hb = warp; hb < h.Gn; hb += kMergeThreads / 32) {
+      float acc[PASSES][PER];
 #pragma unroll
-    for (int i = 0; i < 32; ++i) acc[i] = 0.f;
-    const int e0 = __ldg(blkptr + g * h.Gn + hh), e1 = __ldg(blkptr + g * h.Gn + hh + 1);
-    for (int e = e0; e < e1; ++e) {
-      const int2 en = __ldg(blkent + e);
-      const int al = en.x & 31, bl = (en.x >> 8) & 31;
-      const float w = __ldg(cv + en.y) * Din[jl][bl];
+      for (int r = 0; r < PASSES; ++r)
 #pragma unroll
-      for (int i = 0; i < 32; ++i) acc[i] = fmaf(w, Dout[i][al], acc[i]);
-    }
+        for (int j = 0; j < PER; ++j) acc[r][j] = 0.f;
+      const int e0 = __ldg(blkptr + g * h.Gn + hb), e1 = __ldg(blkptr + g * h.Gn + hb + 1);
+      for (int e = e0; e < e1; ++e) {
+        const int2 en = __ldg(blkent + e);
+        const int al = en.x & 31, bl = (en.x >> 8) & 31;
+        const float c = __ldg(cv + en.y);
+        float din[PER];
 #pragma unroll
-    for (int i = 0; i < 32; ++i) {
-      const size_t off = static_cast<size_t>(32 * g + i) * a.ldw + jc;
-      const float v = fmaf(a.seff, acc[i], static_cast<float>(W0[off]));
-      Wt[off] = static_cast<Elem>(v);
+        for (int j = 0; j < PER; j += 4) {
+          const float4 q = *reinterpret_cast<const float4*>(&DinT[bl][cl * PER + j]);
+          din[j] = q.x;
+          din[j + 1] = q.y;
+          din[j + 2] = q.z;
+          din[j + 3] = q.w;
+        }
+#pragma unroll
+        for (int r = 0; r < PASSES; ++r) {
+          const float u = c * DoutT[al][r * RPP + rl];
+#pragma unroll
+          for (int j = 0; j < PER; ++j) acc[r][j] = fmaf(u, din[j], acc[r][j]);
+        }
+      }
+#pragma unroll
+      for (int r = 0; r < PASSES; ++r) {
+        const int64_t off = static_cast<int64_t>(32 * g + r * RPP + rl) * a.ldw + 32 * hb + cl * PER;
+        float w[PER];
+        IO::unpack(__ldg(reinterpret_cast<const uint4*>(W0 + off)), w);
+#pragma unroll
+        for (int j = 0; j < PER; ++j) w[j] = fmaf(a.seff, acc[r][j], w[j]);
+        *reinterpret_cast<uint4*>(Wt + off) = IO::pack(w);
+      }
     }
   }
 }

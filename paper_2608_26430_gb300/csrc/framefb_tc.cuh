@@ -1,11 +1,11 @@
 // Pipelined bf16 tile kernel on 5th-generation tensor cores (tcgen05, TMEM).
-// Included by framefb_cuda.cu after framefb_pipe.cuh.
+// Included by framefb_cuda.cu after framefb_mma.cuh.
 //
 // The work per one-token tile is that of mma_tile_kernel (Sec. 3.1 update and
-// the Lemma 1 gradient of Appendix A); the schedule is that of
-// pipe_tile_kernel (step s: analysis of tile s and synthesis of tile s-2 on
-// the tensor side, coefficient SpMM of tile s-1, one barrier per step), with
-// these differences:
+// the Lemma 1 gradient of Appendix A), pipelined over one-token tiles: in
+// step s the tensor side runs the analysis of tile s and the synthesis of
+// tile s-2, the SpMM warps the coefficient SpMM of tile s-1, and one barrier
+// ends the step.  Compared with the warp-MMA kernel:
 //   * the group contractions are UMMA instructions, issued by four threads
 //     in parallel (one per operand side; a single issuing thread spends about
 //     150 cycles per instruction at these small shapes):
@@ -32,7 +32,7 @@
 #pragma once
 #include <cuda.h>
 
-#include "framefb_pipe.cuh"
+#include "framefb_mma.cuh"
 
 namespace ffb {
 
@@ -60,6 +60,20 @@ __host__ __device__ __forceinline__ int can_f32_off(int row, int k) {  // floats
 // slots (x >= K) as they are.
 __host__ __device__ __forceinline__ int32_t tc_slot(int32_t x, int32_t K) {
   return x >= K ? x : can_f32_off(x >> 5, x & 31);
+}
+
+// dC partial sums of one plan column (held in registers) to the CTA's
+// workspace slot of the matrix.
+__device__ __forceinline__ void dc_flush(const uint8_t* plan, float* dst, const float (&dc)[kEreg], int col) {
+  const FfbPlanHeader& h = hdr(plan);
+  const int32_t* gq = table<int32_t>(plan, h.off_gq);
+#pragma unroll
+  for (int e = 0; e < kEreg; ++e) {
+    if (e < h.EG) {
+      const int32_t q = __ldg(gq + e * kThreads + col);
+      if (q >= 0) dst[q] = dc[e];
+    }
+  }
 }
 
 // Shared-memory descriptor, no swizzle.
@@ -665,7 +679,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc_tile_kernel(const __grid_con
           if constexpr (C) {
             if (cur >= 0) {
               float* dst = args.partial + static_cast<size_t>(blockIdx.x + cur) * args.stride;
-              pipe_flush(splan, dst, dc, st);
+              dc_flush(splan, dst, dc, st);
             }
           }
           cur = tp.j;
@@ -759,7 +773,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc_tile_kernel(const __grid_con
       if constexpr (C) {
         if (cur >= 0) {
           float* dst = args.partial + static_cast<size_t>(blockIdx.x + cur) * args.stride;
-          pipe_flush(splan, dst, dc, st);
+          dc_flush(splan, dst, dc, st);
         }
       }
     }

@@ -382,7 +382,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2_tile_kernel(const __grid_co
           if constexpr (C) {
             if (cur >= 0) {
               float* dst = args.partial + static_cast<size_t>(blockIdx.x + cur) * args.stride;
-              pipe_flush(splan, dst, dc, st);
+              dc_flush(splan, dst, dc, st);
             }
           }
           cur = tp.j;
@@ -556,7 +556,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2_tile_kernel(const __grid_co
       if constexpr (C) {
         if (cur >= 0) {
           float* dst = args.partial + static_cast<size_t>(blockIdx.x + cur) * args.stride;
-          pipe_flush(splan, dst, dc, st);
+          dc_flush(splan, dst, dc, st);
         }
       }
     }

@@ -28,6 +28,7 @@ EXPORTED = [
     "framefb_workspace_size", "framefb_run", "framefb_forward", "framefb_backward_dx", "framefb_grad_coeff",
     "framefb_backward", "framefb_fused_fwd_bwd", "framefb_merge", "framefb_run_static_ws",
     "framefb_wait_timeouts", "framefb_adamw", "framefb_linear_warmup_lr", "framefb_forward_tenants",
+    "framefb_kernel_names",
 ]
 STATIC_WS_BYTES = 8 << 20
 
@@ -111,6 +112,8 @@ def lib() -> ct.CDLL:
             f = getattr(L, name)
             f.restype = i32
             f.argtypes = [ct.POINTER(framefb_mat), i32, i32, vp, sz, vp]
+        L.framefb_kernel_names.restype = i32
+        L.framefb_kernel_names.argtypes = [ct.POINTER(framefb_mat), i32, i32, i32, ct.c_char_p, sz]
         L.framefb_run_static_ws.restype = i32
         L.framefb_run_static_ws.argtypes = [ct.POINTER(framefb_mat), i32, i32, i32, vp]
         L.framefb_wait_timeouts.restype = i32
@@ -303,6 +306,15 @@ def framefb_run(mats: Sequence[framefb_mat], ops: int, dtype: int, ws=None, stre
     wsp = _ptr(ws)
     wsb = 0 if ws is None else ws.numel() * ws.element_size()
     _check(lib().framefb_run(arr, len(mats), ops, dtype, wsp, wsb, _stream(stream)), "framefb_run")
+
+
+def framefb_kernel_names(mats: Sequence[framefb_mat], ops: int, dtype: int) -> list:
+    """Tile kernels framefb_run would launch for these matrices (no launch)."""
+    buf = ct.create_string_buffer(1024)
+    _check(lib().framefb_kernel_names(_mats_array(mats), len(mats), ops, dtype, buf, len(buf)),
+           "framefb_kernel_names")
+    v = buf.value.decode()
+    return v.split(",") if v else []
 
 
 def framefb_run_static_ws(mats: Sequence[framefb_mat], ops: int, dtype: int, stream=None) -> None:

@@ -95,6 +95,10 @@ WORKLOADS["roberta_blockdiag"] = Workload(
     "roberta_blockdiag", _layers(2, [("q", 768, 768), ("v", 768, 768), ("fc1", 768, 3072)]), N=4096, nnz=1000,
     dtype="bf16", c_std=0.02, support_mode=BLOCKDIAG,
     notes="supports uniform inside the 16 diagonal blocks of C")
+WORKLOADS["roberta_zipf"] = Workload(
+    "roberta_zipf", _layers(2, [("q", 768, 768), ("v", 768, 768)]), N=4096, nnz=1000, dtype="bf16", c_std=0.02,
+    support_mode=ZIPF_ROWS, zipf_s=1.1,
+    notes="heavy-tailed Zipf(1.1) rows at RoBERTa shapes: long runs split over chunks (overflow and fix-up)")
 WORKLOADS["roberta_per_layer"] = Workload(
     "roberta_per_layer", _layers(3, [("q", 768, 768), ("v", 768, 768)]), N=4096, nnz=1000, dtype="bf16",
     c_std=0.02, per_layer_support=True, notes="a distinct uniform support for every matrix")

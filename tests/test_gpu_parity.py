@@ -68,7 +68,7 @@ def test_single_256_fp32(ops, unit):
     check_batch(b, ops)
 
 
-@pytest.mark.parametrize("kernel", ["tile", "pipe", "tc", "tc2"])
+@pytest.mark.parametrize("kernel", ["tile", "tc", "tc2"])
 @pytest.mark.parametrize("N", [37, 1, 4])
 def test_roberta_base_all_matrices(N, kernel, monkeypatch):
     monkeypatch.setenv("FRAMEFB_KERNEL", kernel)
@@ -77,7 +77,7 @@ def test_roberta_base_all_matrices(N, kernel, monkeypatch):
     check_batch(b, ALL)
 
 
-@pytest.mark.parametrize("kernel", ["tile", "pipe", "tc", "tc2"])
+@pytest.mark.parametrize("kernel", ["tile", "tc", "tc2"])
 def test_vit_b16_mixed_shapes(kernel, monkeypatch):
     # many matrices of three shapes per launch: CTAs cross matrix boundaries
     monkeypatch.setenv("FRAMEFB_KERNEL", kernel)
@@ -94,13 +94,12 @@ def test_llama2_shape_small_n():
     check_batch(b, ALL)
 
 
-@pytest.mark.parametrize("kernel", ["tc2", "tc", "pipe", "tile"])
+@pytest.mark.parametrize("kernel", ["tc2", "tc", "tile"])
 @pytest.mark.parametrize("ops", [ffb.OP_FORWARD, ffb.OP_BACKWARD_DX, ffb.OP_GRAD_COEFF,
                                  ffb.OP_BACKWARD_DX | ffb.OP_GRAD_COEFF, ALL])
 def test_bf16_kernels_every_mode(kernel, ops, monkeypatch):
-    # FRAMEFB_KERNEL selects the bf16 kernel: the one-phase-at-a-time tile
-    # kernel (two tokens per tile here, the default), the warp-MMA pipelined
-    # kernel or the tcgen05 pipelined kernel
+    # FRAMEFB_KERNEL selects the bf16 kernel: the one-phase-at-a-time
+    # warp-MMA tile kernel, the one-token or the two-token tcgen05 kernel
     monkeypatch.setenv("FRAMEFB_KERNEL", kernel)
     w = wl.WORKLOADS["llama2_7b_qkvo"]
     b = AdapterBatch(w, DEV, N=13, indices=[0, 5], ops=ops)
@@ -247,7 +246,11 @@ def test_invalid_arguments_return_status():
 # merge
 # ---------------------------------------------------------------------------
 def _merge_case(wname, T=None):
-    w = wl.WORKLOADS[wname]
+    if wname == "single_256_fp32_many":          # 300 tenants x 8 out groups = 2400 work items
+        import dataclasses
+        w = dataclasses.replace(wl.WORKLOADS["single_256_fp32"], merge_tenants=300)
+    else:
+        w = wl.WORKLOADS[wname]
     m, n = w.merge_shape
     T = w.merge_tenants if T is None else T
     fin, fout = ffb.Frame(n, w.k, n // w.k), ffb.Frame(m, w.k, m // w.k)
@@ -302,3 +305,54 @@ def test_llama2_full_size_bench_launch_sampled():
         assert_bf16(host64(buf.dC), e.dc(X, dY), what=f"dC[{j}]")
     del b
     torch.cuda.empty_cache()
+
+
+# ---------------------------------------------------------------------------
+# heavy-tailed supports on the default kernel, fp32 at size, many tenants
+# ---------------------------------------------------------------------------
+def _plan_header(plan):
+    return np.frombuffer(plan.image()[:128].tobytes(), dtype=np.int32)
+
+
+@pytest.mark.parametrize("nnz,N", [(1000, 37), (1000, 4096), (4096, 37)])
+def test_zipf_rows_768_default_tcgen05_kernel(nnz, N):
+    """Zipf(1.1) rows of C at 768 x 768: long runs of one row are split over
+    chunks, so the row path writes overflow slots that the fix-up adds in
+    (ovfZ 152 / 35 fix-ups at 1000 entries; the 4096-entry case fills every
+    register chunk).  Runs on the default two-token tcgen05 kernel."""
+    import dataclasses
+    w = dataclasses.replace(wl.WORKLOADS["roberta_zipf"], nnz=nnz)
+    b = AdapterBatch(w, DEV, N=N, ops=ALL)
+    h = _plan_header(b.plans[(768, 768)])
+    assert h[10] > 0 and h[12] > 0           # ovfZ, nfixZ: the fix-up path is exercised
+    assert ffb.framefb_kernel_names(b.mats, ALL, b.dtype_code) == ["tc2_tile_kernel<7>"]
+    run(b, ALL)
+    check_batch(b, ALL)
+
+
+def test_fp32_large_n_with_sized_workspace():
+    """fp32 activations at 4096 x 4096 and 8192 tokens with exactly the
+    workspace framefb_workspace_size reports (the fp32 kernel's own grid)."""
+    w = wl.Workload("fp32_4096", (wl.MatSpec("w", 4096, 4096),), N=8192, nnz=4096, dtype="f32", c_std=0.01)
+    b = AdapterBatch(w, DEV, ops=ALL)
+    need = ffb.framefb_workspace_size(b.mats, ALL)
+    assert need > 0
+    ws = torch.empty(need, dtype=torch.uint8, device=DEV)
+    assert ffb.framefb_kernel_names(b.mats, ALL, b.dtype_code) == ["fft_tile_kernel<7>"]
+    ffb.framefb_run(b.mats, ALL, b.dtype_code, ws)
+    torch.cuda.synchronize()
+    rows = np.unique(np.concatenate([[0, w.N - 1], np.random.default_rng(3).choice(w.N, 62, replace=False)]))
+    buf, e = b.bufs[0], Expect(b, 0)
+    X, dY = host64(buf.X), host64(buf.dY)
+    sel = torch.from_numpy(rows).to(DEV)
+    assert_f32(host64(buf.Y[sel]), e.y(X[rows], np.zeros((rows.size, 4096))), what="Y rows")
+    assert_f32(host64(buf.dX[sel]), e.dx(dY[rows], np.zeros((rows.size, 4096))), what="dX rows")
+    assert_f32(host64(buf.dC), e.dc(X, dY), what="dC")
+
+
+def test_merge_many_tenants_grid_stride():
+    """More (out group, tenant) items than resident CTAs: every item is taken
+    by the grid-stride loop exactly once."""
+    W0, got, ref = _merge_case("single_256_fp32_many")
+    for t in (0, 1, 77, got.shape[0] - 1):
+        assert_f32(got[t] - W0, ref[t] - W0, what=f"dW[{t}]")

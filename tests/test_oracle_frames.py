@@ -122,3 +122,38 @@ def test_dft_frame_groups_are_disjoint_blocks():
     assert pat.sum() == d * 2 * k                 # structural zeros are stored
     P = frames.real_frame(d, k, rho)
     assert np.count_nonzero(P) < pat.sum()        # some stored values are exact zeros
+
+
+def test_group_table_matches_printed_worked_example():
+    # the printed F of the (6,3,11) walk-through has row supports columns 0-4,
+    # 3-8 and 7-10 (T blocks straddle rows); a group covers the real
+    # coordinates 2j, 2j+1 of its row's complex columns j
+    F = load_real_matrix("st_F_3_11.txt")
+    printed = [(int(np.nonzero(F[r])[0][0]), int(np.nonzero(F[r])[0][-1])) for r in range(3)]
+    assert printed == [(0, 4), (3, 8), (7, 10)]
+    row0, nrows = frames.group_table(22, 6, 6)
+    assert row0.tolist() == [0, 6, 14]
+    assert nrows.tolist() == [10, 12, 8]
+
+
+@pytest.mark.parametrize("d,k,rho", [(22, 6, 6), (40, 7, 8), (46, 10, 10), (24, 4, 6), (256, 16, 16)])
+def test_group_table_is_the_row_span_of_each_groups_columns(d, k, rho):
+    # the columns {i*rho + 2r + s} of group r live exactly on the coordinates
+    # [row0[r], row0[r] + nrows[r]): nothing outside, and both boundary
+    # coordinate pairs used -- checked on the dense frame, so that an
+    # off-by-one in the range (e.g. a T block's spill row) fails
+    row0, nrows = frames.group_table(d, k, rho)
+    P = frames.real_frame(d, k, rho, parseval=False)
+    assert row0.size == nrows.size == rho // 2
+    for r in range(rho // 2):
+        cols = [i * rho + 2 * r + s for i in range(k) for s in (0, 1)]
+        used = np.nonzero(np.any(P[:, cols] != 0, axis=1))[0]
+        lo, hi = int(row0[r]), int(row0[r] + nrows[r])
+        assert used.min() >= lo and used.max() < hi
+        assert {used.min() // 2, used.max() // 2} == {lo // 2, hi // 2 - 1}
+    # T-block frames: consecutive groups overlap by exactly the shared complex column pair
+    sup = frames.row_supports(frames.spectral_tetris(rho // 2, d // 2))
+    for r in range(rho // 2 - 1):
+        overlap = max(0, sup[r][1] - sup[r + 1][0] + 1)
+        assert overlap in (0, 2)
+        assert (row0[r] + nrows[r] - row0[r + 1]) == 2 * overlap

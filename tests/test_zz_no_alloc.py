@@ -40,8 +40,11 @@ def test_static_workspace_matches_caller_workspace_twice():
         ffb.framefb_run(ref.mats, ALL, ref.dtype_code, ws)
         ffb.framefb_run_static_ws(got.mats, ALL, got.dtype_code)
         torch.cuda.synchronize()
+        # the same kernels on the same inputs: bit-equal results, and both
+        # within the bf16 bar of each other
         for a, b in zip(ref.bufs, got.bufs):
             for x, y, nm in ((a.Y, b.Y, "Y"), (a.dX, b.dX, "dX"), (a.dC, b.dC, "dC")):
+                assert torch.equal(x, y), f"call {call} {nm}: static and caller workspace differ"
                 assert_bf16(host64(y), host64(x), what=f"call {call} {nm}")
 
 
