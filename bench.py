@@ -30,8 +30,10 @@ METRIC = "adapter fwd+bwd tokens/sec at LLaMA-7B shape; achieved HBM GB/s vs 8 T
 NOMINAL_GBS = 8000.0
 L2_BYTES = 126 * 1024 * 1024
 
-# evaluation workloads reported in per_config, in the order of their configs
-PER_CONFIG = ("single_256_fp32", "roberta_base_qv", "llama2_7b_qkvo", "llama3_8b_all", "vit_b16_merge")
+# evaluation workloads reported in per_config, in the order of their configs,
+# then the paper's own rho = 2 regime at the LLaMA-2 shape (the dense path)
+PER_CONFIG = ("single_256_fp32", "roberta_base_qv", "llama2_7b_qkvo", "llama3_8b_all", "vit_b16_merge",
+              "llama2_rho2")
 
 
 def parse():
@@ -51,6 +53,7 @@ def parse():
     p.add_argument("--cpu-tokens", type=int, default=8192, help="token sample of the CPU oracle baseline")
     p.add_argument("--cpu-mats", type=int, default=4, help="matrices in the CPU oracle baseline sample")
     p.add_argument("--mats", type=int, default=None, help="first MATS matrices only (small profiling cases)")
+    p.add_argument("--tokens", type=int, default=None, help="tokens per matrix (small profiling cases)")
     return p.parse_args()
 
 
@@ -61,6 +64,26 @@ def peaks():
         return float(d["hbm_gbs"]), "measured"
     except Exception:
         return 6800.0, "fallback"
+
+
+def tensor_peak():
+    """Sustained bf16 tensor peak (TFLOP/s) for kernels timed inside a long step."""
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)["bf16_tflops_sustained"]), "measured"
+    except Exception:
+        return 1700.0, "fallback"
+
+
+def dense_flops(batch) -> float:
+    """Algorithmic flops of one fused step on the dense path: the four dense
+    contractions X Phi_in, dY Phi_out, Z Phi_out^T and G Phi_in^T, each
+    2 N d K (K = k*rho frame columns); the SpMM's 6 N nnz is added."""
+    total = 0.0
+    for b in batch.bufs:
+        fin, fout = batch.frames[b.spec.n], batch.frames[b.spec.m]
+        total += 4.0 * batch.N * (b.spec.n * fin.ncols + b.spec.m * fout.ncols) + 6.0 * batch.N * batch.w.nnz
+    return total
 
 
 class ClockSampler:
@@ -131,6 +154,8 @@ def algorithmic_bytes(batch) -> int:
         zmask = np.frombuffer(img[hdr[21]:hdr[21] + 4 * Gm].tobytes(), dtype=np.uint32)
         gmask = np.frombuffer(img[hdr[22]:hdr[22] + 4 * Gn].tobytes(), dtype=np.uint32)
         r_out, r_in = 32 * int(np.count_nonzero(zmask)), 32 * int(np.count_nonzero(gmask))
+        if int(hdr[26]) == 1:  # dense path: Phi touches every coordinate
+            r_out, r_in = b.spec.m, b.spec.n
         total += 3 * esz * batch.N * (r_in + r_out) + nnz * (4 + 4 + 8)
     return total
 
@@ -143,7 +168,7 @@ def merge_bytes(m: int, n: int, T: int, nnz: int, esz: int) -> int:
 
 # sources of the dominant kernel (bf16: the two-token tcgen05 kernel unless
 # FRAMEFB_KERNEL selects another) and of the plan builder that shapes it
-KERNEL_SOURCES = ("framefb_kernels.cuh", "framefb_mma.cuh", "framefb_tc.cuh", "framefb_tc2.cuh",
+KERNEL_SOURCES = ("framefb_kernels.cuh", "framefb_mma.cuh", "framefb_ptx.cuh", "framefb_tc.cuh", "framefb_tc2.cuh",
                   "plan_layout.h", "framefb_host.cpp")
 
 
@@ -340,12 +365,15 @@ def time_config(name, dev, stream, steps, warmup, flush, with_cpu, headline=None
     w = wl.WORKLOADS[name]
     ops = ffb.OP_FORWARD | ffb.OP_BACKWARD_DX | ffb.OP_GRAD_COEFF
     peak, _ = peaks()
+    flops = None
     if headline is not None:
         ms, alg, kernels = headline
     else:
         batch = AdapterBatch(w, dev, ops=ops)
         ws = batch.workspace(ops)
         alg = algorithmic_bytes(batch)
+        if not all(f.structured for f in batch.frames.values()):
+            flops = dense_flops(batch)
         kernels = ffb.framefb_kernel_names(batch.mats, ops, batch.dtype_code)
         small = alg < 2 * L2_BYTES
         ms = time_steps(lambda: batch.run(ops, ws, stream), stream, steps, warmup, flush if small else None)
@@ -354,8 +382,18 @@ def time_config(name, dev, stream, steps, warmup, flush, with_cpu, headline=None
     gbs = alg / (ms / 1e3) / 1e9
     rec = {"ms_per_step": ms, "tokens_per_s": w.N / (ms / 1e3), "matrices": len(w.mats), "tokens": w.N,
            "dtype": w.dtype, "algorithmic_bytes": alg, "achieved_gbs": gbs, "frac_of_measured": gbs / peak,
-           "frac_of_8tbs": gbs / NOMINAL_GBS, "kernels": kernels + ["dc_reduce_kernel"],
+           "frac_of_8tbs": gbs / NOMINAL_GBS,
+           "kernels": kernels + ([] if any(k.startswith("dense") for k in kernels) else ["dc_reduce_kernel"]),
            "l2": "L2 flushed between steps" if alg < 2 * L2_BYTES else "step moves more than L2"}
+    if flops:
+        tpk, kind = tensor_peak()
+        tf = flops / (ms / 1e3) / 1e12
+        # each algorithmic flop costs two bf16 tensor-core flops on this path:
+        # the analysis multiplies by Phi split into bf16 hi + lo parts, the
+        # synthesis runs at the tf32 rate (half the bf16 rate)
+        rec["roofline"] = {"bound": "tensor", "algorithmic_flops": flops, "achieved_tflops": tf,
+                           "peak_tflops": tpk / 2, "frac": tf / (tpk / 2),
+                           "peak": f"bf16 sustained ({kind}) / 2: two bf16 tensor flops per algorithmic flop"}
     if with_cpu:
         shapes = []
         for j, s in enumerate(w.mats):
@@ -483,6 +521,9 @@ def main():
     world = int(os.environ.get("WORLD_SIZE", "1"))
     from paper_2608_26430_gb300 import workloads as wl
     w = wl.WORKLOADS[args.workload or wl.HEADLINE]
+    if args.tokens is not None:
+        import dataclasses
+        w = dataclasses.replace(w, N=args.tokens)
     if args.impl == "reference":
         return reference_arm(args, w, rank, world)
 
@@ -582,7 +623,7 @@ def main():
     serving = serving_timing(dev, stream) if args.serving else None
 
     per_config = None
-    if rank == 0 and not args.no_per_config and args.mats is None:
+    if rank == 0 and not args.no_per_config and args.mats is None and args.tokens is None:
         flush = L2Flush(dev)
         per_config = {}
         with_cpu = world == 1 and not args.no_cpu
@@ -602,7 +643,8 @@ def main():
                "vs_baseline": None, "dtype": w.dtype, "data": "synthetic", "config": cfg,
                "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                             "frac": achieved / peak,
-                            "traffic": measured_traffic() if args.mats is None and args.workload is None else None,
+                            "traffic": (measured_traffic()
+                                        if args.mats is None and args.workload is None and args.tokens is None else None),
                             "peak_kind": peak_kind,
                             "kernel": ",".join(kernels) + " + dc_reduce_kernel",
                             "kernel_ms": kernel_ms,

@@ -42,7 +42,7 @@
 extern "C" {
 #endif
 
-#define FRAMEFB_ABI_VERSION 1
+#define FRAMEFB_ABI_VERSION 2
 
 /* Threads per CTA of the activation kernels; plans are cut for this count. */
 #define FRAMEFB_THREADS 256
@@ -119,7 +119,21 @@ typedef struct {
 framefb_status framefb_frame_build(int32_t d, const framefb_frame_params* params, framefb_frame* out);
 void framefb_frame_free(framefb_frame* f);
 
-/* Device view of a frame: fp32 copies of the CSC arrays uploaded by the caller. */
+/*
+ * Device view of a frame: fp32 copies of the CSC arrays uploaded by the
+ * caller, and (for frames outside the structured kernels) the dense operand
+ * image.
+ *
+ * Two device paths exist.  Frames with k = 16 and k*rho = d (dft_groups set:
+ * rho/2 disjoint 32-coordinate groups, each a realified DFT_16 block) run on
+ * the structured kernels, which read `val` only.  Every other frame the
+ * builder produces -- the paper's own rho = 2 regime (k*rho = d with one
+ * group: Phi is a dense realified DFT of size d/2) and redundant frames with
+ * T blocks (k*rho > d) -- runs on the dense path, which treats Phi as a
+ * dense d x ncols matrix and reads it from `dense`: a device copy, byte for
+ * byte, of the image framefb_frame_dense_pack() writes (16-byte aligned).
+ * `dense` may be NULL for structured frames.
+ */
 typedef struct {
   int32_t d, k, rho, ncols;
   int32_t dft_groups;
@@ -127,7 +141,21 @@ typedef struct {
   const int64_t* colptr;    /* device [ncols+1] */
   const int32_t* rowidx;    /* device [nnz] */
   const float*   val;       /* device [nnz], fp32 */
+  const void*    dense;     /* device dense operand image, or NULL (see above) */
 } framefb_dev_frame;
+
+/*
+ * Dense operand image of a frame for the dense path (any frame; needed for
+ * frames without dft_groups and k = 16).  framefb_frame_dense_bytes() gives
+ * its size (0 for a NULL or empty frame); framefb_frame_dense_pack() writes
+ * it into the caller's host buffer `out` of `bytes` bytes: Phi's columns as
+ * bf16 hi + lo parts (the analysis operand) and Phi's rows rounded to tf32
+ * (the synthesis operand), zero-padded rows.  The caller copies it verbatim
+ * to the device and points framefb_dev_frame.dense at the copy.
+ * FRAMEFB_EINVAL for a NULL argument or a buffer that is too small.
+ */
+size_t framefb_frame_dense_bytes(const framefb_frame* f);
+framefb_status framefb_frame_dense_pack(const framefb_frame* f, void* out, size_t bytes);
 
 /* ------------------------------------------------------------------------ */
 /* S2  coefficient support (host)                                            */
@@ -163,8 +191,11 @@ framefb_status framefb_support_build(int32_t rows, int32_t cols, int64_t nnz, ui
  * fin, fout: host frames (Phi_in with d = n, Phi_out with d = m).
  * row, col: host, the support in sorted row-major order (as from
  * framefb_support_build); C values passed to the kernels follow this order.
- * The GPU path needs fin->dft_groups and fout->dft_groups with k = 16
- * (FRAMEFB_EUNSUPPORTED otherwise).  nnz may be 0.
+ * C is K_m x K_n with K = the frame's ncols (= k*rho).  When both frames
+ * have dft_groups and k = 16 the plan is cut for the structured kernels
+ * (frame columns re-indexed group-major); otherwise for the dense path
+ * (frame columns in the paper's order).  FRAMEFB_EUNSUPPORTED when a frame
+ * has more than 32767 columns.  nnz may be 0.
  */
 typedef struct framefb_plan framefb_plan;
 framefb_status framefb_plan_build(const framefb_frame* fin, const framefb_frame* fout,

@@ -47,7 +47,7 @@ class AdapterBatch:
         self.indices = list(range(len(w.mats))) if indices is None else list(indices)
         self.dtype = wl.torch_dtype(w)
         self.dtype_code = ffb.FRAMEFB_F32 if w.dtype == "f32" else ffb.FRAMEFB_BF16
-        self.frames = {d: ffb.Frame(d, w.k, d // w.k, parseval=True) for d in w.dims()}
+        self.frames = {d: ffb.Frame(d, *wl.frame_params(w, d), parseval=True) for d in w.dims()}
         self.dev_frames = {d: f.to_device(device) for d, f in self.frames.items()}
         # one support and plan per shape (shared across layers, Sec. 3.3), or
         # per matrix for per-layer supports
@@ -57,7 +57,8 @@ class AdapterBatch:
             if key in self.plans:
                 continue
             m, n = key[0], key[1]
-            row, col, _, _ = ffb.framefb_support_build(m, n, w.nnz, wl.support_seed_of(w, i), w.support_mode,
+            km, kn = self.frames[m].ncols, self.frames[n].ncols  # C is K_m x K_n
+            row, col, _, _ = ffb.framefb_support_build(km, kn, w.nnz, wl.support_seed_of(w, i), w.support_mode,
                                                        w.zipf_s, w.k)
             self.supports[key] = (row, col)
             self.plans[key] = ffb.Plan(self.frames[n], self.frames[m], row, col)
@@ -74,25 +75,38 @@ class AdapterBatch:
             if ops & (ffb.OP_FORWARD | ffb.OP_GRAD_COEFF):
                 if alias_inputs:
                     if spec.n not in shared_x:
-                        shared_x[spec.n] = wl.x_input(w, i, self.N, device)
+                        shared_x[spec.n] = self._pad(wl.x_input(w, i, self.N, device))
                     b.X = shared_x[spec.n]
                 else:
-                    b.X = wl.x_input(w, i, self.N, device)
+                    b.X = self._pad(wl.x_input(w, i, self.N, device))
             if ops & (ffb.OP_BACKWARD_DX | ffb.OP_GRAD_COEFF):
                 if alias_inputs:
                     if spec.m not in shared_dy:
-                        shared_dy[spec.m] = wl.dy_input(w, i, self.N, device)
+                        shared_dy[spec.m] = self._pad(wl.dy_input(w, i, self.N, device))
                     b.dY = shared_dy[spec.m]
                 else:
-                    b.dY = wl.dy_input(w, i, self.N, device)
+                    b.dY = self._pad(wl.dy_input(w, i, self.N, device))
             if ops & ffb.OP_FORWARD:
-                b.Y = self._init((self.N, spec.m), y_init, i, 7)
+                b.Y = self._pad(self._init((self.N, spec.m), y_init, i, 7))
             if ops & ffb.OP_BACKWARD_DX:
-                b.dX = self._init((self.N, spec.n), y_init, i, 8)
+                b.dX = self._pad(self._init((self.N, spec.n), y_init, i, 8))
             if ops & ffb.OP_GRAD_COEFF:
                 b.dC = self.dC[r]
             self.bufs.append(b)
         self.mats = [self._mat(b, key) for b, key in zip(self.bufs, self.keys)]
+
+    def _pad(self, t):
+        """t itself, or a view of it inside rows padded to 16 bytes (the
+        interface's row alignment) when its width needs it."""
+        import torch
+        d = t.shape[1]
+        per = 16 // t.element_size()
+        ld = (d + per - 1) // per * per
+        if ld == d:
+            return t
+        p = torch.zeros((t.shape[0], ld), dtype=t.dtype, device=t.device)
+        p[:, :d] = t
+        return p[:, :d]
 
     def _init(self, shape, kind, i, salt):
         import torch
@@ -102,8 +116,14 @@ class AdapterBatch:
 
     def _mat(self, b: MatBuffers, key):
         spec = b.spec
+        def ld(*ts):
+            for t in ts:
+                if t is not None:
+                    return t.stride(0)
+            return None
         return ffb.make_mat(self.dev_frames[spec.n], self.dev_frames[spec.m], self.plans[key], self.plan_dev[key],
-                            b.c_val, b.scale, self.N, X=b.X, dX=b.dX, dY=b.dY, Y=b.Y, dC=b.dC, ldx=spec.n, ldy=spec.m)
+                            b.c_val, b.scale, self.N, X=b.X, dX=b.dX, dY=b.dY, Y=b.Y, dC=b.dC,
+                            ldx=ld(b.X, b.dX) or spec.n, ldy=ld(b.dY, b.Y) or spec.m)
 
     def workspace(self, ops: int):
         return ffb.workspace(self.mats, ops, self.device)

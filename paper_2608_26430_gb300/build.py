@@ -21,7 +21,7 @@ BUILD = os.path.join(ROOT, "_build")
 LIB = os.path.join(PKG, "libframefb.so")
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-SOURCES = ["framefb_host.cpp", "framefb_cuda.cu"]
+SOURCES = ["framefb_host.cpp", "framefb_cuda.cu", "framefb_dense.cu"]
 
 
 def _nvcc() -> str:

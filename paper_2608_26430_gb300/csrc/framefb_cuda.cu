@@ -12,6 +12,7 @@
 #include <vector>
 
 #include "framefb.h"
+#include "framefb_dense.h"
 #include "framefb_kernels.cuh"
 #include "framefb_mma.cuh"
 #include "framefb_tc.cuh"
@@ -35,6 +36,12 @@ const FfbPlanHeader* plan_header(const framefb_plan* p) {
   if (h->magic != FFB_PLAN_MAGIC || h->version != FFB_PLAN_VERSION || h->P != kThreads) return nullptr;
   if (static_cast<size_t>(h->total_bytes) != p->image.size()) return nullptr;
   return h;
+}
+
+// Plan of the structured kernels (group-major index space), else NULL.
+const FfbPlanHeader* groups_header(const framefb_plan* p) {
+  const FfbPlanHeader* h = plan_header(p);
+  return h && h->layout == FFB_LAYOUT_GROUPS ? h : nullptr;
 }
 
 bool frame_ok(const framefb_dev_frame* f, int32_t d) {
@@ -246,23 +253,8 @@ size_t tc2_smem_map(const framefb_mat* mats, int32_t nmats, int32_t ops, int S, 
   return mbar + 8 * static_cast<size_t>(S + 3);  // stages, analysis, synthesis, RZ/RG written
 }
 
-// cuTensorMapEncodeTiled through the runtime's driver entry point (no link
-// against the driver library).
-using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
-                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
-                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
-EncodeTiledFn encode_tiled() {
-  static const EncodeTiledFn fn = [] {
-    void* p = nullptr;
-    cudaDriverEntryPointQueryResult q{};
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) !=
-            cudaSuccess ||
-        q != cudaDriverEntryPointSuccess)
-      return static_cast<EncodeTiledFn>(nullptr);
-    return reinterpret_cast<EncodeTiledFn>(p);
-  }();
-  return fn;
-}
+using ffb_host::encode_tiled;
+using ffb_host::EncodeTiledFn;
 
 // Tensor map of the bf16 rows of one activation tensor (d features, N
 // tokens, leading dimension ld elements): {32 coordinates, d / 32 groups, N
@@ -301,7 +293,7 @@ framefb_status prepare(const framefb_mat* mats, int32_t nmats, int32_t ops, fram
   bool reg = true;
   int32_t nnz_max = 0;
   for (int32_t j = 0; j < nmats; ++j) {
-    const FfbPlanHeader* h = plan_header(mats[j].plan);
+    const FfbPlanHeader* h = groups_header(mats[j].plan);
     if (!h) return FRAMEFB_EINVAL;
     if (h->EZ > ffb::kEreg || h->EG > ffb::kEreg) reg = false;
     nnz_max = std::max(nnz_max, h->nnz);
@@ -501,8 +493,10 @@ bool ops_ok(int32_t ops) { return ops == 1 || ops == 2 || ops == 4 || ops == 6 |
 
 }  // namespace
 
-extern "C" size_t framefb_workspace_size(const framefb_mat* mats, int32_t nmats, int32_t ops) {
-  if (!mats || nmats <= 0 || !ops_ok(ops)) return 0;
+namespace {
+
+size_t structured_workspace(const framefb_mat* mats, int32_t nmats, int32_t ops) {
+  if (nmats <= 0) return 0;
   Buffers b;
   size_t need = 0;
   // the workspace depends on the launch chunking, the kernel and its grid,
@@ -526,24 +520,26 @@ extern "C" size_t framefb_workspace_size(const framefb_mat* mats, int32_t nmats,
   return any ? need : 0;
 }
 
-extern "C" framefb_status framefb_run(const framefb_mat* mats, int32_t nmats, int32_t ops, framefb_dtype dtype,
-                                      void* ws, size_t ws_bytes, void* stream) {
-  if (nmats < 0 || (nmats > 0 && !mats) || !ops_ok(ops)) return FRAMEFB_EINVAL;
-  if (dtype != FRAMEFB_F32 && dtype != FRAMEFB_BF16) return FRAMEFB_EINVAL;
-  if (nmats == 0) return FRAMEFB_OK;
-  cudaStream_t st = static_cast<cudaStream_t>(stream);
+// Validate every launch chunk of the structured matrices; *need = the
+// workspace the largest chunk needs.
+framefb_status structured_check(const framefb_mat* mats, int32_t nmats, int32_t ops, framefb_dtype dtype,
+                                size_t* need) {
+  *need = 0;
   Buffers b;
-  // validate every chunk before queueing anything
   for (int32_t j0 = 0, nm = 0; j0 < nmats; j0 += nm) {
     nm = chunk_len(mats + j0, nmats - j0, dtype);
     Prepared P = b.prep();
     const framefb_status s = prepare(mats + j0, nm, ops, dtype, P);
     if (s != FRAMEFB_OK) return s;
-    if (P.ws_bytes > 0) {
-      if (!ws || ws_bytes < P.ws_bytes) return FRAMEFB_EWORKSPACE;
-      if (reinterpret_cast<uintptr_t>(ws) & 255u) return FRAMEFB_EINVAL;
-    }
+    *need = std::max(*need, P.ws_bytes);
   }
+  return FRAMEFB_OK;
+}
+
+// Queue the structured kernels (after structured_check).
+framefb_status structured_run(const framefb_mat* mats, int32_t nmats, int32_t ops, framefb_dtype dtype, void* ws,
+                              cudaStream_t st) {
+  Buffers b;
   for (int32_t j0 = 0, nm = 0; j0 < nmats; j0 += nm) {
     nm = chunk_len(mats + j0, nmats - j0, dtype);
     Prepared P = b.prep();
@@ -580,14 +576,9 @@ extern "C" framefb_status framefb_run(const framefb_mat* mats, int32_t nmats, in
   return FRAMEFB_OK;
 }
 
-extern "C" framefb_status framefb_kernel_names(const framefb_mat* mats, int32_t nmats, int32_t ops,
-                                               framefb_dtype dtype, char* buf, size_t len) {
-  if (!buf || len == 0) return FRAMEFB_EINVAL;
-  buf[0] = '\0';
-  if (nmats < 0 || (nmats > 0 && !mats) || !ops_ok(ops)) return FRAMEFB_EINVAL;
-  if (dtype != FRAMEFB_F32 && dtype != FRAMEFB_BF16) return FRAMEFB_EINVAL;
+framefb_status structured_names(const framefb_mat* mats, int32_t nmats, int32_t ops, framefb_dtype dtype,
+                                std::vector<std::string>& names) {
   Buffers b;
-  std::vector<std::string> names;
   for (int32_t j0 = 0, nm = 0; j0 < nmats; j0 += nm) {
     nm = chunk_len(mats + j0, nmats - j0, dtype);
     Prepared P = b.prep();
@@ -599,6 +590,85 @@ extern "C" framefb_status framefb_kernel_names(const framefb_mat* mats, int32_t 
                            : (dtype == FRAMEFB_BF16 ? "mma_tile_kernel" : "fft_tile_kernel");
     k += "<" + std::to_string(ops) + ">";
     if (std::find(names.begin(), names.end(), k) == names.end()) names.push_back(k);
+  }
+  return FRAMEFB_OK;
+}
+
+
+// Matrices of a call split by path: plans cut for the structured kernels
+// and plans of the dense path, each in call order.
+framefb_status split_paths(const framefb_mat* mats, int32_t nmats, std::vector<framefb_mat>& grp,
+                           std::vector<framefb_mat>& den) {
+  try {
+    for (int32_t j = 0; j < nmats; ++j) {
+      const FfbPlanHeader* h = plan_header(mats[j].plan);
+      if (!h) return FRAMEFB_EINVAL;
+      (h->layout == FFB_LAYOUT_DENSE ? den : grp).push_back(mats[j]);
+    }
+  } catch (const std::bad_alloc&) {
+    return FRAMEFB_ENOMEM;
+  }
+  return FRAMEFB_OK;
+}
+
+}  // namespace
+
+extern "C" size_t framefb_workspace_size(const framefb_mat* mats, int32_t nmats, int32_t ops) {
+  if (!mats || nmats <= 0 || !ops_ok(ops)) return 0;
+  std::vector<framefb_mat> grp, den;
+  if (split_paths(mats, nmats, grp, den) != FRAMEFB_OK) return 0;
+  size_t dneed = 0;
+  if (!den.empty() && ffb_host::dense_check(den.data(), static_cast<int32_t>(den.size()), ops, FRAMEFB_BF16, &dneed) !=
+                          FRAMEFB_OK)
+    return 0;
+  return std::max(structured_workspace(grp.data(), static_cast<int32_t>(grp.size()), ops), dneed);
+}
+
+extern "C" framefb_status framefb_run(const framefb_mat* mats, int32_t nmats, int32_t ops, framefb_dtype dtype,
+                                      void* ws, size_t ws_bytes, void* stream) {
+  if (nmats < 0 || (nmats > 0 && !mats) || !ops_ok(ops)) return FRAMEFB_EINVAL;
+  if (dtype != FRAMEFB_F32 && dtype != FRAMEFB_BF16) return FRAMEFB_EINVAL;
+  if (nmats == 0) return FRAMEFB_OK;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  std::vector<framefb_mat> grp, den;
+  framefb_status s = split_paths(mats, nmats, grp, den);
+  if (s != FRAMEFB_OK) return s;
+  // validate everything before queueing anything; the two paths run one
+  // after the other on the stream and share the workspace
+  size_t gneed = 0, dneed = 0;
+  s = structured_check(grp.data(), static_cast<int32_t>(grp.size()), ops, dtype, &gneed);
+  if (s != FRAMEFB_OK) return s;
+  s = ffb_host::dense_check(den.data(), static_cast<int32_t>(den.size()), ops, dtype, &dneed);
+  if (s != FRAMEFB_OK) return s;
+  const size_t need = std::max(gneed, dneed);
+  if (need > 0) {
+    if (!ws || ws_bytes < need) return FRAMEFB_EWORKSPACE;
+    if (reinterpret_cast<uintptr_t>(ws) & 255u) return FRAMEFB_EINVAL;
+  }
+  s = structured_run(grp.data(), static_cast<int32_t>(grp.size()), ops, dtype, ws, st);
+  if (s != FRAMEFB_OK) return s;
+  return ffb_host::dense_run(den.data(), static_cast<int32_t>(den.size()), ops, dtype, ws, ws_bytes, st);
+}
+
+extern "C" framefb_status framefb_kernel_names(const framefb_mat* mats, int32_t nmats, int32_t ops,
+                                               framefb_dtype dtype, char* buf, size_t len) {
+  if (!buf || len == 0) return FRAMEFB_EINVAL;
+  buf[0] = '\0';
+  if (nmats < 0 || (nmats > 0 && !mats) || !ops_ok(ops)) return FRAMEFB_EINVAL;
+  if (dtype != FRAMEFB_F32 && dtype != FRAMEFB_BF16) return FRAMEFB_EINVAL;
+  std::vector<framefb_mat> grp, den;
+  framefb_status s = split_paths(mats, nmats, grp, den);
+  if (s != FRAMEFB_OK) return s;
+  std::vector<std::string> names;
+  s = structured_names(grp.data(), static_cast<int32_t>(grp.size()), ops, dtype, names);
+  if (s != FRAMEFB_OK) return s;
+  if (!den.empty()) {
+    size_t need = 0;
+    s = ffb_host::dense_check(den.data(), static_cast<int32_t>(den.size()), ops, dtype, &need);
+    if (s != FRAMEFB_OK) return s;
+    bool any_tokens = false;
+    for (const framefb_mat& M : den) any_tokens = any_tokens || M.N > 0;
+    if (any_tokens) ffb_host::dense_kernel_names(ops, names);
   }
   std::string out;
   for (const std::string& k : names) out += (out.empty() ? "" : ",") + k;
@@ -635,7 +705,9 @@ extern "C" framefb_status framefb_merge(const void* W0, framefb_dtype dtype, int
                                         int32_t T, float scale, void* Wout, void* stream) {
   if (dtype != FRAMEFB_F32 && dtype != FRAMEFB_BF16) return FRAMEFB_EINVAL;
   const FfbPlanHeader* h = plan_header(plan);
-  if (!h || m <= 0 || n <= 0 || T < 0 || h->m != m || h->n != n) return FRAMEFB_EINVAL;
+  if (!h || m <= 0 || n <= 0 || T < 0) return FRAMEFB_EINVAL;
+  if (h->layout != FFB_LAYOUT_GROUPS) return FRAMEFB_EUNSUPPORTED;  // the merge kernel takes DFT_16-group frames
+  if (h->m != m || h->n != n) return FRAMEFB_EINVAL;
   if (!frame_ok(fin, n) || !frame_ok(fout, m)) return FRAMEFB_EINVAL;
   const size_t esz = dtype == FRAMEFB_BF16 ? 2 : 4;
   if (ldw < n || (ldw * esz) % 16 || !std::isfinite(scale)) return FRAMEFB_EINVAL;
@@ -831,6 +903,10 @@ extern "C" framefb_status framefb_run_static_ws(const framefb_mat* mats, int32_t
 
 extern "C" framefb_status framefb_wait_timeouts(uint32_t* count) {
   if (!count) return FRAMEFB_EINVAL;
-  if (cudaMemcpyFromSymbol(count, ffb::g_wait_timeouts, sizeof(uint32_t)) != cudaSuccess) return FRAMEFB_ECUDA;
+  uint32_t structured = 0, dense = 0;
+  if (cudaMemcpyFromSymbol(&structured, ffb::g_wait_timeouts, sizeof(uint32_t)) != cudaSuccess) return FRAMEFB_ECUDA;
+  const framefb_status s = ffb_host::dense_wait_timeouts(&dense);
+  if (s != FRAMEFB_OK) return s;
+  *count = structured + dense;
   return FRAMEFB_OK;
 }

@@ -1,0 +1,387 @@
+// Launchers of the dense path of libframefb (frames outside the structured
+// kernels): validation, workspace sizing, tensor maps, and per matrix and
+// token chunk the sequence analysis GEMM -> coefficient SpMM -> synthesis
+// GEMM, then the deterministic dC reduction.  See framefb_dense.cuh.
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "dense_layout.h"
+#include "framefb.h"
+#include "framefb_dense.cuh"
+#include "framefb_dense.h"
+#include "plan_internal.h"
+#include "plan_layout.h"
+
+namespace ffb_host {
+
+EncodeTiledFn encode_tiled() {
+  static const EncodeTiledFn fn = [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q{};
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) !=
+            cudaSuccess ||
+        q != cudaDriverEntryPointSuccess)
+      return static_cast<EncodeTiledFn>(nullptr);
+    return reinterpret_cast<EncodeTiledFn>(p);
+  }();
+  return fn;
+}
+
+namespace {
+
+namespace fd = ffb::dense;
+
+constexpr int kAnBN = 128;          // analysis tile columns (bf16 hi + lo operands)
+constexpr int kSyBN = 256;          // synthesis tile columns (tf32 operand)
+constexpr int64_t kChunk = 8192;    // tokens per pass: bounds the workspace
+constexpr int kSmemOptin = 227 * 1024;
+
+using AnShape = fd::GemmShape<fd::KIND_BF16_HILO, kAnBN>;
+using SyShape = fd::GemmShape<fd::KIND_TF32, kSyBN>;
+
+inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+inline int64_t rup(int64_t x, int64_t a) { return (x + a - 1) / a * a; }
+
+const FfbPlanHeader* header_of(const framefb_plan* p) {
+  if (!p || p->image.size() < sizeof(FfbPlanHeader)) return nullptr;
+  const FfbPlanHeader* h = reinterpret_cast<const FfbPlanHeader*>(p->image.data());
+  if (h->magic != FFB_PLAN_MAGIC || h->version != FFB_PLAN_VERSION || h->P != fd::kSpmmThreads) return nullptr;
+  if (static_cast<size_t>(h->total_bytes) != p->image.size()) return nullptr;
+  return h;
+}
+
+// One SpMM pass: the MODE bits it runs, its tokens per unit and shared memory.
+struct SpmmPass {
+  int mode, TT;
+  size_t smem;
+  int32_t oV, oU, oRZ, oRG, oDC;
+};
+
+// Shared-memory map of a SpMM pass (floats), 0 bytes when it does not fit.
+SpmmPass spmm_pass(const FfbPlanHeader& h, int mode, int TT) {
+  const bool F = mode & 1, D = mode & 2, C = mode & 4;
+  SpmmPass s{mode, TT, 0, 0, 0, 0, 0, 0};
+  int64_t off = 0;
+  auto take = [&](int64_t floats) {
+    const int32_t o = static_cast<int32_t>(off);
+    off = rup(off + floats, 4);
+    return o;
+  };
+  s.oV = take((F || C) ? rup(h.n, 4) * TT : 0);
+  s.oU = take((D || C) ? rup(h.m, 4) * TT : 0);
+  s.oRZ = take(F ? rup(h.m + h.ovfZ, 4) * TT : 0);
+  s.oRG = take(D ? rup(h.n + h.ovfG, 4) * TT : 0);
+  s.oDC = take(C ? static_cast<int64_t>(h.EG) * fd::kSpmmThreads : 0);
+  const size_t bytes = static_cast<size_t>(off) * 4;
+  s.smem = bytes <= static_cast<size_t>(kSmemOptin) ? std::max<size_t>(bytes, 16) : 0;
+  return s;
+}
+
+// The SpMM passes of `ops` (one pass when everything fits, else the column
+// path with dC first -- it still needs V -- then the row path, which
+// overwrites V with Z); empty when even one token per unit does not fit.
+std::vector<SpmmPass> spmm_passes(const FfbPlanHeader& h, int32_t ops) {
+  const int all = ops & 7;
+  for (int TT = 2; TT >= 1; --TT) {
+    const SpmmPass s = spmm_pass(h, all, TT);
+    if (s.smem) return {s};
+  }
+  const int col = all & 6, row = all & 1;
+  std::vector<SpmmPass> out;
+  for (const int m : {col, row}) {
+    if (!m) continue;
+    SpmmPass best{};
+    for (int TT = 2; TT >= 1 && !best.smem; --TT) best = spmm_pass(h, m, TT);
+    if (!best.smem) return {};
+    out.push_back(best);
+  }
+  return out;
+}
+
+// Geometry of one dense-path matrix.
+struct Geom {
+  const FfbPlanHeader* h;
+  int64_t Nc;       // tokens per chunk
+  int64_t nchunks;
+  int64_t ld;       // floats per workspace row (V/Z and U/G)
+  int32_t grid;     // SpMM CTAs of a full chunk
+  int32_t stride;   // dC partial slot stride (floats)
+  std::vector<SpmmPass> passes;
+  size_t off_ug, off_part, bytes;  // workspace map
+};
+
+framefb_status geom_of(const framefb_mat& M, int32_t ops, int sms, Geom& g) {
+  g.h = header_of(M.plan);
+  if (!g.h) return FRAMEFB_EINVAL;
+  const FfbPlanHeader& h = *g.h;
+  g.Nc = std::min<int64_t>(std::max<int32_t>(M.N, 1), kChunk);
+  g.nchunks = M.N > 0 ? (M.N + g.Nc - 1) / g.Nc : 0;
+  g.ld = rup(std::max(h.n, h.m), 4);
+  g.passes = spmm_passes(h, ops);
+  if (g.passes.empty()) return FRAMEFB_EUNSUPPORTED;
+  int tt = 2;
+  for (const SpmmPass& p : g.passes) tt = std::min(tt, p.TT);
+  const int64_t units = (g.Nc + tt - 1) / tt;
+  g.grid = static_cast<int32_t>(std::max<int64_t>(1, std::min<int64_t>(units, static_cast<int64_t>(sms) * 2)));
+  g.stride = (h.nnz + 63) & ~63;
+  const size_t rows = static_cast<size_t>(g.Nc) * g.ld * 4;
+  g.off_ug = rup(rows, 256);
+  g.off_part = g.off_ug + rup(rows, 256);
+  const size_t part = (ops & FRAMEFB_OP_GRAD_COEFF) && h.nnz > 0
+                          ? static_cast<size_t>(g.nchunks) * g.grid * g.stride * 4
+                          : 0;
+  g.bytes = g.off_part + rup(part, 256);
+  return FRAMEFB_OK;
+}
+
+int sm_count() {
+  int dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    return 0;
+  return sms;
+}
+
+bool check_mat(const framefb_mat& M, int32_t ops, const FfbPlanHeader& h) {
+  const bool F = ops & FRAMEFB_OP_FORWARD, D = ops & FRAMEFB_OP_BACKWARD_DX, C = ops & FRAMEFB_OP_GRAD_COEFF;
+  const framefb_dev_frame* fi = M.fin;
+  const framefb_dev_frame* fo = M.fout;
+  if (!fi || !fo || !fi->dense || !fo->dense || !aligned16(fi->dense) || !aligned16(fo->dense)) return false;
+  if (h.layout != FFB_LAYOUT_DENSE || h.n != fi->ncols || h.m != fo->ncols) return false;
+  if (h.d_in != M.n || h.d_out != M.m || fi->d != M.n || fo->d != M.m) return false;
+  if (M.N < 0 || !std::isfinite(M.scale)) return false;
+  if ((F || D) && h.nnz > 0 && !M.c_val) return false;
+  if (C && h.nnz > 0 && !M.dC) return false;
+  if (M.N == 0) return true;
+  const bool needX = F || C, needdY = D || C;
+  if ((needX || D) && (M.ldx < M.n || (M.ldx * 2) % 16)) return false;
+  if ((needdY || F) && (M.ldy < M.m || (M.ldy * 2) % 16)) return false;
+  if (needX && (!M.X || !aligned16(M.X))) return false;
+  if (needdY && (!M.dY || !aligned16(M.dY))) return false;
+  if (F && (!M.Y || !aligned16(M.Y))) return false;
+  if (D && (!M.dX || !aligned16(M.dX))) return false;
+  return true;
+}
+
+// 2-D tensor map of a row-major [rows][cols] matrix (pitch in bytes), box
+// {128 bytes of columns, box_rows rows}, 128-byte swizzle, zeros outside.
+bool encode_2d(CUtensorMap* map, CUtensorMapDataType type, int esz, const void* base, int64_t cols, int64_t rows,
+               int64_t pitch, int box_rows) {
+  const EncodeTiledFn fn = encode_tiled();
+  if (!fn || cols <= 0 || rows <= 0) return false;
+  const cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
+  const cuuint64_t strides[1] = {static_cast<cuuint64_t>(pitch)};
+  const cuuint32_t box[2] = {static_cast<cuuint32_t>(fd::kRowBytes / esz), static_cast<cuuint32_t>(box_rows)};
+  const cuuint32_t estr[2] = {1, 1};
+  return fn(map, type, 2, const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+            CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) ==
+         CUDA_SUCCESS;
+}
+
+void* spmm_kernel_ptr(int mode, int TT) {
+#define FFB_SPMM(M)                                                                       \
+  case M:                                                                                 \
+    return TT == 2 ? reinterpret_cast<void*>(fd::dense_spmm_kernel<M, 2>)                 \
+                   : reinterpret_cast<void*>(fd::dense_spmm_kernel<M, 1>);
+  switch (mode) {
+    FFB_SPMM(1)
+    FFB_SPMM(2)
+    FFB_SPMM(3)
+    FFB_SPMM(4)
+    FFB_SPMM(5)
+    FFB_SPMM(6)
+    FFB_SPMM(7)
+    default: return nullptr;
+  }
+#undef FFB_SPMM
+}
+
+void* an_kernel() { return reinterpret_cast<void*>(fd::dense_gemm_kernel<fd::KIND_BF16_HILO, fd::EPI_STORE_F32, kAnBN>); }
+void* sy_kernel() { return reinterpret_cast<void*>(fd::dense_gemm_kernel<fd::KIND_TF32, fd::EPI_ACCUM_BF16, kSyBN>); }
+
+// Queue one contraction launch over `L` (problems filled, tiles counted).
+framefb_status launch_gemm(void* fn, uint32_t smem, fd::GemmLaunch& L, int sms, cudaStream_t st) {
+  if (L.total_tiles == 0) return FRAMEFB_OK;
+  if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)) != cudaSuccess)
+    return FRAMEFB_ECUDA;
+  const int grid = std::min(L.total_tiles, sms);
+  void* args[] = {&L};
+  if (cudaLaunchKernel(fn, dim3(grid), dim3(fd::kGemmThreads), args, smem, st) != cudaSuccess) return FRAMEFB_ECUDA;
+  return FRAMEFB_OK;
+}
+
+// Append a problem to a launch: out[M][N] (+)= A[M][K] B[N][K]^T.
+void add_problem(fd::GemmLaunch& L, int BN, void* out, int64_t ldo, int64_t M, int64_t N, int64_t K, float alpha) {
+  fd::GemmProblem& P = L.p[L.nprob];
+  P.out = out;
+  P.ldo = ldo;
+  P.M = static_cast<int32_t>(M);
+  P.N = static_cast<int32_t>(N);
+  P.K = static_cast<int32_t>(K);
+  P.nt = static_cast<int32_t>((N + BN - 1) / BN);
+  P.tile0 = L.total_tiles;
+  P.alpha = alpha;
+  L.total_tiles += static_cast<int32_t>((M + fd::kBM - 1) / fd::kBM) * P.nt;
+  ++L.nprob;
+}
+
+}  // namespace
+
+framefb_status dense_check(const framefb_mat* mats, int32_t nmats, int32_t ops, framefb_dtype dt, size_t* ws_need) {
+  *ws_need = 0;
+  if (nmats == 0) return FRAMEFB_OK;
+  if (dt != FRAMEFB_BF16) return FRAMEFB_EUNSUPPORTED;  // the dense path takes bf16 activations
+  if (!encode_tiled()) return FRAMEFB_ECUDA;
+  const int sms = sm_count();
+  if (sms <= 0) return FRAMEFB_ECUDA;
+  for (int32_t j = 0; j < nmats; ++j) {
+    Geom g;
+    const framefb_status s = geom_of(mats[j], ops, sms, g);
+    if (s != FRAMEFB_OK) return s;
+    if (!check_mat(mats[j], ops, *g.h)) return FRAMEFB_EINVAL;
+    if (mats[j].N > 0 || ((ops & FRAMEFB_OP_GRAD_COEFF) && g.h->nnz > 0)) *ws_need = std::max(*ws_need, g.bytes);
+  }
+  return FRAMEFB_OK;
+}
+
+framefb_status dense_run(const framefb_mat* mats, int32_t nmats, int32_t ops, framefb_dtype dt, void* ws,
+                         size_t ws_bytes, cudaStream_t st) {
+  (void)dt;
+  (void)ws_bytes;
+  const bool F = ops & FRAMEFB_OP_FORWARD, D = ops & FRAMEFB_OP_BACKWARD_DX, C = ops & FRAMEFB_OP_GRAD_COEFF;
+  const int sms = sm_count();
+  if (sms <= 0) return FRAMEFB_ECUDA;
+  uint8_t* w = static_cast<uint8_t*>(ws);
+  for (int32_t j = 0; j < nmats; ++j) {
+    const framefb_mat& M = mats[j];
+    Geom g;
+    if (geom_of(M, ops, sms, g) != FRAMEFB_OK) return FRAMEFB_EINVAL;
+    const FfbPlanHeader& h = *g.h;
+    const int64_t Kn = h.n, Km = h.m;
+    float* VZ = reinterpret_cast<float*>(w);
+    float* UG = reinterpret_cast<float*>(w + g.off_ug);
+    float* part = reinterpret_cast<float*>(w + g.off_part);
+    const FfbDenseLayout Li = ffb_dense_layout(M.n, Kn), Lo = ffb_dense_layout(M.m, Km);
+    const uint8_t* di = static_cast<const uint8_t*>(M.fin->dense);
+    const uint8_t* dO = static_cast<const uint8_t*>(M.fout->dense);
+    int32_t slots = 0;
+    for (int64_t c = 0; c < g.nchunks; ++c) {
+      const int64_t t0 = c * g.Nc, Nc = std::min<int64_t>(g.Nc, M.N - t0);
+      // analysis: V = X Phi_in, U = dY Phi_out
+      if (F || C || D) {
+        fd::GemmLaunch L;
+        std::memset(&L, 0, sizeof(L));
+        if (F || C) {
+          fd::GemmProblem& P = L.p[L.nprob];
+          if (!encode_2d(&P.a, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+                         static_cast<const __nv_bfloat16*>(M.X) + t0 * M.ldx, M.n, Nc, M.ldx * 2, fd::kBM) ||
+              !encode_2d(&P.b0, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, di + Li.off_hi, M.n, Kn, Li.dp * 2, kAnBN) ||
+              !encode_2d(&P.b1, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, di + Li.off_lo, M.n, Kn, Li.dp * 2, kAnBN))
+            return FRAMEFB_ECUDA;
+          add_problem(L, kAnBN, VZ, g.ld, Nc, Kn, M.n, 1.f);
+        }
+        if (D || C) {
+          fd::GemmProblem& P = L.p[L.nprob];
+          if (!encode_2d(&P.a, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+                         static_cast<const __nv_bfloat16*>(M.dY) + t0 * M.ldy, M.m, Nc, M.ldy * 2, fd::kBM) ||
+              !encode_2d(&P.b0, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, dO + Lo.off_hi, M.m, Km, Lo.dp * 2, kAnBN) ||
+              !encode_2d(&P.b1, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, dO + Lo.off_lo, M.m, Km, Lo.dp * 2, kAnBN))
+            return FRAMEFB_ECUDA;
+          add_problem(L, kAnBN, UG, g.ld, Nc, Km, M.m, 1.f);
+        }
+        const framefb_status s = launch_gemm(an_kernel(), AnShape::SMEM, L, sms, st);
+        if (s != FRAMEFB_OK) return s;
+      }
+      // coefficient SpMM (Z over V, G over U, dC partials)
+      for (const SpmmPass& p : g.passes) {
+        fd::SpmmLaunch a;
+        std::memset(&a, 0, sizeof(a));
+        a.plan = static_cast<const uint8_t*>(M.plan_dev);
+        a.c_val = M.c_val;
+        a.VZ = VZ;
+        a.UG = UG;
+        a.partial = part;
+        a.ld = g.ld;
+        a.N = static_cast<int32_t>(Nc);
+        a.stride = g.stride;
+        a.slot0 = slots;
+        a.oV = p.oV;
+        a.oU = p.oU;
+        a.oRZ = p.oRZ;
+        a.oRG = p.oRG;
+        a.oDC = p.oDC;
+        const int64_t units = (Nc + p.TT - 1) / p.TT;
+        const int grid = static_cast<int>(std::min<int64_t>(units, g.grid));
+        void* fn = spmm_kernel_ptr(p.mode, p.TT);
+        if (!fn ||
+            cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(p.smem)) !=
+                cudaSuccess)
+          return FRAMEFB_ECUDA;
+        void* args[] = {&a};
+        if (cudaLaunchKernel(fn, dim3(grid), dim3(fd::kSpmmThreads), args, p.smem, st) != cudaSuccess)
+          return FRAMEFB_ECUDA;
+        if (p.mode & 4) slots += grid;
+      }
+      // synthesis: Y += s Z Phi_out^T, dX += s G Phi_in^T
+      if (F || D) {
+        fd::GemmLaunch L;
+        std::memset(&L, 0, sizeof(L));
+        if (F) {
+          fd::GemmProblem& P = L.p[L.nprob];
+          if (!encode_2d(&P.a, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, VZ, Km, Nc, g.ld * 4, fd::kBM) ||
+              !encode_2d(&P.b0, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, dO + Lo.off_sy, Km, M.m, Lo.cp * 4, kSyBN))
+            return FRAMEFB_ECUDA;
+          P.b1 = P.b0;
+          add_problem(L, kSyBN, static_cast<__nv_bfloat16*>(M.Y) + t0 * M.ldy, M.ldy, Nc, M.m, Km, M.scale);
+        }
+        if (D) {
+          fd::GemmProblem& P = L.p[L.nprob];
+          if (!encode_2d(&P.a, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, UG, Kn, Nc, g.ld * 4, fd::kBM) ||
+              !encode_2d(&P.b0, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, di + Li.off_sy, Kn, M.n, Li.cp * 4, kSyBN))
+            return FRAMEFB_ECUDA;
+          P.b1 = P.b0;
+          add_problem(L, kSyBN, static_cast<__nv_bfloat16*>(M.dX) + t0 * M.ldx, M.ldx, Nc, M.n, Kn, M.scale);
+        }
+        const framefb_status s = launch_gemm(sy_kernel(), SyShape::SMEM, L, sms, st);
+        if (s != FRAMEFB_OK) return s;
+      }
+    }
+    if (C && h.nnz > 0) {
+      if (slots == 0) {  // no tokens: the gradient is zero
+        if (cudaMemsetAsync(M.dC, 0, sizeof(float) * h.nnz, st) != cudaSuccess) return FRAMEFB_ECUDA;
+      } else {
+        const float* pp = part;
+        int32_t ns = slots, stride = g.stride, nnz = h.nnz;
+        float alpha = M.scale;
+        float* dC = M.dC;
+        void* args[] = {&pp, &ns, &stride, &nnz, &alpha, &dC};
+        if (cudaLaunchKernel(reinterpret_cast<void*>(fd::dense_dc_reduce_kernel), dim3((nnz + 255) / 256),
+                             dim3(256), args, 0, st) != cudaSuccess)
+          return FRAMEFB_ECUDA;
+      }
+    }
+  }
+  return FRAMEFB_OK;
+}
+
+void dense_kernel_names(int32_t ops, std::vector<std::string>& out) {
+  const bool F = ops & FRAMEFB_OP_FORWARD, D = ops & FRAMEFB_OP_BACKWARD_DX, C = ops & FRAMEFB_OP_GRAD_COEFF;
+  std::vector<std::string> k = {"dense_gemm_kernel<bf16_hilo>", "dense_spmm_kernel<" + std::to_string(ops & 7) + ">"};
+  if (F || D) k.push_back("dense_gemm_kernel<tf32>");
+  if (C) k.push_back("dense_dc_reduce_kernel");
+  for (const std::string& s : k)
+    if (std::find(out.begin(), out.end(), s) == out.end()) out.push_back(s);
+}
+
+framefb_status dense_wait_timeouts(uint32_t* count) {
+  if (cudaMemcpyFromSymbol(count, fd::g_dense_timeouts, sizeof(uint32_t)) != cudaSuccess) return FRAMEFB_ECUDA;
+  return FRAMEFB_OK;
+}
+
+}  // namespace ffb_host

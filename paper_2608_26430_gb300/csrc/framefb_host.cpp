@@ -1,6 +1,7 @@
 // Host side of libframefb: frame construction (S1), support sampling (S2),
 // plan building and status strings.  Plain C++17, no CUDA calls.
 #include "framefb.h"
+#include "dense_layout.h"
 #include "plan_layout.h"
 #include "plan_internal.h"
 
@@ -293,6 +294,60 @@ extern "C" framefb_status framefb_support_build(int32_t rows, int32_t cols, int6
 }
 
 // ---------------------------------------------------------------------------
+// Dense operand image of a frame (dense_layout.h).
+// ---------------------------------------------------------------------------
+namespace {
+
+inline uint32_t float_bits(float x) {
+  uint32_t u;
+  std::memcpy(&u, &x, 4);
+  return u;
+}
+inline float bits_float(uint32_t u) {
+  float x;
+  std::memcpy(&x, &u, 4);
+  return x;
+}
+// Round to nearest, ties to even, keeping the top `keep` bits of the fp32
+// pattern (finite inputs): 16 gives bf16, 19 gives tf32.
+inline uint32_t round_bits(float x, int keep) {
+  const int drop = 32 - keep;
+  uint32_t u = float_bits(x);
+  u += ((1u << (drop - 1)) - 1u) + ((u >> drop) & 1u);
+  return u & ~((1u << drop) - 1u);
+}
+
+}  // namespace
+
+extern "C" size_t framefb_frame_dense_bytes(const framefb_frame* f) {
+  if (!f || f->d <= 0 || f->ncols <= 0 || !f->csc_colptr || !f->csc_rowidx || !f->csc_val) return 0;
+  return static_cast<size_t>(ffb_dense_layout(f->d, f->ncols).total);
+}
+
+extern "C" framefb_status framefb_frame_dense_pack(const framefb_frame* f, void* out, size_t bytes) {
+  const size_t need = framefb_frame_dense_bytes(f);
+  if (need == 0 || !out || bytes < need) return FRAMEFB_EINVAL;
+  const FfbDenseLayout L = ffb_dense_layout(f->d, f->ncols);
+  uint8_t* base = static_cast<uint8_t*>(out);
+  std::memset(base, 0, need);
+  uint16_t* hi = reinterpret_cast<uint16_t*>(base + L.off_hi);
+  uint16_t* lo = reinterpret_cast<uint16_t*>(base + L.off_lo);
+  float* sy = reinterpret_cast<float*>(base + L.off_sy);
+  for (int32_t c = 0; c < f->ncols; ++c) {
+    for (int64_t e = f->csc_colptr[c]; e < f->csc_colptr[c + 1]; ++e) {
+      const int32_t j = f->csc_rowidx[e];
+      const double v = f->csc_val[e];
+      const uint32_t h = round_bits(static_cast<float>(v), 16);
+      const uint32_t l = round_bits(static_cast<float>(v - static_cast<double>(bits_float(h))), 16);
+      hi[static_cast<int64_t>(c) * L.dp + j] = static_cast<uint16_t>(h >> 16);
+      lo[static_cast<int64_t>(c) * L.dp + j] = static_cast<uint16_t>(l >> 16);
+      sy[static_cast<int64_t>(j) * L.cp + c] = bits_float(round_bits(static_cast<float>(v), 19));
+    }
+  }
+  return FRAMEFB_OK;
+}
+
+// ---------------------------------------------------------------------------
 // Plan: the support re-indexed group-major and cut into per-thread chunks.
 // ---------------------------------------------------------------------------
 namespace {
@@ -350,7 +405,7 @@ struct PathBanks {
 // Outputs: pos[p * E + e] = entry index or -1 (padding), store[entry] = its
 // store target or FFB_NO_STORE.
 void pack_runs(const std::vector<Entry>& ent, int32_t P, int32_t E, int32_t base, int32_t nkeys,
-               const PathBanks& bk, std::vector<int32_t>& pos, std::vector<int32_t>& store,
+               const PathBanks& bk, bool search, std::vector<int32_t>& pos, std::vector<int32_t>& store,
                std::vector<int32_t>& fix, int32_t& novf) {
   const int32_t nnz = static_cast<int32_t>(ent.size());
   pos.assign(static_cast<size_t>(P) * E, -1);
@@ -482,7 +537,7 @@ void pack_runs(const std::vector<Entry>& ent, int32_t P, int32_t E, int32_t base
     if (pl[k].len >= 2) multi.push_back(static_cast<int32_t>(k));
   }
   SplitMix64 rng{0x6A09E667F3BCC909ull ^ static_cast<uint64_t>(nnz)};
-  const int64_t iters = std::min<int64_t>(static_cast<int64_t>(nnz) * 4000, 60000000);
+  const int64_t iters = search ? std::min<int64_t>(static_cast<int64_t>(nnz) * 4000, 60000000) : 0;
   std::vector<std::pair<int32_t, int32_t>> cells;
   std::vector<int32_t> groups, newcost;
   auto add_cell = [&](int32_t p, int32_t e) {
@@ -601,10 +656,15 @@ extern "C" framefb_status framefb_plan_build(const framefb_frame* fin, const fra
   if (!out) return FRAMEFB_EINVAL;
   *out = nullptr;
   if (!fin || !fout || nnz < 0 || (nnz > 0 && (!row || !col))) return FRAMEFB_EINVAL;
-  if (!fin->dft_groups || !fout->dft_groups || fin->k != 16 || fout->k != 16) return FRAMEFB_EUNSUPPORTED;
-  const int32_t n = fin->d, m = fout->d;
-  if (n % FFB_GROUP || m % FFB_GROUP || fin->ncols != n || fout->ncols != m) return FRAMEFB_EUNSUPPORTED;
-  if (n > 32768 || m > 32768) return FRAMEFB_EUNSUPPORTED;  // 16-bit shared-memory offsets
+  if (fin->ncols <= 0 || fout->ncols <= 0 || fin->d <= 0 || fout->d <= 0) return FRAMEFB_EINVAL;
+  // structured kernels: both frames k = 16 with k*rho = d (32-coordinate
+  // DFT_16 groups); every other frame pair goes to the dense path
+  auto groups16 = [](const framefb_frame* f) {
+    return f->dft_groups && f->k == 16 && f->ncols == f->d && f->d % FFB_GROUP == 0;
+  };
+  const bool structured = groups16(fin) && groups16(fout);
+  const int32_t n = fin->ncols, m = fout->ncols;            // index spaces K_n, K_m
+  if (n > 32768 || m > 32768) return FRAMEFB_EUNSUPPORTED;  // 15-bit indices, 16-bit store targets
   if (nnz > static_cast<int64_t>(m) * n || nnz > (1 << 24)) return FRAMEFB_EINVAL;
   const int32_t nz = static_cast<int32_t>(nnz);
   for (int32_t q = 0; q < nz; ++q) {
@@ -617,10 +677,11 @@ extern "C" framefb_status framefb_plan_build(const framefb_frame* fin, const fra
   }
   try {
     const int32_t P = FRAMEFB_THREADS;
-    const int32_t Gn = n / FFB_GROUP, Gm = m / FFB_GROUP;
+    const int32_t Gn = (n + FFB_GROUP - 1) / FFB_GROUP, Gm = (m + FFB_GROUP - 1) / FFB_GROUP;
     std::vector<Entry> byrow(nz), bycol(nz);
     for (int32_t q = 0; q < nz; ++q) {
-      const int32_t a = group_major(row[q], fout->rho), b = group_major(col[q], fin->rho);
+      const int32_t a = structured ? group_major(row[q], fout->rho) : row[q];
+      const int32_t b = structured ? group_major(col[q], fin->rho) : col[q];
       byrow[q] = Entry{a, b, q};
       bycol[q] = Entry{b, a, q};
     }
@@ -656,7 +717,7 @@ extern "C" framefb_status framefb_plan_build(const framefb_frame* fin, const fra
       std::exception_ptr ez, eg;
       auto run_z = [&]() {
         try {
-          pack_runs(byrow, P, EZ, m, m, bkZ, posZ, storeZ, fixZ, novfZ);
+          pack_runs(byrow, P, EZ, m, m, bkZ, structured, posZ, storeZ, fixZ, novfZ);
         } catch (...) {
           ez = std::current_exception();
         }
@@ -668,7 +729,7 @@ extern "C" framefb_status framefb_plan_build(const framefb_frame* fin, const fra
         run_z();
       }
       try {
-        pack_runs(bycol, P, EG, n, n, bkG, posG, storeG, fixG, novfG);
+        pack_runs(bycol, P, EG, n, n, bkG, structured, posG, storeG, fixG, novfG);
       } catch (...) {
         eg = std::current_exception();
       }
@@ -677,8 +738,14 @@ extern "C" framefb_status framefb_plan_build(const framefb_frame* fin, const fra
       if (eg) std::rethrow_exception(eg);
     }
 
+    // store targets (own slots and overflow slots) are 16-bit fields
+    if (m + novfZ >= static_cast<int32_t>(FFB_NO_STORE) || n + novfG >= static_cast<int32_t>(FFB_NO_STORE))
+      return FRAMEFB_EUNSUPPORTED;
     FfbPlanHeader h;
     std::memset(&h, 0, sizeof(h));
+    h.layout = structured ? FFB_LAYOUT_GROUPS : FFB_LAYOUT_DENSE;
+    h.d_in = fin->d;
+    h.d_out = fout->d;
     h.magic = FFB_PLAN_MAGIC;
     h.version = FFB_PLAN_VERSION;
     h.n = n;

@@ -2,12 +2,15 @@
 // offsets in bytes from the start of the image, every table 16-byte aligned.
 // Shared by the host builder (framefb_host.cpp) and the kernels (framefb_cuda.cu).
 //
-// Index spaces.  A frame column in the paper's order c = i*rho + 2r + s
-// (subspace i, Spectral Tetris row r, realified part s) is re-indexed
-// group-major as x = 32 r + 2 i + s, so that group r (coordinates
+// Index spaces.  For the structured kernels (FFB_LAYOUT_GROUPS) a frame
+// column in the paper's order c = i*rho + 2r + s (subspace i, Spectral
+// Tetris row r, realified part s) is re-indexed group-major as
+// x = 32 r + 2 i + s, so that group r (coordinates
 // [32 r, 32 r + 32) of a k = 16, k*rho = d frame) owns the 32 contiguous
 // columns [32 r, 32 r + 32): its coefficient vector is the 16 complex values
-// (Re, Im interleaved) of the DFT_16 of that coordinate block.
+// (Re, Im interleaved) of the DFT_16 of that coordinate block.  For the dense
+// path (FFB_LAYOUT_DENSE) the index is the paper's column c itself, and the
+// 32-wide "groups" of the masks are blocks of 32 consecutive columns.
 //
 // The tables hold these group-major indices.  A store target t < K (K = m
 // for the row side, n for the column side) is the index of the run's own
@@ -27,14 +30,16 @@
 #endif
 
 #define FFB_PLAN_MAGIC 0x50424646  /* "FFBP" */
-#define FFB_PLAN_VERSION 1
+#define FFB_PLAN_VERSION 2
+#define FFB_LAYOUT_GROUPS 0        /* structured kernels: group-major column index (k = 16, k*rho = d) */
+#define FFB_LAYOUT_DENSE 1         /* dense path: frame columns in the paper's order */
 #define FFB_GROUP 32               /* real coordinates (and frame columns) per group */
 #define FFB_NO_STORE 0xFFFFu
 #define FFB_ENTRY_BLOCK 8          /* entries a thread loads together in the sparse phase */
 
 struct FfbPlanHeader {
   int32_t magic, version;
-  int32_t n, m;            // in / out features (= K_n, K_m: k*rho = d)
+  int32_t n, m;            // index spaces K_n, K_m (frame columns; = features when k*rho = d)
   int32_t Gn, Gm;          // groups of 32 on the input / output side
   int32_t nnz;
   int32_t P;               // threads the chunks were cut for
@@ -48,7 +53,9 @@ struct FfbPlanHeader {
   int32_t off_blkptr;              // merge: [Gm*Gn + 1] entry ranges of each 32x32 block (g, h)
   int32_t off_blkent;              // merge: int2 {a_local | b_local << 8, c index}
   int32_t total_bytes;
-  int32_t reserved[6];
+  int32_t layout;          // FFB_LAYOUT_GROUPS or FFB_LAYOUT_DENSE (index space of the tables)
+  int32_t d_in, d_out;     // features of the frames (= n, m for FFB_LAYOUT_GROUPS)
+  int32_t reserved[3];
 };
 
 // Slot of group-major index x (x < K) in a tile buffer.  Slots come in

@@ -28,9 +28,10 @@ EXPORTED = [
     "framefb_workspace_size", "framefb_run", "framefb_forward", "framefb_backward_dx", "framefb_grad_coeff",
     "framefb_backward", "framefb_fused_fwd_bwd", "framefb_merge", "framefb_run_static_ws",
     "framefb_wait_timeouts", "framefb_adamw", "framefb_linear_warmup_lr", "framefb_forward_tenants",
-    "framefb_kernel_names",
+    "framefb_kernel_names", "framefb_frame_dense_bytes", "framefb_frame_dense_pack",
 ]
 STATIC_WS_BYTES = 8 << 20
+ABI_VERSION = 2  # FRAMEFB_ABI_VERSION of the structs below
 
 
 class FramefbError(RuntimeError):
@@ -57,7 +58,7 @@ class framefb_frame(ct.Structure):
 class framefb_dev_frame(ct.Structure):
     _fields_ = [("d", ct.c_int32), ("k", ct.c_int32), ("rho", ct.c_int32), ("ncols", ct.c_int32),
                 ("dft_groups", ct.c_int32), ("pad_", ct.c_int32),
-                ("colptr", ct.c_void_p), ("rowidx", ct.c_void_p), ("val", ct.c_void_p)]
+                ("colptr", ct.c_void_p), ("rowidx", ct.c_void_p), ("val", ct.c_void_p), ("dense", ct.c_void_p)]
 
 
 class framefb_mat(ct.Structure):
@@ -90,6 +91,10 @@ def lib() -> ct.CDLL:
         L.framefb_abi_version.restype = i32
         L.framefb_frame_build.restype = i32
         L.framefb_frame_build.argtypes = [i32, ct.POINTER(framefb_frame_params), ct.POINTER(framefb_frame)]
+        L.framefb_frame_dense_bytes.restype = sz
+        L.framefb_frame_dense_bytes.argtypes = [ct.POINTER(framefb_frame)]
+        L.framefb_frame_dense_pack.restype = i32
+        L.framefb_frame_dense_pack.argtypes = [ct.POINTER(framefb_frame), vp, sz]
         L.framefb_frame_free.restype = None
         L.framefb_frame_free.argtypes = [ct.POINTER(framefb_frame)]
         L.framefb_support_build.restype = i32
@@ -127,6 +132,9 @@ def lib() -> ct.CDLL:
         L.framefb_adamw.argtypes = [vp, vp, vp, vp, i64, ct.POINTER(framefb_adamw_params), i64, vp]
         L.framefb_linear_warmup_lr.restype = ct.c_double
         L.framefb_linear_warmup_lr.argtypes = [i64, i64, i64, ct.c_double]
+        if L.framefb_abi_version() != ABI_VERSION:
+            raise RuntimeError(f"{LIB_PATH} has ABI version {L.framefb_abi_version()}, the binding expects "
+                               f"{ABI_VERSION}: rebuild it")
         _lib = L
     return _lib
 
@@ -181,6 +189,19 @@ class Frame:
         return (np.ctypeslib.as_array(s.grp_row0, (s.ngroups,)).copy(),
                 np.ctypeslib.as_array(s.grp_nrows, (s.ngroups,)).copy())
 
+    @property
+    def structured(self) -> bool:
+        """True when the structured kernels take this frame (k = 16, k*rho = d)."""
+        s = self._s
+        return bool(s.dft_groups) and s.k == 16 and s.ncols == s.d and s.d % 32 == 0
+
+    def dense_image(self) -> np.ndarray:
+        """The dense operand image of the frame (framefb_frame_dense_pack)."""
+        n = int(lib().framefb_frame_dense_bytes(ct.byref(self._s)))
+        out = np.zeros(max(n, 1), dtype=np.uint8)
+        _check(lib().framefb_frame_dense_pack(ct.byref(self._s), out.ctypes.data, n), "framefb_frame_dense_pack")
+        return out[:n]
+
     def to_device(self, device) -> "DevFrame":
         return DevFrame(self, device)
 
@@ -190,16 +211,22 @@ def framefb_frame_build(d: int, k: int, rho: int, parseval: bool = True) -> Fram
 
 
 class DevFrame:
-    """fp32 device copy of a frame's CSC arrays plus the framefb_dev_frame view."""
+    """fp32 device copy of a frame's CSC arrays plus the framefb_dev_frame view;
+    frames outside the structured kernels also get their dense operand image
+    (or always, with dense=True)."""
 
-    def __init__(self, frame: Frame, device):
+    def __init__(self, frame: Frame, device, dense: bool | None = None):
         import torch
         colptr, rowidx, val = frame.csc()
         self.colptr = torch.from_numpy(colptr).to(device)
         self.rowidx = torch.from_numpy(rowidx).to(device)
         self.val = torch.from_numpy(val.astype(np.float32)).to(device)
+        self.dense = None
+        if dense if dense is not None else not frame.structured:
+            self.dense = torch.from_numpy(frame.dense_image()).to(device)
         self.struct = framefb_dev_frame(frame.d, frame.k, frame.rho, frame.ncols, frame.dft_groups, 0,
-                                        self.colptr.data_ptr(), self.rowidx.data_ptr(), self.val.data_ptr())
+                                        self.colptr.data_ptr(), self.rowidx.data_ptr(), self.val.data_ptr(),
+                                        _ptr(self.dense))
 
 
 # ---------------------------------------------------------------------------

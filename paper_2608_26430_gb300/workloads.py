@@ -41,6 +41,7 @@ class Workload:
     w0_std: float = 0.02
     support_seed: int = 1
     per_layer_support: bool = False  # one support per matrix instead of one per shape
+    frames: tuple = ()           # (d, k, rho) frame parameters overriding k = 16, rho = d / 16 for dimension d
     notes: str = ""
 
     def shapes(self):
@@ -103,8 +104,40 @@ WORKLOADS["roberta_per_layer"] = Workload(
     "roberta_per_layer", _layers(3, [("q", 768, 768), ("v", 768, 768)]), N=4096, nnz=1000, dtype="bf16",
     c_std=0.02, per_layer_support=True, notes="a distinct uniform support for every matrix")
 
+# The paper's own frame regime, rho = 2 (k = d / 2 subspaces of real dimension
+# 2, k*rho = d): every frame is one dense realified DFT of size d / 2
+# (Sec. 4 fine-tuning setup and the subspace-dimension ablation), at the
+# LLaMA-2 and RoBERTa shapes; and redundant frames with T blocks (k*rho > d,
+# the (6,3,11)-style construction of the appendix) at small odd shapes.
+WORKLOADS["llama2_rho2"] = Workload(
+    "llama2_rho2", _layers(32, [("q", 4096, 4096), ("k", 4096, 4096), ("v", 4096, 4096), ("o", 4096, 4096)]),
+    N=4 * 2048, nnz=4096, dtype="bf16", c_std=0.01, frames=((4096, 2048, 2),),
+    notes="LLaMA-2-7B q/k/v/o adapters with rho = 2 frames (dense DFT_2048 per token)")
+WORKLOADS["roberta_rho2"] = Workload(
+    "roberta_rho2", _layers(12, [("q", 768, 768), ("v", 768, 768)]), N=32 * 128, nnz=1000, dtype="bf16",
+    c_std=0.02, frames=((768, 384, 2),), notes="RoBERTa-base q/v adapters with rho = 2 frames (dense DFT_384)")
+WORKLOADS["tblock_tff"] = Workload(
+    "tblock_tff", (MatSpec("a", 40, 22), MatSpec("b", 46, 46), MatSpec("c", 22, 40)), N=300, nnz=200,
+    dtype="bf16", c_std=0.02, frames=((40, 7, 8), (22, 6, 6), (46, 10, 10)),
+    notes="redundant tight fusion frames with T blocks: (d, k, rho) = (40, 7, 8), (22, 6, 6), (46, 10, 10)")
+
 # The configuration the headline metric is quoted on.
 HEADLINE = "llama2_7b_qkvo"
+
+
+def frame_params(w: Workload, d: int):
+    """(k, rho) of the frame of dimension d in workload w."""
+    for dd, k, rho in w.frames:
+        if dd == d:
+            return k, rho
+    return w.k, d // w.k
+
+
+def coef_dims(w: Workload, spec: MatSpec):
+    """(K_m, K_n): rows and columns of C (frame columns k*rho of each side)."""
+    km, rm = frame_params(w, spec.m)
+    kn, rn = frame_params(w, spec.n)
+    return km * rm, kn * rn
 
 
 def support_key(w: Workload, mat_index: int):

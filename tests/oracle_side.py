@@ -14,8 +14,8 @@ from paper_2608_26430_gb300 import workloads as wl
 
 
 @lru_cache(maxsize=8)
-def frame(d: int, k: int) -> np.ndarray:
-    return frames.real_frame(d, k, d // k, parseval=True)
+def frame(d: int, k: int, rho: int | None = None) -> np.ndarray:
+    return frames.real_frame(d, k, d // k if rho is None else rho, parseval=True)
 
 
 @lru_cache(maxsize=16)
@@ -35,13 +35,15 @@ class Expect:
         spec = b.spec
         self.spec, self.scale = spec, b.scale
         seed = wl.support_seed_of(w, batch.indices[j])
-        row, col, _, _ = oracle_support(spec.m, spec.n, w.nnz, seed, w.support_mode, w.zipf_s, w.k)
+        km, kn = wl.coef_dims(w, spec)
+        row, col, _, _ = oracle_support(km, kn, w.nnz, seed, w.support_mode, w.zipf_s, w.k)
         lrow, lcol = batch.supports[batch.keys[j]]
         assert np.array_equal(row, lrow) and np.array_equal(col, lcol), "support differs from the oracle's"
         self.row, self.col = row, col
-        self.Pin, self.Pout = frame(spec.n, w.k), frame(spec.m, w.k)
+        self.Pin = frame(spec.n, *wl.frame_params(w, spec.n))
+        self.Pout = frame(spec.m, *wl.frame_params(w, spec.m))
         self.c = host64(b.c_val)
-        self.C = adapter.dense_C(spec.m, spec.n, row, col, self.c)
+        self.C = adapter.dense_C(km, kn, row, col, self.c)
         self._dW = None
 
     @property

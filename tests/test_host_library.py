@@ -29,7 +29,7 @@ def test_library_exports_every_declared_function():
     assert len(names) >= 17
     got = ffb.exported_symbols(names)
     assert all(got.values()), [n for n, ok in got.items() if not ok]
-    assert ffb.lib().framefb_abi_version() == 1
+    assert ffb.lib().framefb_abi_version() == 2
 
 
 @pytest.mark.parametrize("d,k,rho,parseval", [(256, 16, 16, True), (768, 16, 48, True), (22, 6, 6, False),
@@ -104,7 +104,7 @@ def test_support_build_rejects():
 # ---------------------------------------------------------------------------
 HDR = ["magic", "version", "n", "m", "Gn", "Gm", "nnz", "P", "EZ", "EG", "ovfZ", "ovfG", "nfixZ", "nfixG",
        "off_zb", "off_zq", "off_ga", "off_gb", "off_gq", "off_fixZ", "off_fixG", "off_zmask", "off_gmask",
-       "off_blkptr", "off_blkent", "total_bytes"]
+       "off_blkptr", "off_blkent", "total_bytes", "layout", "d_in", "d_out"]
 
 
 def decode(img):
@@ -170,17 +170,33 @@ PLAN_CASES = [(256, 256, 128, 0), (768, 768, 1000, 0), (768, 3072, 2000, 0), (40
               (768, 768, 1000, 2), (3072, 768, 2000, 2)]
 
 
-@pytest.mark.parametrize("n,m,nnz,mode", PLAN_CASES)
+# frames outside the structured kernels: plans cut for the dense path, whose
+# index space is the paper's column order (rho = 2 frames, T-block frames)
+DENSE_PLAN_CASES = [((768, 384, 2), (768, 384, 2), 1000, 0), ((4096, 2048, 2), (1024, 512, 2), 8192, 1),
+                    ((40, 7, 8), (22, 6, 6), 200, 0), ((46, 10, 10), (46, 10, 10), 2000, 1),
+                    ((256, 16, 16), (22, 6, 6), 300, 0)]
+
+
+@pytest.mark.parametrize("n,m,nnz,mode", PLAN_CASES + DENSE_PLAN_CASES)
 def test_plan_replays_coefficient_products(n, m, nnz, mode):
-    fin, fout = ffb.Frame(n, 16, n // 16), ffb.Frame(m, 16, m // 16)
+    pin = n if isinstance(n, tuple) else (n, 16, n // 16)
+    pout = m if isinstance(m, tuple) else (m, 16, m // 16)
+    fin, fout = ffb.Frame(*pin), ffb.Frame(*pout)
+    structured = fin.structured and fout.structured
+    n, m = pin[1] * pin[2], pout[1] * pout[2]  # index spaces K_n, K_m
     row, col, _, _ = support.sample_support(m, n, nnz, 1, mode, 1.1, 16)  # k: the diagonal blocks of mode 2
     t = decode(ffb.Plan(fin, fout, row, col).image())
     h = t["h"]
     assert h["magic"] == 0x50424646 and h["P"] == ffb.THREADS and h["nnz"] == nnz
+    assert h["layout"] == (0 if structured else 1) and (h["n"], h["m"]) == (n, m)
+    assert (h["d_in"], h["d_out"]) == (pin[0], pout[0])
     # every entry appears once in each chunk table
     assert sorted(t["zq"][t["zq"] >= 0].tolist()) == list(range(nnz))
     assert sorted(t["gq"][t["gq"] >= 0].tolist()) == list(range(nnz))
-    a_int, b_int = group_major(row, m // 16), group_major(col, n // 16)
+    if structured:
+        a_int, b_int = group_major(row, m // 16), group_major(col, n // 16)
+    else:
+        a_int, b_int = np.asarray(row), np.asarray(col)
     assert len(set(a_int.tolist())) == len(set(row.tolist()))
     # masks
     zm = np.zeros(h["Gm"], np.uint32)
@@ -258,13 +274,42 @@ def test_plan_rejects_unsorted_and_unsupported():
     with pytest.raises(ffb.FramefbError) as e:
         ffb.Plan(f256, f256, np.array([256], np.int32), np.array([0], np.int32))
     assert e.value.status == ffb.FRAMEFB_EINVAL
-    red = ffb.Frame(22, 6, 6)
-    with pytest.raises(ffb.FramefbError) as e:
-        ffb.Plan(red, red, np.array([0], np.int32), np.array([0], np.int32))
-    assert e.value.status == ffb.FRAMEFB_EUNSUPPORTED
-    dense = ffb.Frame(64, 32, 2)  # rho = 2: one dense DFT, no 32-wide groups (no device path yet)
-    with pytest.raises(ffb.FramefbError) as e:
-        ffb.Plan(dense, dense, np.array([0], np.int32), np.array([0], np.int32))
-    assert e.value.status == ffb.FRAMEFB_EUNSUPPORTED
+    # T-block and rho = 2 frames get plans cut for the dense path; a mixed
+    # pair (one structured frame) does too
+    red, dense = ffb.Frame(22, 6, 6), ffb.Frame(64, 32, 2)
+    for fi, fo, K in ((red, red, 36), (dense, dense, 64), (f256, red, 36)):
+        h = decode(ffb.Plan(fi, fo, np.array([0, 1], np.int32), np.array([0, 3], np.int32)).image())["h"]
+        assert h["layout"] == 1 and h["m"] == K
+    with pytest.raises(ffb.FramefbError) as e:  # row outside K_m = 36
+        ffb.Plan(red, red, np.array([36], np.int32), np.array([0], np.int32))
+    assert e.value.status == ffb.FRAMEFB_EINVAL
     p = ffb.Plan(f256, f256, np.zeros(0, np.int32), np.zeros(0, np.int32))
     assert decode(p.image())["h"]["nnz"] == 0
+
+
+@pytest.mark.parametrize("d,k,rho", [(22, 6, 6), (40, 7, 8), (64, 32, 2), (768, 384, 2), (256, 16, 16)])
+def test_dense_operand_image_matches_oracle_frame(d, k, rho):
+    """framefb_frame_dense_pack against the oracle's dense frame: the bf16
+    hi + lo analysis operand (rows = columns of Phi) carries Phi to 2^-16
+    relative, the synthesis operand (rows = rows of Phi) is Phi rounded to
+    tf32, and padding is zero."""
+    f = ffb.Frame(d, k, rho)
+    P = frames.real_frame(d, k, rho, parseval=True)
+    K = k * rho
+    img = f.dense_image()
+    dp, cp = -(-d // 8) * 8, -(-K // 4) * 4
+    an = -(-(K * dp * 2) // 1024) * 1024
+    assert img.size == 2 * an + -(-(d * cp * 4) // 1024) * 1024
+
+    def bf16(words):
+        return (np.asarray(words, np.uint32) << 16).view(np.float32).astype(np.float64)
+    hi = bf16(img[:K * dp * 2].view(np.uint16)).reshape(K, dp)
+    lo = bf16(img[an:an + K * dp * 2].view(np.uint16)).reshape(K, dp)
+    sy = img[2 * an:2 * an + d * cp * 4].view(np.float32).astype(np.float64).reshape(d, cp)
+    amax = np.abs(P).max()
+    assert np.max(np.abs(hi[:, :d] + lo[:, :d] - P.T)) <= 2.0 ** -16 * amax
+    assert np.max(np.abs(hi[:, :d] - P.T)) <= 2.0 ** -8 * amax             # hi is the bf16 rounding
+    assert np.max(np.abs(sy[:, :K] - P)) <= 2.0 ** -11 * amax                # tf32 rounding
+    assert not hi[:, d:].any() and not lo[:, d:].any() and not sy[:, K:].any()
+    bits = img[2 * an:2 * an + d * cp * 4].view(np.uint32)
+    assert np.all(bits & 0x1FFF == 0)                                        # 10-bit mantissas
