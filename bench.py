@@ -54,6 +54,7 @@ def parse():
     p.add_argument("--cpu-mats", type=int, default=4, help="matrices in the CPU oracle baseline sample")
     p.add_argument("--mats", type=int, default=None, help="first MATS matrices only (small profiling cases)")
     p.add_argument("--tokens", type=int, default=None, help="tokens per matrix (small profiling cases)")
+    p.add_argument("--merge-only", action="store_true", help="time only the 64-tenant ViT-B/16 merge")
     return p.parse_args()
 
 
@@ -543,6 +544,12 @@ def main():
     build()
     from paper_2608_26430_gb300 import framefb as ffb
     from paper_2608_26430_gb300.batch import AdapterBatch
+
+    if args.merge_only:
+        rec = time_merge(dev, torch.cuda.current_stream(), args.steps, args.warmup, L2Flush(dev))
+        if rank == 0:
+            print(json.dumps({"merge": rec}), flush=True)
+        return
 
     ops = ffb.OP_FORWARD | ffb.OP_BACKWARD_DX | ffb.OP_GRAD_COEFF
     timeouts0 = ffb.framefb_wait_timeouts()
