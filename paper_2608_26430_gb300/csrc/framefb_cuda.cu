@@ -595,15 +595,29 @@ framefb_status structured_names(const framefb_mat* mats, int32_t nmats, int32_t 
 }
 
 
-// Matrices of a call split by path: plans cut for the structured kernels
-// and plans of the dense path, each in call order.
-framefb_status split_paths(const framefb_mat* mats, int32_t nmats, std::vector<framefb_mat>& grp,
+// The fused tcgen05 kernels take the plan: register-resident chunks and
+// group counts a multiple of 8, at most 256 per side.
+bool fused_tc_ok(const FfbPlanHeader& h) {
+  return h.EZ <= ffb::kEreg && h.EG <= ffb::kEreg && h.Gn % 8 == 0 && h.Gm % 8 == 0 &&
+         h.Gn <= 128 * ffb::kTcMaxTiles && h.Gm <= 128 * ffb::kTcMaxTiles;
+}
+
+// Matrices of a call split by path, each in call order: the fused kernels
+// (structured plans they take, fp32, or rows with padding), and the
+// contraction path of framefb_dense.cu (dense-layout plans, and bf16
+// structured plans the fused tcgen05 kernels do not take, with unpadded
+// rows).  FRAMEFB_KERNEL=tile keeps every structured plan on the warp-MMA
+// kernel.
+framefb_status split_paths(const framefb_mat* mats, int32_t nmats, framefb_dtype dt, std::vector<framefb_mat>& grp,
                            std::vector<framefb_mat>& den) {
   try {
     for (int32_t j = 0; j < nmats; ++j) {
-      const FfbPlanHeader* h = plan_header(mats[j].plan);
+      const framefb_mat& M = mats[j];
+      const FfbPlanHeader* h = plan_header(M.plan);
       if (!h) return FRAMEFB_EINVAL;
-      (h->layout == FFB_LAYOUT_DENSE ? den : grp).push_back(mats[j]);
+      const bool split = h->layout == FFB_LAYOUT_GROUPS && dt == FRAMEFB_BF16 && tc_allowed() && !fused_tc_ok(*h) &&
+                         M.ldx == M.n && M.ldy == M.m;
+      (h->layout == FFB_LAYOUT_DENSE || split ? den : grp).push_back(M);
     }
   } catch (const std::bad_alloc&) {
     return FRAMEFB_ENOMEM;
@@ -615,13 +629,18 @@ framefb_status split_paths(const framefb_mat* mats, int32_t nmats, std::vector<f
 
 extern "C" size_t framefb_workspace_size(const framefb_mat* mats, int32_t nmats, int32_t ops) {
   if (!mats || nmats <= 0 || !ops_ok(ops)) return 0;
-  std::vector<framefb_mat> grp, den;
-  if (split_paths(mats, nmats, grp, den) != FRAMEFB_OK) return 0;
-  size_t dneed = 0;
-  if (!den.empty() && ffb_host::dense_check(den.data(), static_cast<int32_t>(den.size()), ops, FRAMEFB_BF16, &dneed) !=
-                          FRAMEFB_OK)
-    return 0;
-  return std::max(structured_workspace(grp.data(), static_cast<int32_t>(grp.size()), ops), dneed);
+  // the routing depends on the dtype: the larger need of the two
+  size_t need = 0;
+  for (const framefb_dtype dt : {FRAMEFB_BF16, FRAMEFB_F32}) {
+    std::vector<framefb_mat> grp, den;
+    if (split_paths(mats, nmats, dt, grp, den) != FRAMEFB_OK) return 0;
+    size_t dneed = 0;
+    if (!den.empty() &&
+        ffb_host::dense_check(den.data(), static_cast<int32_t>(den.size()), ops, dt, &dneed) != FRAMEFB_OK)
+      continue;
+    need = std::max({need, structured_workspace(grp.data(), static_cast<int32_t>(grp.size()), ops), dneed});
+  }
+  return need;
 }
 
 extern "C" framefb_status framefb_run(const framefb_mat* mats, int32_t nmats, int32_t ops, framefb_dtype dtype,
@@ -631,7 +650,7 @@ extern "C" framefb_status framefb_run(const framefb_mat* mats, int32_t nmats, in
   if (nmats == 0) return FRAMEFB_OK;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   std::vector<framefb_mat> grp, den;
-  framefb_status s = split_paths(mats, nmats, grp, den);
+  framefb_status s = split_paths(mats, nmats, dtype, grp, den);
   if (s != FRAMEFB_OK) return s;
   // validate everything before queueing anything; the two paths run one
   // after the other on the stream and share the workspace
@@ -657,7 +676,7 @@ extern "C" framefb_status framefb_kernel_names(const framefb_mat* mats, int32_t 
   if (nmats < 0 || (nmats > 0 && !mats) || !ops_ok(ops)) return FRAMEFB_EINVAL;
   if (dtype != FRAMEFB_F32 && dtype != FRAMEFB_BF16) return FRAMEFB_EINVAL;
   std::vector<framefb_mat> grp, den;
-  framefb_status s = split_paths(mats, nmats, grp, den);
+  framefb_status s = split_paths(mats, nmats, dtype, grp, den);
   if (s != FRAMEFB_OK) return s;
   std::vector<std::string> names;
   s = structured_names(grp.data(), static_cast<int32_t>(grp.size()), ops, dtype, names);
@@ -666,9 +685,7 @@ extern "C" framefb_status framefb_kernel_names(const framefb_mat* mats, int32_t 
     size_t need = 0;
     s = ffb_host::dense_check(den.data(), static_cast<int32_t>(den.size()), ops, dtype, &need);
     if (s != FRAMEFB_OK) return s;
-    bool any_tokens = false;
-    for (const framefb_mat& M : den) any_tokens = any_tokens || M.N > 0;
-    if (any_tokens) ffb_host::dense_kernel_names(ops, names);
+    ffb_host::dense_kernel_names(den.data(), static_cast<int32_t>(den.size()), ops, names);
   }
   std::string out;
   for (const std::string& k : names) out += (out.empty() ? "" : ",") + k;

@@ -283,8 +283,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1) dense_gemm_kernel(const __gri
       tc_fence_after();
       const uint32_t taddr = tmem + (static_cast<uint32_t>(32 * q) << 16) + buf * BN;
       const int r = mt * kBM + row;
+      const int cend = min(BN, P.N - nt * BN);  // columns of this tile inside the output
 #pragma unroll 1
-      for (int c0 = 0; c0 < BN; c0 += 32) {
+      for (int c0 = 0; c0 < cend; c0 += 32) {
         float v[32];
         tmem_ld32(taddr + c0, v);
         epilogue32<EPI>(P, r, nt * BN + c0, v);
@@ -310,19 +311,21 @@ __global__ void __launch_bounds__(kGemmThreads, 1) dense_gemm_kernel(const __gri
 // plan column p of the row path (run sums of c V[b] into RZ) and of the
 // column path (c U[a] into RG, U[a] . V[b] into its dC accumulators), the
 // fix-up list adds the pieces of runs split between columns, and the rows
-// of Z = V C^T and G = U C are written over the rows of V and U they came
-// from (the unit read them first), rounded to tf32 for the synthesis.
+// of Z = V C^T and G = U C are written out rounded to tf32 for the
+// synthesis.
 // MODE bits: 1 row path (Z), 2 column path (G), 4 dC.
 // ---------------------------------------------------------------------------
 constexpr int kSpmmThreads = 256;  // = plan columns (FRAMEFB_THREADS)
 
 struct SpmmLaunch {
-  const uint8_t* plan;  // device plan image (FFB_LAYOUT_DENSE)
+  const uint8_t* plan;  // device plan image (either layout: the tables index V / U / Z / G rows)
   const float* c_val;   // [nnz]
-  float* VZ;            // [N][ld]: V in, Z out
-  float* UG;            // [N][ld]: U in, G out
+  const float* V;       // [N][ldv] analysis of X (K_n columns)
+  const float* U;       // [N][ldu] analysis of dY (K_m columns)
+  float* Z;             // [N][ldz] row sums for Y (K_m columns)
+  float* G;             // [N][ldg] column sums for dX (K_n columns)
   float* partial;       // dC partial sums: slot (slot0 + CTA) of stride floats
-  int64_t ld;           // floats per row (multiple of 4)
+  int64_t ldv, ldu, ldz, ldg;  // floats per row (multiples of 4)
   int32_t N;            // tokens of the chunk
   int32_t stride, slot0;
   // shared-memory map (floats): V, U, RZ, RG token-minor regions, dC accumulators
@@ -431,8 +434,8 @@ __global__ void __launch_bounds__(kSpmmThreads) dense_spmm_kernel(const __grid_c
     const int64_t t0 = u * TT;
     const int tc = static_cast<int>(min(static_cast<int64_t>(TT), a.N - t0));
     __syncthreads();  // the previous unit's rows are written out
-    if constexpr (F || C) stage_rows<TT>(V, a.VZ, a.ld, t0, tc, h.n);
-    if constexpr (D || C) stage_rows<TT>(U, a.UG, a.ld, t0, tc, h.m);
+    if constexpr (F || C) stage_rows<TT>(V, a.V, a.ldv, t0, tc, h.n);
+    if constexpr (D || C) stage_rows<TT>(U, a.U, a.ldu, t0, tc, h.m);
     __syncthreads();
     if constexpr (F) {  // row path: Z[a] = sum over the run of c V[b]
       TokVec<TT> acc{};
@@ -490,8 +493,8 @@ __global__ void __launch_bounds__(kSpmmThreads) dense_spmm_kernel(const __grid_c
         }
       }
       __syncthreads();
-      if constexpr (F) write_rows<TT>(a.VZ, RZ, a.ld, t0, tc, h.m);
-      if constexpr (D) write_rows<TT>(a.UG, RG, a.ld, t0, tc, h.n);
+      if constexpr (F) write_rows<TT>(a.Z, RZ, a.ldz, t0, tc, h.m);
+      if constexpr (D) write_rows<TT>(a.G, RG, a.ldg, t0, tc, h.n);
     }
   }
   if constexpr (C) {
@@ -501,6 +504,30 @@ __global__ void __launch_bounds__(kSpmmThreads) dense_spmm_kernel(const __grid_c
       if (qi >= 0) dst[qi] = DC[e * kSpmmThreads + p];
     }
   }
+}
+
+// Operands of the 32 x 32 group block D of a k = 16, k*rho = d frame (every
+// group of coordinates [32r, 32r + 32) carries the same block, Sec. 3.2
+// construction): D[w][x] = Phi[w][column of x], x = 2i + s <-> column
+// i*rho + s, read from the frame's fp32 CSC values (32 per column).
+//   out_hi / out_lo [x][w] bf16:  analysis B (rows = coefficients)
+//   out_sy          [w][x] fp32:  synthesis B (rows = coordinates), tf32
+// One CTA of 1024 threads per frame (blockIdx.x), one entry per thread.
+struct GroupBlockArgs {
+  const float* val[8];
+  int32_t rho[8];
+  uint8_t* out[8];  // 2 KB hi, 2 KB lo, 4 KB sy
+};
+
+__global__ void __launch_bounds__(1024) group_block_kernel(const __grid_constant__ GroupBlockArgs a) {
+  const int f = blockIdx.x, w = threadIdx.x >> 5, x = threadIdx.x & 31;
+  const float v = __ldg(a.val[f] + 32 * ((x >> 1) * a.rho[f] + (x & 1)) + w);
+  const __nv_bfloat16 hi = __float2bfloat16_rn(v);
+  const __nv_bfloat16 lo = __float2bfloat16_rn(v - __bfloat162float(hi));
+  __nv_bfloat16* bh = reinterpret_cast<__nv_bfloat16*>(a.out[f]);
+  bh[32 * x + w] = hi;
+  bh[1024 + 32 * x + w] = lo;
+  reinterpret_cast<float*>(a.out[f] + 4096)[32 * w + x] = __uint_as_float(to_tf32(v));
 }
 
 // dC_q = alpha * sum over partial slots [0, nslots) in slot order.

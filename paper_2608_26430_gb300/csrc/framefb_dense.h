@@ -28,7 +28,7 @@ framefb_status dense_run(const framefb_mat* mats, int32_t nmats, int32_t ops, fr
                          size_t ws_bytes, cudaStream_t st);
 
 // Kernels dense_run launches for `ops` (appended to `out`, no duplicates).
-void dense_kernel_names(int32_t ops, std::vector<std::string>& out);
+void dense_kernel_names(const framefb_mat* mats, int32_t nmats, int32_t ops, std::vector<std::string>& out);
 
 // Bounded waits of the dense kernels that gave up on the current device.
 framefb_status dense_wait_timeouts(uint32_t* count);

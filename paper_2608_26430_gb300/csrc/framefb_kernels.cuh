@@ -796,9 +796,10 @@ struct MergeIO<float> {
 };
 
 constexpr int kMergeThreads = 256;
+constexpr int kMergeStage = 2048;  // entries of one out-group row staged in shared memory
 
 template <typename Elem>
-__global__ void __launch_bounds__(kMergeThreads) merge_kernel(const __grid_constant__ MergeK a) {
+__global__ void __launch_bounds__(kMergeThreads, 2) merge_kernel(const __grid_constant__ MergeK a) {
   using IO = MergeIO<Elem>;
   constexpr int PER = IO::kPer;             // elements per lane chunk
   constexpr int CPR = 32 / PER;             // chunks per 32-element block row
@@ -806,12 +807,13 @@ __global__ void __launch_bounds__(kMergeThreads) merge_kernel(const __grid_const
   constexpr int PASSES = 32 / RPP;          // passes over the block's 32 rows
   __shared__ float DoutT[32][33];           // [a][i] = Dout[i][a]
   __shared__ __align__(16) float DinT[32][32];  // [b][j] = Din[j][b]
+  __shared__ int32_t ent_s[kMergeStage];    // a_local | b_local << 8 of the row's entries
+  __shared__ float cv_s[kMergeStage];       // the tenant's value of each
   for (int idx = threadIdx.x; idx < 1024; idx += blockDim.x) {
     const int w = idx & 31, x = idx >> 5, i = x >> 1, s = x & 1;  // column x = 2i + s of the group block, row w
     DoutT[x][w] = 4.f * __ldg(a.fout_val + 32 * (i * a.rho_out + s) + w);
     DinT[x][w] = 4.f * __ldg(a.fin_val + 32 * (i * a.rho_in + s) + w);
   }
-  __syncthreads();
   const FfbPlanHeader& h = hdr(a.plan);
   const int32_t* blkptr = table<int32_t>(a.plan, h.off_blkptr);
   const int2* blkent = table<int2>(a.plan, h.off_blkent);
@@ -824,7 +826,26 @@ __global__ void __launch_bounds__(kMergeThreads) merge_kernel(const __grid_const
     const int64_t t = it / h.Gm;
     const float* cv = a.c_vals + t * a.nnz;
     Elem* Wt = static_cast<Elem*>(a.Wout) + t * static_cast<int64_t>(a.m) * a.ldw;
+    // the entries of out-group g (blocks (g, 0 .. Gn-1) are contiguous in the
+    // plan) and the tenant's values, staged with one cooperative load
+    const int eg0 = __ldg(blkptr + g * h.Gn), eg1 = __ldg(blkptr + (g + 1) * h.Gn);
+    const bool staged = eg1 - eg0 <= kMergeStage;
+    __syncthreads();  // the previous item is done with the stage
+    if (staged) {
+      for (int e = threadIdx.x; e < eg1 - eg0; e += kMergeThreads) {
+        const int2 en = __ldg(blkent + eg0 + e);
+        ent_s[e] = en.x;
+        cv_s[e] = __ldg(cv + en.y);
+      }
+    }
+    __syncthreads();
     for (int hb = warp; hb < h.Gn; hb += kMergeThreads / 32) {
+      // W0 chunks first: their latency overlaps the entry loop
+      uint4 w0[PASSES];
+#pragma unroll
+      for (int r = 0; r < PASSES; ++r)
+        w0[r] = __ldg(reinterpret_cast<const uint4*>(W0 + static_cast<int64_t>(32 * g + r * RPP + rl) * a.ldw +
+                                                     32 * hb + cl * PER));
       float acc[PASSES][PER];
 #pragma unroll
       for (int r = 0; r < PASSES; ++r)
@@ -832,9 +853,17 @@ __global__ void __launch_bounds__(kMergeThreads) merge_kernel(const __grid_const
         for (int j = 0; j < PER; ++j) acc[r][j] = 0.f;
       const int e0 = __ldg(blkptr + g * h.Gn + hb), e1 = __ldg(blkptr + g * h.Gn + hb + 1);
       for (int e = e0; e < e1; ++e) {
-        const int2 en = __ldg(blkent + e);
-        const int al = en.x & 31, bl = (en.x >> 8) & 31;
-        const float c = __ldg(cv + en.y);
+        int ex;
+        float c;
+        if (staged) {
+          ex = ent_s[e - eg0];
+          c = cv_s[e - eg0];
+        } else {
+          const int2 en = __ldg(blkent + e);
+          ex = en.x;
+          c = __ldg(cv + en.y);
+        }
+        const int al = ex & 31, bl = (ex >> 8) & 31;
         float din[PER];
 #pragma unroll
         for (int j = 0; j < PER; j += 4) {
@@ -855,7 +884,7 @@ __global__ void __launch_bounds__(kMergeThreads) merge_kernel(const __grid_const
       for (int r = 0; r < PASSES; ++r) {
         const int64_t off = static_cast<int64_t>(32 * g + r * RPP + rl) * a.ldw + 32 * hb + cl * PER;
         float w[PER];
-        IO::unpack(__ldg(reinterpret_cast<const uint4*>(W0 + off)), w);
+        IO::unpack(w0[r], w);
 #pragma unroll
         for (int j = 0; j < PER; ++j) w[j] = fmaf(a.seff, acc[r][j], w[j]);
         *reinterpret_cast<uint4*>(Wt + off) = IO::pack(w);

@@ -119,7 +119,8 @@ def test_blockdiag_and_per_layer_supports(wname, kernel, monkeypatch):
 
 
 def test_llama3_zipf_nonsquare():
-    # nnz = 8192 exceeds the register-resident chunk: exercises the streamed-plan path
+    # nnz = 8192 exceeds the register-resident chunk of the fused kernels:
+    # the split contraction path (X and dY shared by the layer's matrices)
     w = wl.WORKLOADS["llama3_8b_all"]
     b = AdapterBatch(w, DEV, N=9, indices=list(range(7)), alias_inputs=True, ops=ALL)
     run(b, ALL)
@@ -356,3 +357,55 @@ def test_merge_many_tenants_grid_stride():
     W0, got, ref = _merge_case("single_256_fp32_many")
     for t in (0, 1, 77, got.shape[0] - 1):
         assert_f32(got[t] - W0, ref[t] - W0, what=f"dW[{t}]")
+
+
+# ---------------------------------------------------------------------------
+# plans the fused tcgen05 kernels do not take: the split contraction path
+# ---------------------------------------------------------------------------
+def test_llama3_shapes_take_the_split_path():
+    """LLaMA-3 shapes (Zipf support with 32 entries per plan column, d up to
+    14336 = 448 groups) run as grouped K = 32 contractions around the SpMM;
+    with FRAMEFB_KERNEL=tile the same call runs on the warp-MMA kernel, and
+    both agree with the oracle."""
+    w = wl.WORKLOADS["llama3_8b_all"]
+    b = AdapterBatch(w, DEV, N=45, indices=list(range(7)), ops=ALL)
+    names = ffb.framefb_kernel_names(b.mats, ALL, b.dtype_code)
+    assert "dense_gemm_kernel<bf16_hilo><grouped>" in names and "mma_tile_kernel<7>" not in names
+    run(b, ALL)
+    check_batch(b, ALL)
+
+
+def test_llama3_shapes_on_the_warp_mma_kernel(monkeypatch):
+    monkeypatch.setenv("FRAMEFB_KERNEL", "tile")
+    w = wl.WORKLOADS["llama3_8b_all"]
+    b = AdapterBatch(w, DEV, N=21, indices=[1, 4, 6], ops=ALL)
+    assert ffb.framefb_kernel_names(b.mats, ALL, b.dtype_code) == ["mma_tile_kernel<7>"]
+    run(b, ALL)
+    check_batch(b, ALL)
+
+
+def test_padded_rows_keep_large_plans_on_the_warp_mma_kernel():
+    """The split path views rows as [tokens * groups][32]: padded rows (a
+    leading dimension above the features) stay on the fused warp-MMA kernel."""
+    w = wl.WORKLOADS["llama3_8b_all"]
+    N, pad = 17, 64
+    src = AdapterBatch(w, DEV, N=N, indices=[1], ops=ALL)   # k: 4096 -> 1024
+    bb = src.bufs[0]
+    n, m = bb.spec.n, bb.spec.m
+    Xp = torch.zeros(N, n + pad, device=DEV, dtype=torch.bfloat16)
+    Xp[:, :n] = bb.X
+    dYp = torch.zeros(N, m + pad, device=DEV, dtype=torch.bfloat16)
+    dYp[:, :m] = bb.dY
+    Yp = torch.zeros(N, m + pad, device=DEV, dtype=torch.bfloat16)
+    dXp = torch.zeros(N, n + pad, device=DEV, dtype=torch.bfloat16)
+    dC = torch.zeros(w.nnz, device=DEV)
+    key = src.keys[0]
+    mat = ffb.make_mat(src.dev_frames[n], src.dev_frames[m], src.plans[key], src.plan_dev[key], bb.c_val, bb.scale, N,
+                       X=Xp, dX=dXp, dY=dYp, Y=Yp, dC=dC, ldx=n + pad, ldy=m + pad)
+    assert ffb.framefb_kernel_names([mat], ALL, ffb.FRAMEFB_BF16) == ["mma_tile_kernel<7>"]
+    ffb.framefb_run([mat], ALL, ffb.FRAMEFB_BF16, ffb.workspace([mat], ALL, DEV))
+    torch.cuda.synchronize()
+    e = Expect(src, 0)
+    assert_bf16(host64(Yp[:, :m]), e.y(host64(bb.X), np.zeros((N, m))), what="Y padded")
+    assert_bf16(host64(dXp[:, :n]), e.dx(host64(bb.dY), np.zeros((N, n))), what="dX padded")
+    assert_bf16(host64(dC), e.dc(host64(bb.X), host64(bb.dY)), what="dC padded")
