@@ -759,8 +759,11 @@ extern "C" framefb_status framefb_merge(const void* W0, framefb_dtype dtype, int
   if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
       cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, ffb::kMergeThreads, 0) != cudaSuccess)
     return FRAMEFB_ECUDA;
-  const int64_t items = static_cast<int64_t>(h->Gm) * T;
-  const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(items, static_cast<int64_t>(sms) * std::max(per_sm, 1)));
+  // one warp per (out group, tenant, run of blocks) item
+  const int64_t items =
+      static_cast<int64_t>(h->Gm) * T * ((h->Gn + ffb::kMergeBlocks - 1) / ffb::kMergeBlocks);
+  const int64_t grid = std::max<int64_t>(
+      1, std::min<int64_t>((items + ffb::kMergeWarps - 1) / ffb::kMergeWarps, static_cast<int64_t>(sms) * std::max(per_sm, 1)));
   if (cudaLaunchKernel(fn, dim3(static_cast<unsigned>(grid)), dim3(ffb::kMergeThreads), kargs, 0,
                        static_cast<cudaStream_t>(stream)) != cudaSuccess)
     return FRAMEFB_ECUDA;

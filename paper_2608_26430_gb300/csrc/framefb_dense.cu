@@ -91,7 +91,7 @@ SpmmPass spmm_pass(const FfbPlanHeader& h, int mode, int TT) {
   s.oU = take((D || C) ? rup(h.m, 4) * TT : 0);
   s.oRZ = take(F ? rup(h.m + h.ovfZ, 4) * TT : 0);
   s.oRG = take(D ? rup(h.n + h.ovfG, 4) * TT : 0);
-  s.oDC = take(C ? static_cast<int64_t>(h.EG) * fd::kSpmmThreads : 0);
+  s.oDC = take(0);  // the dC sums live in registers
   const size_t bytes = static_cast<size_t>(off) * 4;
   s.smem = bytes <= static_cast<size_t>(kSmemOptin) ? std::max<size_t>(bytes, 16) : 0;
   return s;
@@ -116,6 +116,13 @@ std::vector<SpmmPass> spmm_passes(const FfbPlanHeader& h, int32_t ops) {
     out.push_back(best);
   }
   return out;
+}
+
+// Register chunk length of the SpMM for a plan (0: more entries per column
+// than the kernels hold).
+int spmm_e(const FfbPlanHeader& h) {
+  const int e = std::max(h.EZ, h.EG);
+  return e <= 8 ? 8 : e <= 16 ? 16 : e <= 32 ? 32 : 0;
 }
 
 // Geometry of one matrix.  Workspace of a call: the group block operands of
@@ -145,11 +152,12 @@ framefb_status geom_of(const framefb_mat& M, int32_t ops, int sms, Geom& g) {
   g.ldv = g.grouped ? h.n : rup(h.n, 4);
   g.ldu = g.grouped ? h.m : rup(h.m, 4);
   g.passes = spmm_passes(h, ops);
-  if (g.passes.empty()) return FRAMEFB_EUNSUPPORTED;
+  if (g.passes.empty() || spmm_e(h) == 0) return FRAMEFB_EUNSUPPORTED;  // at most 32 entries per plan column
   int tt = 2;
   for (const SpmmPass& p : g.passes) tt = std::min(tt, p.TT);
   const int64_t units = (g.Nc + tt - 1) / tt;
-  g.grid = static_cast<int32_t>(std::max<int64_t>(1, std::min<int64_t>(units, static_cast<int64_t>(sms) * 2)));
+  // one CTA per SM: each CTA loads its plan chunk into registers once
+  g.grid = static_cast<int32_t>(std::max<int64_t>(1, std::min<int64_t>(units, sms)));
   g.stride = (h.nnz + 63) & ~63;
   const size_t rv = rup(static_cast<size_t>(g.Nc) * g.ldv * 4, 256), ru = rup(static_cast<size_t>(g.Nc) * g.ldu * 4, 256);
   g.off_u = rv;
@@ -229,22 +237,29 @@ bool encode_2d(CUtensorMap* map, CUtensorMapDataType type, int esz, const void* 
          CUDA_SUCCESS;
 }
 
-void* spmm_kernel_ptr(int mode, int TT) {
-#define FFB_SPMM(M)                                                                       \
-  case M:                                                                                 \
-    return TT == 2 ? reinterpret_cast<void*>(fd::dense_spmm_kernel<M, 2>)                 \
-                   : reinterpret_cast<void*>(fd::dense_spmm_kernel<M, 1>);
-  switch (mode) {
+void* spmm_kernel_ptr(int mode, int TT, int E) {
+#define FFB_SPMM_E(M, T)                                                   \
+  return E == 8    ? reinterpret_cast<void*>(fd::dense_spmm_kernel<M, T, 8>)  \
+         : E == 16 ? reinterpret_cast<void*>(fd::dense_spmm_kernel<M, T, 16>) \
+                   : reinterpret_cast<void*>(fd::dense_spmm_kernel<M, T, 32>);
+#define FFB_SPMM(M)         \
+  case M:                   \
+    if (TT == 2) {          \
+      FFB_SPMM_E(M, 2)      \
+    } else {                \
+      FFB_SPMM_E(M, 1)      \
+    }
+  if (E != 8 && E != 16 && E != 32) return nullptr;
+  switch (mode) {  // single passes take ops & 7; split passes the column part (& 6) and the row part (1)
     FFB_SPMM(1)
     FFB_SPMM(2)
-    FFB_SPMM(3)
     FFB_SPMM(4)
-    FFB_SPMM(5)
     FFB_SPMM(6)
     FFB_SPMM(7)
     default: return nullptr;
   }
 #undef FFB_SPMM
+#undef FFB_SPMM_E
 }
 
 struct GemmKind {
@@ -437,7 +452,7 @@ framefb_status dense_run(const framefb_mat* mats, int32_t nmats, int32_t ops, fr
         a.oDC = p.oDC;
         const int64_t units = (Nc + p.TT - 1) / p.TT;
         const int grid = static_cast<int>(std::min<int64_t>(units, g.grid));
-        void* fn = spmm_kernel_ptr(p.mode, p.TT);
+        void* fn = spmm_kernel_ptr(p.mode, p.TT, spmm_e(h));
         if (!fn ||
             cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(p.smem)) !=
                 cudaSuccess)

@@ -402,8 +402,12 @@ __device__ __forceinline__ void write_rows(float* dst, const float* src, int64_t
   }
 }
 
-template <int MODE, int TT>
-__global__ void __launch_bounds__(kSpmmThreads) dense_spmm_kernel(const __grid_constant__ SpmmLaunch a) {
+// E: entries per plan column held in registers (the plan's EZ and EG are at
+// most E): the entry words and the coefficient values are loaded once per
+// CTA, so that the loop over a unit's entries only gathers from shared
+// memory; the dC sums live in registers as well.
+template <int MODE, int TT, int E>
+__global__ void __launch_bounds__(kSpmmThreads, 1) dense_spmm_kernel(const __grid_constant__ SpmmLaunch a) {
   constexpr bool F = MODE & 1, D = MODE & 2, C = MODE & 4;
   extern __shared__ float4 smem4[];
   float* sm = reinterpret_cast<float*>(smem4);
@@ -422,14 +426,31 @@ __global__ void __launch_bounds__(kSpmmThreads) dense_spmm_kernel(const __grid_c
   float* U = sm + a.oU;
   float* RZ = sm + a.oRZ;
   float* RG = sm + a.oRG;
-  float* DC = sm + a.oDC;
+  // this thread's plan column: padding entries gather slot 0, add 0, store nowhere
+  uint32_t zb[E], ga[E], gb[E];
+  float zc[E], gc[E], dc[E];
+#pragma unroll
+  for (int e = 0; e < E; ++e) {
+    zb[e] = ga[e] = FFB_NO_STORE << 16;
+    gb[e] = 0;
+    zc[e] = gc[e] = dc[e] = 0.f;
+    if (F && e < h.EZ) {
+      zb[e] = static_cast<uint32_t>(__ldg(tzb + e * kSpmmThreads + p)) & ~0x8000u;  // drop the parity bit
+      const int32_t qi = __ldg(tzq + e * kSpmmThreads + p);
+      zc[e] = qi >= 0 ? __ldg(a.c_val + qi) : 0.f;
+    }
+    if ((D || C) && e < h.EG) {
+      ga[e] = static_cast<uint32_t>(__ldg(tga + e * kSpmmThreads + p)) & ~0x8000u;
+      gb[e] = static_cast<uint32_t>(__ldg(tgb + e * kSpmmThreads + p));
+      const int32_t qi = __ldg(tgq + e * kSpmmThreads + p);
+      gc[e] = (D && qi >= 0) ? __ldg(a.c_val + qi) : 0.f;
+    }
+  }
   // run-sum slots that no run writes stay zero for every unit
   if constexpr (F)
     for (int i = p; i < (h.m + h.ovfZ) * TT; i += kSpmmThreads) RZ[i] = 0.f;
   if constexpr (D)
     for (int i = p; i < (h.n + h.ovfG) * TT; i += kSpmmThreads) RG[i] = 0.f;
-  if constexpr (C)
-    for (int e = 0; e < h.EG; ++e) DC[e * kSpmmThreads + p] = 0.f;
   for (int64_t u = u0; u < u1; ++u) {
     const int64_t t0 = u * TT;
     const int tc = static_cast<int>(min(static_cast<int64_t>(TT), a.N - t0));
@@ -439,38 +460,32 @@ __global__ void __launch_bounds__(kSpmmThreads) dense_spmm_kernel(const __grid_c
     __syncthreads();
     if constexpr (F) {  // row path: Z[a] = sum over the run of c V[b]
       TokVec<TT> acc{};
-      for (int e = 0; e < h.EZ; ++e) {
-        const uint32_t w = static_cast<uint32_t>(__ldg(tzb + e * kSpmmThreads + p));
-        const int32_t qi = __ldg(tzq + e * kSpmmThreads + p);
-        const float c = qi >= 0 ? __ldg(a.c_val + qi) : 0.f;
-        const TokVec<TT> x = tv_load<TT>(V, w & 0x7FFFu);
 #pragma unroll
-        for (int k = 0; k < TT; ++k) acc.v[k] = fmaf(c, x.v[k], acc.v[k]);
-        if ((w >> 16) != FFB_NO_STORE) {
-          tv_store<TT>(RZ, w >> 16, acc);
+      for (int e = 0; e < E; ++e) {
+        const TokVec<TT> x = tv_load<TT>(V, zb[e] & 0xFFFFu);
+#pragma unroll
+        for (int k = 0; k < TT; ++k) acc.v[k] = fmaf(zc[e], x.v[k], acc.v[k]);
+        if ((zb[e] >> 16) != FFB_NO_STORE) {
+          tv_store<TT>(RZ, zb[e] >> 16, acc);
           acc = TokVec<TT>{};
         }
       }
     }
     if constexpr (D || C) {  // column path: G[b] = sum over the run of c U[a]; dC += U[a] . V[b]
       TokVec<TT> acc{};
-      for (int e = 0; e < h.EG; ++e) {
-        const uint32_t w = static_cast<uint32_t>(__ldg(tga + e * kSpmmThreads + p));
-        const int32_t qi = __ldg(tgq + e * kSpmmThreads + p);
-        const TokVec<TT> x = tv_load<TT>(U, w & 0x7FFFu);
-        if constexpr (C) {
-          const TokVec<TT> y = tv_load<TT>(V, __ldg(tgb + e * kSpmmThreads + p));
-          float dsum = 0.f;
 #pragma unroll
-          for (int k = 0; k < TT; ++k) dsum = fmaf(x.v[k], y.v[k], dsum);
-          DC[e * kSpmmThreads + p] += dsum;
+      for (int e = 0; e < E; ++e) {
+        const TokVec<TT> x = tv_load<TT>(U, ga[e] & 0xFFFFu);
+        if constexpr (C) {
+          const TokVec<TT> y = tv_load<TT>(V, gb[e]);
+#pragma unroll
+          for (int k = 0; k < TT; ++k) dc[e] = fmaf(x.v[k], y.v[k], dc[e]);
         }
         if constexpr (D) {
-          const float c = qi >= 0 ? __ldg(a.c_val + qi) : 0.f;
 #pragma unroll
-          for (int k = 0; k < TT; ++k) acc.v[k] = fmaf(c, x.v[k], acc.v[k]);
-          if ((w >> 16) != FFB_NO_STORE) {
-            tv_store<TT>(RG, w >> 16, acc);
+          for (int k = 0; k < TT; ++k) acc.v[k] = fmaf(gc[e], x.v[k], acc.v[k]);
+          if ((ga[e] >> 16) != FFB_NO_STORE) {
+            tv_store<TT>(RG, ga[e] >> 16, acc);
             acc = TokVec<TT>{};
           }
         }
@@ -499,9 +514,12 @@ __global__ void __launch_bounds__(kSpmmThreads) dense_spmm_kernel(const __grid_c
   }
   if constexpr (C) {
     float* dst = a.partial + static_cast<int64_t>(a.slot0 + blockIdx.x) * a.stride;
-    for (int e = 0; e < h.EG; ++e) {
-      const int32_t qi = __ldg(tgq + e * kSpmmThreads + p);
-      if (qi >= 0) dst[qi] = DC[e * kSpmmThreads + p];
+#pragma unroll
+    for (int e = 0; e < E; ++e) {
+      if (e < h.EG) {
+        const int32_t qi = __ldg(tgq + e * kSpmmThreads + p);
+        if (qi >= 0) dst[qi] = dc[e];
+      }
     }
   }
 }

@@ -749,14 +749,16 @@ __global__ void __launch_bounds__(256) dc_reduce_kernel(const __grid_constant__ 
 // Merge (Sec. 3.4 "Storage efficiency", Alg. 1 step 6 per tenant):
 //   W_t[32g + i][32h + j] = W0[..] + (s/16) sum_{e in block (g,h)} c_{t,e} Dout[i][a_e] Din[j][b_e],
 // D = 4 x the group-0 block of each frame (k = 16, k*rho = d frames), staged
-// once per CTA.  Work items are (out group g, tenant t), taken grid-stride
-// (any number of tenants); inside an item warp w owns the 32 x 32 blocks
-// h = w, w + 8, ...  A lane owns one 16-byte chunk of one row per row pass:
-// lanes (row l / CPR, chunk l % CPR), CPR = 16-byte chunks per 32-element
-// row (4 bf16, 8 fp32), so a warp's store covers whole 64- or 128-byte row
-// segments.  The block's entries are uniform over the warp: no divergence.
-// Bound: HBM (W_t written once; W0 and the plan are L2-resident across
-// tenants).
+// once per CTA.  Work items are (out group g, tenant t, a run of four 32 x 32
+// blocks h of that row); each warp takes items grid-stride (any number of
+// tenants).  A warp first stages its item's entries (the blocks (g, .) are
+// contiguous in the plan) and the tenant's values in its own slice of
+// shared memory, so no CTA barrier ties the warps together and one warp's
+// staging latency hides behind the others' arithmetic.  A
+// lane owns one 16-byte chunk of one row per row pass: lanes (row l / CPR,
+// chunk l % CPR), CPR = 16-byte chunks per 32-element row (4 bf16, 8 fp32),
+// so a warp's store covers whole 64- or 128-byte row segments.  Bound: HBM
+// (W_t written once; W0 and the plan are L2-resident across tenants).
 // ---------------------------------------------------------------------------
 template <typename Elem>
 struct MergeIO;
@@ -796,7 +798,9 @@ struct MergeIO<float> {
 };
 
 constexpr int kMergeThreads = 256;
-constexpr int kMergeStage = 2048;  // entries of one out-group row staged in shared memory
+constexpr int kMergeWarps = kMergeThreads / 32;
+constexpr int kMergeStage = 512;  // entries of one item a warp stages (longer rows read them from L2)
+constexpr int kMergeBlocks = 4;   // 32 x 32 blocks per work item
 
 template <typename Elem>
 __global__ void __launch_bounds__(kMergeThreads, 2) merge_kernel(const __grid_constant__ MergeK a) {
@@ -807,57 +811,76 @@ __global__ void __launch_bounds__(kMergeThreads, 2) merge_kernel(const __grid_co
   constexpr int PASSES = 32 / RPP;          // passes over the block's 32 rows
   __shared__ float DoutT[32][33];           // [a][i] = Dout[i][a]
   __shared__ __align__(16) float DinT[32][32];  // [b][j] = Din[j][b]
-  __shared__ int32_t ent_s[kMergeStage];    // a_local | b_local << 8 of the row's entries
-  __shared__ float cv_s[kMergeStage];       // the tenant's value of each
+  __shared__ int32_t ent_s[kMergeWarps][kMergeStage];  // a_local | b_local << 8, per warp
+  __shared__ float cv_s[kMergeWarps][kMergeStage];     // the tenant's value of each
+  __shared__ int32_t bp_s[kMergeWarps][kMergeBlocks + 1];  // block boundaries of the item
   for (int idx = threadIdx.x; idx < 1024; idx += blockDim.x) {
     const int w = idx & 31, x = idx >> 5, i = x >> 1, s = x & 1;  // column x = 2i + s of the group block, row w
     DoutT[x][w] = 4.f * __ldg(a.fout_val + 32 * (i * a.rho_out + s) + w);
     DinT[x][w] = 4.f * __ldg(a.fin_val + 32 * (i * a.rho_in + s) + w);
   }
+  __syncthreads();
   const FfbPlanHeader& h = hdr(a.plan);
   const int32_t* blkptr = table<int32_t>(a.plan, h.off_blkptr);
   const int2* blkent = table<int2>(a.plan, h.off_blkent);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int rl = lane / CPR, cl = lane % CPR;  // row in the pass, chunk in the row
+  int32_t* ent = ent_s[warp];
+  float* cvw = cv_s[warp];
+  int32_t* bp = bp_s[warp];
   const Elem* W0 = static_cast<const Elem*>(a.W0);
-  const int64_t items = static_cast<int64_t>(h.Gm) * a.T;
-  for (int64_t it = blockIdx.x; it < items; it += gridDim.x) {
-    const int g = static_cast<int>(it % h.Gm);
-    const int64_t t = it / h.Gm;
+  // work items: (out group g, tenant t, run of kMergeBlocks blocks)
+  const int nsub = (h.Gn + kMergeBlocks - 1) / kMergeBlocks;
+  const int64_t items = static_cast<int64_t>(h.Gm) * nsub * a.T;
+  for (int64_t it = static_cast<int64_t>(blockIdx.x) * kMergeWarps + warp; it < items;
+       it += static_cast<int64_t>(gridDim.x) * kMergeWarps) {
+    const int sub = static_cast<int>(it % nsub);
+    const int g = static_cast<int>((it / nsub) % h.Gm);
+    const int64_t t = it / (static_cast<int64_t>(nsub) * h.Gm);
+    const int hb0 = sub * kMergeBlocks, hb1 = min(h.Gn, hb0 + kMergeBlocks);
     const float* cv = a.c_vals + t * a.nnz;
     Elem* Wt = static_cast<Elem*>(a.Wout) + t * static_cast<int64_t>(a.m) * a.ldw;
-    // the entries of out-group g (blocks (g, 0 .. Gn-1) are contiguous in the
-    // plan) and the tenant's values, staged with one cooperative load
-    const int eg0 = __ldg(blkptr + g * h.Gn), eg1 = __ldg(blkptr + (g + 1) * h.Gn);
+    const int eg0 = __ldg(blkptr + g * h.Gn + hb0), eg1 = __ldg(blkptr + g * h.Gn + hb1);
     const bool staged = eg1 - eg0 <= kMergeStage;
-    __syncthreads();  // the previous item is done with the stage
+    __syncwarp();  // the warp's previous item is done with its slice
     if (staged) {
-      for (int e = threadIdx.x; e < eg1 - eg0; e += kMergeThreads) {
+      for (int e = lane; e < eg1 - eg0; e += 32) {
         const int2 en = __ldg(blkent + eg0 + e);
-        ent_s[e] = en.x;
-        cv_s[e] = __ldg(cv + en.y);
+        ent[e] = en.x;
+        cvw[e] = __ldg(cv + en.y);
       }
+      if (lane <= hb1 - hb0) bp[lane] = __ldg(blkptr + g * h.Gn + hb0 + lane);
     }
-    __syncthreads();
-    for (int hb = warp; hb < h.Gn; hb += kMergeThreads / 32) {
-      // W0 chunks first: their latency overlaps the entry loop
+    __syncwarp();
+    // W0 chunks one block ahead: their latency overlaps the previous block
+    uint4 w0n[PASSES];
+#pragma unroll
+    for (int r = 0; r < PASSES; ++r)
+      w0n[r] = __ldg(reinterpret_cast<const uint4*>(W0 + static_cast<int64_t>(32 * g + r * RPP + rl) * a.ldw +
+                                                    32 * hb0 + cl * PER));
+    for (int hb = hb0; hb < hb1; ++hb) {
       uint4 w0[PASSES];
 #pragma unroll
-      for (int r = 0; r < PASSES; ++r)
-        w0[r] = __ldg(reinterpret_cast<const uint4*>(W0 + static_cast<int64_t>(32 * g + r * RPP + rl) * a.ldw +
-                                                     32 * hb + cl * PER));
+      for (int r = 0; r < PASSES; ++r) w0[r] = w0n[r];
+      if (hb + 1 < hb1) {
+#pragma unroll
+        for (int r = 0; r < PASSES; ++r)
+          w0n[r] = __ldg(reinterpret_cast<const uint4*>(W0 + static_cast<int64_t>(32 * g + r * RPP + rl) * a.ldw +
+                                                        32 * (hb + 1) + cl * PER));
+      }
       float acc[PASSES][PER];
 #pragma unroll
       for (int r = 0; r < PASSES; ++r)
 #pragma unroll
         for (int j = 0; j < PER; ++j) acc[r][j] = 0.f;
-      const int e0 = __ldg(blkptr + g * h.Gn + hb), e1 = __ldg(blkptr + g * h.Gn + hb + 1);
+      const int e0 = staged ? bp[hb - hb0] : __ldg(blkptr + g * h.Gn + hb);
+      const int e1 = staged ? bp[hb - hb0 + 1] : __ldg(blkptr + g * h.Gn + hb + 1);
       for (int e = e0; e < e1; ++e) {
         int ex;
         float c;
         if (staged) {
-          ex = ent_s[e - eg0];
-          c = cv_s[e - eg0];
+          ex = ent[e - eg0];
+          c = cvw[e - eg0];
         } else {
           const int2 en = __ldg(blkent + e);
           ex = en.x;

@@ -49,9 +49,11 @@ def test_static_workspace_matches_caller_workspace_twice():
 
 
 def test_static_workspace_rejects_oversized_calls():
-    # 224 matrices with 8192-entry supports need more than the 8 MiB array
-    w = wl.WORKLOADS["llama3_8b_all"]
-    b = AdapterBatch(w, DEV, N=1, alias_inputs=True, ops=ALL)
+    # rho = 2 frames at 768 over 4096 tokens: the contraction path keeps the
+    # frame coefficients of the tokens in its workspace (about 50 MB), more
+    # than the 8 MiB array
+    w = wl.WORKLOADS["roberta_rho2"]
+    b = AdapterBatch(w, DEV, indices=[0], ops=ALL)
     assert ffb.framefb_workspace_size(b.mats, ALL) > ffb.STATIC_WS_BYTES
     with pytest.raises(ffb.FramefbError) as e:
         ffb.framefb_run_static_ws(b.mats, ALL, b.dtype_code)
