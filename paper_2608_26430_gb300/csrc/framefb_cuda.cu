@@ -17,6 +17,7 @@
 #include "framefb_mma.cuh"
 #include "framefb_tc.cuh"
 #include "framefb_tc2.cuh"
+#include "framefb_tc2p.cuh"
 #include "plan_internal.h"
 #include "plan_layout.h"
 
@@ -59,6 +60,7 @@ struct Prepared {
   bool reg;
   bool tc;    // bf16: pipelined kernel on tcgen05 tensor cores
   bool tc2;   // bf16: the same, two tokens per unit
+  bool pack;  // tc2: some matrix packs several token pairs per unit
   int T;      // tile tokens of the bf16 kernel
   int threads;
 };
@@ -74,15 +76,35 @@ void* tc_kernel_ptr(int mode) {
   }
 }
 
-void* tc2_kernel_ptr(int mode) {
+// two-token kernel, or its packed form (several token pairs per unit)
+void* tc2_kernel_ptr(int mode, bool pack) {
+#define FFB_TC2(M) \
+  case M:          \
+    return pack ? reinterpret_cast<void*>(ffb::tc2p_tile_kernel<M>) : reinterpret_cast<void*>(ffb::tc2_tile_kernel<M>);
   switch (mode) {
-    case 1: return reinterpret_cast<void*>(ffb::tc2_tile_kernel<1>);
-    case 2: return reinterpret_cast<void*>(ffb::tc2_tile_kernel<2>);
-    case 4: return reinterpret_cast<void*>(ffb::tc2_tile_kernel<4>);
-    case 6: return reinterpret_cast<void*>(ffb::tc2_tile_kernel<6>);
-    case 7: return reinterpret_cast<void*>(ffb::tc2_tile_kernel<7>);
+    FFB_TC2(1)
+    FFB_TC2(2)
+    FFB_TC2(4)
+    FFB_TC2(6)
+    FFB_TC2(7)
     default: return nullptr;
   }
+#undef FFB_TC2
+}
+
+// Token pairs per slot of the two-token kernel for a plan: P tokens of a
+// slot share one 128-lane tile (lane p G + g), so P G <= 128 on both sides;
+// at most kTc2MaxPairs; 1 for plans with more entries per chunk than the
+// packed kernel holds in registers.
+constexpr int kTc2MaxPairs = 8;
+int tc2_pairs(const FfbPlanHeader& h) {
+  if (h.EZ > ffb::kEregPack || h.EG > ffb::kEregPack) return 1;
+  const int G = std::max(h.Gn, h.Gm);
+  return std::max(1, std::min(kTc2MaxPairs, 128 / std::max(G, 1)));
+}
+bool pack_allowed() {
+  const char* e = std::getenv("FRAMEFB_PACK");
+  return !(e && std::strcmp(e, "0") == 0);
 }
 
 // bf16 activations: tensor-core kernel with staged rows (tile of T = 1 or 2
@@ -201,35 +223,44 @@ size_t tc_smem_map(const framefb_mat* mats, int32_t nmats, int32_t ops, int S, f
   return mbar + 8 * static_cast<size_t>(S + 1);
 }
 
-// Shared-memory map of the two-token tensor-core kernel: a ring of S stages
-// (two token rows of X, then two of dY, each a swizzled K-major operand of
-// one 128-group tile), B operands (8 KB), one V/U set (float2 per
-// coefficient: both tokens), one RZ/RG set per token in the canonical tf32
-// layout (padded to a whole tile), the fix-up item cache, S + 2 mbarriers.
-// Returns the total bytes, or 0 when a matrix does not fit the shape rules
-// (group counts a multiple of 8 and at most 128).
-size_t tc2_smem_map(const framefb_mat* mats, int32_t nmats, int32_t ops, int S, ffb::TcLaunchK* a) {
+// Shared-memory map of the two-token tensor-core kernel and its packed
+// form: a ring of S stages (two slots of X rows, then two of dY, each a
+// swizzled K-major operand of one 128-lane tile: one token row, or P of them
+// when packed), B operands (8 KB), the V/U sets (float2 per coefficient:
+// both tokens of a pair; unpacked: V over the largest n, then U; packed: one
+// set of n + m per pair), one RZ/RG set per slot in the canonical tf32
+// layout (P canonical blocks padded to a whole tile, then the pairs'
+// overflow slots), the fix-up item cache, S + 2 mbarriers.  P of matrix j is
+// pairs[j] (all 1 unless pack).  Returns the total bytes, or 0 when a matrix
+// does not fit the shape rules (group counts a multiple of 8 and at most
+// 128, P G <= 128).
+size_t tc2_smem_map(const framefb_mat* mats, int32_t nmats, int32_t ops, int S, const int* pairs, bool pack,
+                    ffb::TcLaunchK* a) {
   const bool F = ops & FRAMEFB_OP_FORWARD, D = ops & FRAMEFB_OP_BACKWARD_DX, C = ops & FRAMEFB_OP_GRAD_COEFF;
   const bool needV = F || C, needU = D || C;
-  size_t nfix = 0;
-  int32_t nmax = 0, mmax = 0, ovfZ = 0, ovfG = 0;
+  size_t nfix = 0, vuset = 0, szRZ = 0, szRG = 0;
+  int32_t nmax = 0, mmax = 0;
   for (int32_t j = 0; j < nmats; ++j) {
     const FfbPlanHeader* h = plan_header(mats[j].plan);
+    const size_t P = static_cast<size_t>(pairs[j]);
     if (h->Gn % 8 || h->Gm % 8 || h->Gn > 128 || h->Gm > 128) return 0;
+    if (P < 1 || (!pack && P != 1) || P * h->Gn > 128 || P * h->Gm > 128) return 0;
     nmax = std::max(nmax, h->n);
     mmax = std::max(mmax, h->m);
-    ovfZ = std::max(ovfZ, h->ovfZ);
-    ovfG = std::max(ovfG, h->ovfG);
+    vuset = std::max(vuset, P * static_cast<size_t>(h->n + h->m));
+    if (F) szRZ = std::max(szRZ, P * static_cast<size_t>(h->m + h->ovfZ));
+    if (D) szRG = std::max(szRG, P * static_cast<size_t>(h->n + h->ovfG));
     nfix = std::max<size_t>(nfix, (F ? h->nfixZ : 0) + (D ? h->nfixG : 0));
   }
   const size_t tok_x = needV ? 8192 : 0, tok_u = needU ? 8192 : 0;
   const size_t stage = 2 * tok_x + 2 * tok_u;
   const size_t bops = S * stage;
   const size_t vu = bops + 8192;
-  const size_t oU = needV ? nmax : 0;  // float2 units
-  const size_t rzg = vu + round_up((oU + (needU ? mmax : 0)) * 8, 128);
-  const size_t szRZ = F ? round_up(std::max<size_t>(128 * 32, mmax + ovfZ), 32) : 0;
-  const size_t szRG = D ? round_up(std::max<size_t>(128 * 32, nmax + ovfG), 32) : 0;
+  const size_t oU = pack ? 0 : (needV ? nmax : 0);  // float2 units; packed: per matrix
+  if (!pack) vuset = oU + (needU ? mmax : 0);
+  const size_t rzg = vu + round_up(vuset * 8, 128);
+  szRZ = F ? round_up(std::max<size_t>(128 * 32, szRZ), 32) : 0;
+  szRG = D ? round_up(std::max<size_t>(128 * 32, szRG), 32) : 0;
   const size_t rzg_tok = szRZ + szRG;  // floats
   const size_t fixc = rzg + 2 * rzg_tok * 4;
   const size_t mbar = round_up(fixc + 16 * nfix, 16);
@@ -258,13 +289,14 @@ using ffb_host::EncodeTiledFn;
 
 // Tensor map of the bf16 rows of one activation tensor (d features, N
 // tokens, leading dimension ld elements): {32 coordinates, d / 32 groups, N
-// tokens}, box {32, d / 32, 1}, 64-byte swizzle.
-bool encode_rows(CUtensorMap* map, const void* base, int32_t d, int32_t N, int64_t ld) {
+// tokens}, box {32, d / 32, rows} (rows consecutive tokens, one row per
+// group, token-major), 64-byte swizzle.
+bool encode_rows(CUtensorMap* map, const void* base, int32_t d, int32_t N, int64_t ld, int32_t rows = 1) {
   const EncodeTiledFn fn = encode_tiled();
   if (!fn) return false;
   const cuuint64_t dims[3] = {32, static_cast<cuuint64_t>(d / 32), static_cast<cuuint64_t>(N)};
   const cuuint64_t strides[2] = {64, static_cast<cuuint64_t>(ld) * 2};
-  const cuuint32_t box[3] = {32, static_cast<cuuint32_t>(d / 32), 1};
+  const cuuint32_t box[3] = {32, static_cast<cuuint32_t>(d / 32), static_cast<cuuint32_t>(rows)};
   const cuuint32_t estr[3] = {1, 1, 1};
   return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -273,7 +305,8 @@ bool encode_rows(CUtensorMap* map, const void* base, int32_t d, int32_t N, int64
 
 // Kernel choice for bf16: the two-token tensor-core kernel wherever it
 // applies (register-resident plans, group counts a multiple of 8 and at most
-// 128, its shared-memory map fits), else the one-token tensor-core kernel
+// 128, its shared-memory map fits; packed units where a side has at most 64
+// groups, unless FRAMEFB_PACK=0), else the one-token tensor-core kernel
 // (group counts up to 256), else the one-phase-at-a-time tile kernel.
 // FRAMEFB_KERNEL=tc2, =tc or =tile selects one of them where it applies
 // (for comparison and tests).
@@ -302,21 +335,36 @@ framefb_status prepare(const framefb_mat* mats, int32_t nmats, int32_t ops, fram
   size_t smem = 0;
   int T_mma = 0;
   bool tc = false, tc2 = false;
+  int pairs[ffb::kTcMaxMats];
+  bool pack = false;
   if (dt == FRAMEFB_BF16 && reg && tc2_allowed() && nmats <= ffb::kTcMaxMats && encode_tiled()) {
-    // two-token tensor-core kernel: two stages
+    // two-token tensor-core kernel: two stages; small dimensions pack
+    // several token pairs per unit
+    for (int32_t j = 0; j < nmats; ++j) {
+      pairs[j] = pack_allowed() ? tc2_pairs(*plan_header(mats[j].plan)) : 1;
+      pack = pack || pairs[j] > 1;
+    }
     int dev = 0, optin = 0;
     cudaFuncAttributes fa{};
     if (cudaGetDevice(&dev) != cudaSuccess ||
         cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess ||
-        cudaFuncGetAttributes(&fa, tc2_kernel_ptr(ops)) != cudaSuccess)
+        cudaFuncGetAttributes(&fa, tc2_kernel_ptr(ops, pack)) != cudaSuccess)
       return FRAMEFB_ECUDA;
-    const size_t budget = static_cast<size_t>(optin) - fa.sharedSizeBytes;
-    const size_t need = tc2_smem_map(mats, nmats, ops, 2, nullptr);
+    size_t budget = static_cast<size_t>(optin) - fa.sharedSizeBytes;
+    size_t need = tc2_smem_map(mats, nmats, ops, 2, pairs, pack, nullptr);
+    if (pack && (need == 0 || need > budget)) {
+      // packed sets do not fit: unpacked units
+      for (int32_t j = 0; j < nmats; ++j) pairs[j] = 1;
+      pack = false;
+      if (cudaFuncGetAttributes(&fa, tc2_kernel_ptr(ops, pack)) != cudaSuccess) return FRAMEFB_ECUDA;
+      budget = static_cast<size_t>(optin) - fa.sharedSizeBytes;
+      need = tc2_smem_map(mats, nmats, ops, 2, pairs, pack, nullptr);
+    }
     if (need > 0 && need <= budget) {
       tc2 = true;
       T_mma = 2;
       std::memset(P.tcargs, 0, sizeof(ffb::TcLaunchK));
-      smem = tc2_smem_map(mats, nmats, ops, 2, P.tcargs);
+      smem = tc2_smem_map(mats, nmats, ops, 2, pairs, pack, P.tcargs);
     }
   }
   if (dt == FRAMEFB_BF16 && reg && !tc2 && tc_allowed() && nmats <= ffb::kTcMaxMats && encode_tiled()) {
@@ -373,7 +421,7 @@ framefb_status prepare(const framefb_mat* mats, int32_t nmats, int32_t ops, fram
     }
     if (C && h->nnz > 0 && !M.dC) return FRAMEFB_EINVAL;
     // tokens per tile: as many as fit in shared memory, at most kTmax
-    int T = T_mma;
+    int T = tc2 ? 2 * pairs[j] : T_mma;
     if (dt != FRAMEFB_BF16) {
       T = kTmax;
       while (T > 1 && ffb_tile_layout(*h, ops, T, C).total * 4 > kSmemBudget) --T;
@@ -423,8 +471,9 @@ framefb_status prepare(const framefb_mat* mats, int32_t nmats, int32_t ops, fram
       A.m[j] = P.args->m[j];
       const framefb_mat& M = mats[j];
       if (M.N == 0) continue;
-      if ((F || C) && !encode_rows(&A.maps[2 * j], M.X, M.n, M.N, M.ldx)) return FRAMEFB_ECUDA;
-      if ((D || C) && !encode_rows(&A.maps[2 * j + 1], M.dY, M.m, M.N, M.ldy)) return FRAMEFB_ECUDA;
+      const int32_t rows = tc2 ? pairs[j] : 1;
+      if ((F || C) && !encode_rows(&A.maps[2 * j], M.X, M.n, M.N, M.ldx, rows)) return FRAMEFB_ECUDA;
+      if ((D || C) && !encode_rows(&A.maps[2 * j + 1], M.dY, M.m, M.N, M.ldy, rows)) return FRAMEFB_ECUDA;
     }
   }
   P.red->nmats = nmats;
@@ -433,13 +482,14 @@ framefb_status prepare(const framefb_mat* mats, int32_t nmats, int32_t ops, fram
   P.reg = reg;
   P.tc = tc;
   P.tc2 = tc2;
+  P.pack = tc2 && pack;
   P.threads = (tc || tc2) ? ffb::kTcThreads : kThreads;
   P.T = T_mma;
   P.smem = std::max<size_t>(smem, 16);
   P.grid = 0;
   P.ws_bytes = 0;
   if (units == 0) return FRAMEFB_OK;
-  void* fn = tc2 ? tc2_kernel_ptr(ops) : tc ? tc_kernel_ptr(ops) : tile_kernel_ptr(dt, ops, reg, T_mma);
+  void* fn = tc2 ? tc2_kernel_ptr(ops, P.pack) : tc ? tc_kernel_ptr(ops) : tile_kernel_ptr(dt, ops, reg, T_mma);
   if (!fn) return FRAMEFB_EINVAL;
   int dev = 0, sms = 0, per_sm = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return FRAMEFB_ECUDA;
@@ -475,9 +525,21 @@ struct Buffers {
 // kTcMaxMats; the chunk is that short only when the kernel applies to it.
 int32_t chunk_len(const framefb_mat* mats, int32_t rest, framefb_dtype dt) {
   if (dt == FRAMEFB_BF16 && tc_allowed()) {
-    // launches of equal size (at most 64 matrices each): no small tail launch
-    const int32_t launches = (rest + ffb::kTcMaxMats - 1) / ffb::kTcMaxMats;
-    const int32_t k = (rest + launches - 1) / launches;
+    // matrices of one pair count only (units of equal cost in a launch; the
+    // caller's order is sorted by it), in launches of equal size (at most 64
+    // matrices each): no small tail launch
+    int32_t run = rest;
+    if (tc2_allowed() && pack_allowed()) {
+      const FfbPlanHeader* h0 = plan_header(mats[0].plan);
+      run = 1;
+      while (h0 && run < rest) {
+        const FfbPlanHeader* h = plan_header(mats[run].plan);
+        if (!h || tc2_pairs(*h) != tc2_pairs(*h0)) break;
+        ++run;
+      }
+    }
+    const int32_t launches = (run + ffb::kTcMaxMats - 1) / ffb::kTcMaxMats;
+    const int32_t k = (run + launches - 1) / launches;
     bool ok = true;
     for (int32_t j = 0; j < k && ok; ++j) {
       const FfbPlanHeader* h = plan_header(mats[j].plan);
@@ -557,7 +619,8 @@ framefb_status structured_run(const framefb_mat* mats, int32_t nmats, int32_t op
     P.args->partial = static_cast<float*>(ws);
     P.tcargs->partial = static_cast<float*>(ws);
     P.red->partial = static_cast<const float*>(ws);
-    void* fn = P.tc2 ? tc2_kernel_ptr(ops) : P.tc ? tc_kernel_ptr(ops) : tile_kernel_ptr(dtype, ops, P.reg, P.T);
+    void* fn =
+        P.tc2 ? tc2_kernel_ptr(ops, P.pack) : P.tc ? tc_kernel_ptr(ops) : tile_kernel_ptr(dtype, ops, P.reg, P.T);
     void* kargs[] = {(P.tc || P.tc2) ? static_cast<void*>(P.tcargs) : static_cast<void*>(P.args)};
     if (cudaLaunchKernel(fn, dim3(P.grid), dim3(P.threads), kargs, P.smem, st) != cudaSuccess)
       return FRAMEFB_ECUDA;
@@ -585,9 +648,10 @@ framefb_status structured_names(const framefb_mat* mats, int32_t nmats, int32_t 
     const framefb_status s = prepare(mats + j0, nm, ops, dtype, P);
     if (s != FRAMEFB_OK) return s;
     if (P.grid == 0) continue;
-    std::string k = P.tc2  ? "tc2_tile_kernel"
-                    : P.tc ? "tc_tile_kernel"
-                           : (dtype == FRAMEFB_BF16 ? "mma_tile_kernel" : "fft_tile_kernel");
+    std::string k = P.pack  ? "tc2p_tile_kernel"
+                    : P.tc2 ? "tc2_tile_kernel"
+                    : P.tc  ? "tc_tile_kernel"
+                            : (dtype == FRAMEFB_BF16 ? "mma_tile_kernel" : "fft_tile_kernel");
     k += "<" + std::to_string(ops) + ">";
     if (std::find(names.begin(), names.end(), k) == names.end()) names.push_back(k);
   }
@@ -619,6 +683,13 @@ framefb_status split_paths(const framefb_mat* mats, int32_t nmats, framefb_dtype
                          M.ldx == M.n && M.ldy == M.m;
       (h->layout == FFB_LAYOUT_DENSE || split ? den : grp).push_back(M);
     }
+    // the two-token kernel's units carry P token pairs of a matrix (P = 1
+    // for large dimensions): matrices of one P launch together, largest P
+    // first (results do not depend on the order of the matrices)
+    if (dt == FRAMEFB_BF16 && tc2_allowed() && pack_allowed())
+      std::stable_sort(grp.begin(), grp.end(), [](const framefb_mat& x, const framefb_mat& y) {
+        return tc2_pairs(*plan_header(x.plan)) > tc2_pairs(*plan_header(y.plan));
+      });
   } catch (const std::bad_alloc&) {
     return FRAMEFB_ENOMEM;
   }

@@ -64,11 +64,12 @@ __host__ __device__ __forceinline__ int32_t tc_slot(int32_t x, int32_t K) {
 
 // dC partial sums of one plan column (held in registers) to the CTA's
 // workspace slot of the matrix.
+template <int KE = kEreg>
 __device__ __forceinline__ void dc_flush(const uint8_t* plan, float* dst, const float (&dc)[kEreg], int col) {
   const FfbPlanHeader& h = hdr(plan);
   const int32_t* gq = table<int32_t>(plan, h.off_gq);
 #pragma unroll
-  for (int e = 0; e < kEreg; ++e) {
+  for (int e = 0; e < KE; ++e) {
     if (e < h.EG) {
       const int32_t q = __ldg(gq + e * kThreads + col);
       if (q >= 0) dst[q] = dc[e];

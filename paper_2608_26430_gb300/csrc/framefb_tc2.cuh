@@ -45,9 +45,9 @@ __device__ __forceinline__ bool spmm_bar_or(bool f) {
   return out != 0;
 }
 
-// Register chunk of plan column `col`: gather slots in the float2 V / U
-// layout, store targets in the canonical RZ / RG layout.
-template <int MODE>
+// Register chunk of plan column `col` (its first KE entries): gather slots
+// in the float2 V / U layout, store targets in the canonical RZ / RG layout.
+template <int MODE, int KE = kEreg>
 __device__ __forceinline__ void tc2_load_chunk(Chunk<MODE, true, false>& ch, const uint8_t* plan, const float* c_val,
                                                int col) {
   constexpr bool F = MODE & MODE_F, D = MODE & MODE_D, C = MODE & MODE_C;
@@ -69,7 +69,7 @@ __device__ __forceinline__ void tc2_load_chunk(Chunk<MODE, true, false>& ch, con
     return slo | (shi << 16);
   };
 #pragma unroll
-  for (int e = 0; e < kEreg; ++e) {
+  for (int e = 0; e < KE; ++e) {
     ch.zb[e] = FFB_NO_STORE << 16;
     ch.ga[e] = FFB_NO_STORE << 16;
     ch.gb[e] = 0;

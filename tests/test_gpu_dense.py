@@ -115,7 +115,7 @@ def test_structured_and_dense_matrices_in_one_call():
     bd = AdapterBatch(wd, DEV, N=64, indices=[0, 1], ops=ALL)
     mats = [bs.mats[0], bd.mats[0], bs.mats[1], bd.mats[1]]
     names = ffb.framefb_kernel_names(mats, ALL, ffb.FRAMEFB_BF16)
-    assert "tc2_tile_kernel<7>" in names and "dense_gemm_kernel<tf32>" in names
+    assert "tc2p_tile_kernel<7>" in names and "dense_gemm_kernel<tf32>" in names
     ws = ffb.workspace(mats, ALL, DEV)
     ffb.framefb_run(mats, ALL, ffb.FRAMEFB_BF16, ws)
     check(bs, ALL)

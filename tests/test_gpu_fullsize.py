@@ -56,7 +56,7 @@ def test_roberta_full_size_every_matrix():
     """24 q/v matrices of 768 x 768 at 4096 tokens: every row of every matrix."""
     w = wl.WORKLOADS["roberta_base_qv"]
     b = AdapterBatch(w, DEV, ops=ALL)
-    assert ffb.framefb_kernel_names(b.mats, ALL, b.dtype_code) == ["tc2_tile_kernel<7>"]
+    assert ffb.framefb_kernel_names(b.mats, ALL, b.dtype_code) == ["tc2p_tile_kernel<7>"]
     run_full(b)
     check_sampled(b, range(len(b.bufs)), np.arange(w.N))
 
