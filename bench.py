@@ -439,8 +439,10 @@ def time_merge(dev, stream, steps, warmup, flush):
 
 def serving_timing(dev, stream, reps: int = 10):
     """Forward-only ViT-B/16 step (72 matrices, 64 images x 197 tokens) with
-    one tenant per image through framefb_forward_tenants, against the same
-    step with one tenant for all tokens (framefb_forward)."""
+    one tenant per image through framefb_forward_tenants (the segment table
+    in the kernel's launch parameters, and, for comparison, one launch
+    matrix per (matrix, segment) with FRAMEFB_SEG_KERNEL=0), against the
+    same step with one tenant for all tokens (framefb_forward)."""
     import torch
     from paper_2608_26430_gb300 import framefb as ffb
     from paper_2608_26430_gb300 import workloads as wl
@@ -469,10 +471,16 @@ def serving_timing(dev, stream, reps: int = 10):
         return a.elapsed_time(z) / reps
 
     ms_t = timed(lambda: ffb.framefb_forward_tenants(mats, b.dtype_code, starts, tenants, T, stream))
+    os.environ["FRAMEFB_SEG_KERNEL"] = "0"
+    try:
+        ms_s = timed(lambda: ffb.framefb_forward_tenants(mats, b.dtype_code, starts, tenants, T, stream))
+    finally:
+        del os.environ["FRAMEFB_SEG_KERNEL"]
     ms_1 = timed(lambda: ffb.framefb_forward(b.mats, b.dtype_code, None, stream))
     return {"workload": "vit_b16 forward, 72 matrices, 64 images x 197 tokens", "tenants": T,
-            "ms_mixed_tenants": ms_t, "ms_one_tenant": ms_1, "tokens_per_s_mixed": w.N / (ms_t / 1e3),
-            "tokens_per_s_one_tenant": w.N / (ms_1 / 1e3)}
+            "ms_mixed_tenants": ms_t, "ms_one_tenant": ms_1, "mixed_over_one_tenant": ms_t / ms_1,
+            "ms_mixed_per_segment_launches": ms_s, "tokens_per_s_mixed": w.N / (ms_t / 1e3),
+            "tokens_per_s_one_tenant": w.N / (ms_1 / 1e3), "l2": "step moves more than L2"}
 
 
 def e2e_timing(batch, ops, ws, stream, steps, world, dev, barrier):
@@ -638,6 +646,8 @@ def main():
             per_config[name] = time_config(name, dev, stream, 5, 3, flush, with_cpu,
                                            headline if name == w.name else None)
         per_config["vit_b16_merge.merge"] = time_merge(dev, stream, 20, 3, flush)
+        if "vit_b16_merge" in args.configs.split(","):
+            per_config["vit_b16_merge.serving"] = serving if serving is not None else serving_timing(dev, stream)
         del flush
         torch.cuda.empty_cache()
 

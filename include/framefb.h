@@ -323,10 +323,15 @@ framefb_status framefb_fused_fwd_bwd(const framefb_mat* mats, int32_t nmats, fra
  * seg_start non-decreasing from 0 to N, empty segments allowed; tenants in
  * [0, ntenants)).  Each framefb_mat describes the whole batch (N = seg_start[nseg],
  * X and Y as for framefb_forward) and its c_val points to the tenants'
- * values, tenant-major: [ntenants][nnz] fp32 on the device.  Every segment
- * of every matrix is run as its own matrix of framefb_forward (rows offset
- * into X and Y, the tenant's row of c_val), so the coefficient SpMM loads a
- * tenant's values once per segment.  dX and dC are not touched.
+ * values, tenant-major: [ntenants][nnz] fp32 on the device.  For bf16
+ * activations on the two-token tcgen05 kernels, and at most 256 segments,
+ * the segment table travels in the kernel's launch parameters: each matrix's
+ * units of work stay inside segments, and the coefficient SpMM loads a
+ * tenant's values where the tenant changes (one launch per chunk of
+ * matrices, as framefb_forward).  Otherwise every segment of every matrix
+ * runs as its own matrix of framefb_forward (rows offset into X and Y, the
+ * tenant's row of c_val).  Both give the same Y, bit for bit.  dX and dC are
+ * not touched.
  * Errors as framefb_forward, and FRAMEFB_EINVAL for an inconsistent segment
  * table.
  */

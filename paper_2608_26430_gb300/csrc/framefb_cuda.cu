@@ -24,6 +24,9 @@
 namespace {
 
 using ffb::kMaxMats;
+
+// kernel parameters of the tensor-core launches (CUDA 12.1+: 32764 bytes)
+static_assert(sizeof(ffb::TcLaunchK) <= 32764, "tensor-core launch parameters exceed the parameter space");
 using ffb::kThreads;
 using ffb::kTmax;
 
@@ -61,6 +64,7 @@ struct Prepared {
   bool tc;    // bf16: pipelined kernel on tcgen05 tensor cores
   bool tc2;   // bf16: the same, two tokens per unit
   bool pack;  // tc2: some matrix packs several token pairs per unit
+  bool seg;   // tc2: the launch carries a segment table (mixed tenants)
   int T;      // tile tokens of the bf16 kernel
   int threads;
 };
@@ -74,6 +78,12 @@ void* tc_kernel_ptr(int mode) {
     case 7: return reinterpret_cast<void*>(ffb::tc_tile_kernel<7>);
     default: return nullptr;
   }
+}
+
+// forward of the two-token kernels with a segment table (mixed tenants)
+void* tc2_seg_kernel_ptr(bool pack) {
+  return pack ? reinterpret_cast<void*>(ffb::tc2p_tile_kernel<1, true>)
+              : reinterpret_cast<void*>(ffb::tc2_tile_kernel<1, true>);
 }
 
 // two-token kernel, or its packed form (several token pairs per unit)
@@ -317,8 +327,19 @@ bool kernel_is(const char* name) {
 bool tc_allowed() { return !kernel_is("tile"); }
 bool tc2_allowed() { return tc_allowed() && !kernel_is("tc"); }
 
-// Validate one chunk of matrices and fill the launch parameters.
-framefb_status prepare(const framefb_mat* mats, int32_t nmats, int32_t ops, framefb_dtype dt, Prepared& P) {
+// Segments of a mixed-tenant forward: tokens [start[i], start[i + 1]) of
+// every matrix belong to tenant tenant[i].
+struct SegTable {
+  int32_t nseg;
+  const int32_t* start;
+  const int32_t* tenant;
+};
+
+// Validate one chunk of matrices and fill the launch parameters.  With a
+// segment table the chunk must run on a two-token kernel with one pair
+// count for all its matrices (else FRAMEFB_EUNSUPPORTED).
+framefb_status prepare(const framefb_mat* mats, int32_t nmats, int32_t ops, framefb_dtype dt, Prepared& P,
+                       const SegTable* seg = nullptr) {
   const size_t esz = dt == FRAMEFB_BF16 ? 2 : 4;
   const bool F = ops & FRAMEFB_OP_FORWARD, D = ops & FRAMEFB_OP_BACKWARD_DX, C = ops & FRAMEFB_OP_GRAD_COEFF;
   std::memset(P.args, 0, sizeof(ffb::LaunchK));
@@ -401,6 +422,11 @@ framefb_status prepare(const framefb_mat* mats, int32_t nmats, int32_t ops, fram
     if (!T_mma) return FRAMEFB_EUNSUPPORTED;
     smem = mma_smem_map(mats, nmats, ops, reg, T_mma, staged, P.args);
   }
+  if (seg) {
+    if (!tc2 || ops != FRAMEFB_OP_FORWARD || seg->nseg > ffb::kTcMaxSeg) return FRAMEFB_EUNSUPPORTED;
+    for (int32_t j = 1; j < nmats; ++j)
+      if (pairs[j] != pairs[0]) return FRAMEFB_EUNSUPPORTED;
+  }
   for (int32_t j = 0; j < nmats; ++j) {
     const framefb_mat& M = mats[j];
     const FfbPlanHeader* h = plan_header(M.plan);
@@ -429,7 +455,13 @@ framefb_status prepare(const framefb_mat* mats, int32_t nmats, int32_t ops, fram
       if (bytes > static_cast<size_t>(kSmemBudget)) return FRAMEFB_EUNSUPPORTED;
       smem = std::max(smem, bytes);
     }
-    const int32_t ntiles = (M.N + T - 1) / T;
+    int32_t ntiles = (M.N + T - 1) / T;
+    if (seg) {  // the segments' runs of units
+      int64_t nt = 0;
+      for (int32_t i = 0; i < seg->nseg; ++i) nt += (seg->start[i + 1] - seg->start[i] + T - 1) / T;
+      if (nt > INT32_MAX / 2) return FRAMEFB_EUNSUPPORTED;
+      ntiles = static_cast<int32_t>(nt);
+    }
     ffb::MatK& K = P.args->m[j];
     K.X = M.X;
     K.dX = M.dX;
@@ -459,6 +491,18 @@ framefb_status prepare(const framefb_mat* mats, int32_t nmats, int32_t ops, fram
     units += ntiles;
     if (units > INT32_MAX / 2) return FRAMEFB_EUNSUPPORTED;
   }
+  if (seg) {
+    ffb::TcLaunchK& A = *P.tcargs;
+    const int32_t T = 2 * pairs[0];
+    A.nseg = seg->nseg;
+    A.seg_u0[0] = 0;
+    for (int32_t i = 0; i < seg->nseg; ++i) {
+      A.seg_tok[i] = seg->start[i];
+      A.seg_tenant[i] = seg->tenant[i];
+      A.seg_u0[i + 1] = A.seg_u0[i] + (seg->start[i + 1] - seg->start[i] + T - 1) / T;
+    }
+    A.seg_tok[seg->nseg] = seg->start[seg->nseg];
+  }
   P.args->nmats = nmats;
   P.args->total_units = static_cast<int32_t>(units);
   P.args->stride = (nnz_max + 63) & ~63;
@@ -483,13 +527,15 @@ framefb_status prepare(const framefb_mat* mats, int32_t nmats, int32_t ops, fram
   P.tc = tc;
   P.tc2 = tc2;
   P.pack = tc2 && pack;
+  P.seg = seg != nullptr;
   P.threads = (tc || tc2) ? ffb::kTcThreads : kThreads;
   P.T = T_mma;
   P.smem = std::max<size_t>(smem, 16);
   P.grid = 0;
   P.ws_bytes = 0;
   if (units == 0) return FRAMEFB_OK;
-  void* fn = tc2 ? tc2_kernel_ptr(ops, P.pack) : tc ? tc_kernel_ptr(ops) : tile_kernel_ptr(dt, ops, reg, T_mma);
+  void* fn = P.seg ? tc2_seg_kernel_ptr(P.pack)
+             : tc2 ? tc2_kernel_ptr(ops, P.pack) : tc ? tc_kernel_ptr(ops) : tile_kernel_ptr(dt, ops, reg, T_mma);
   if (!fn) return FRAMEFB_EINVAL;
   int dev = 0, sms = 0, per_sm = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return FRAMEFB_ECUDA;
@@ -585,13 +631,13 @@ size_t structured_workspace(const framefb_mat* mats, int32_t nmats, int32_t ops)
 // Validate every launch chunk of the structured matrices; *need = the
 // workspace the largest chunk needs.
 framefb_status structured_check(const framefb_mat* mats, int32_t nmats, int32_t ops, framefb_dtype dtype,
-                                size_t* need) {
+                                size_t* need, const SegTable* seg = nullptr) {
   *need = 0;
   Buffers b;
   for (int32_t j0 = 0, nm = 0; j0 < nmats; j0 += nm) {
     nm = chunk_len(mats + j0, nmats - j0, dtype);
     Prepared P = b.prep();
-    const framefb_status s = prepare(mats + j0, nm, ops, dtype, P);
+    const framefb_status s = prepare(mats + j0, nm, ops, dtype, P, seg);
     if (s != FRAMEFB_OK) return s;
     *need = std::max(*need, P.ws_bytes);
   }
@@ -600,12 +646,12 @@ framefb_status structured_check(const framefb_mat* mats, int32_t nmats, int32_t 
 
 // Queue the structured kernels (after structured_check).
 framefb_status structured_run(const framefb_mat* mats, int32_t nmats, int32_t ops, framefb_dtype dtype, void* ws,
-                              cudaStream_t st) {
+                              cudaStream_t st, const SegTable* seg = nullptr) {
   Buffers b;
   for (int32_t j0 = 0, nm = 0; j0 < nmats; j0 += nm) {
     nm = chunk_len(mats + j0, nmats - j0, dtype);
     Prepared P = b.prep();
-    const framefb_status s = prepare(mats + j0, nm, ops, dtype, P);
+    const framefb_status s = prepare(mats + j0, nm, ops, dtype, P, seg);
     if (s != FRAMEFB_OK) return s;
     if (P.grid == 0) {
       if (ops & FRAMEFB_OP_GRAD_COEFF) {  // no tokens: the gradient is zero
@@ -619,8 +665,10 @@ framefb_status structured_run(const framefb_mat* mats, int32_t nmats, int32_t op
     P.args->partial = static_cast<float*>(ws);
     P.tcargs->partial = static_cast<float*>(ws);
     P.red->partial = static_cast<const float*>(ws);
-    void* fn =
-        P.tc2 ? tc2_kernel_ptr(ops, P.pack) : P.tc ? tc_kernel_ptr(ops) : tile_kernel_ptr(dtype, ops, P.reg, P.T);
+    void* fn = P.seg   ? tc2_seg_kernel_ptr(P.pack)
+               : P.tc2 ? tc2_kernel_ptr(ops, P.pack)
+               : P.tc  ? tc_kernel_ptr(ops)
+                       : tile_kernel_ptr(dtype, ops, P.reg, P.T);
     void* kargs[] = {(P.tc || P.tc2) ? static_cast<void*>(P.tcargs) : static_cast<void*>(P.args)};
     if (cudaLaunchKernel(fn, dim3(P.grid), dim3(P.threads), kargs, P.smem, st) != cudaSuccess)
       return FRAMEFB_ECUDA;
@@ -850,7 +898,27 @@ extern "C" framefb_status framefb_forward_tenants(const framefb_mat* mats, int32
   for (int32_t i = 0; i < nseg; ++i)
     if (seg_start[i + 1] < seg_start[i] || seg_tenant[i] < 0 || seg_tenant[i] >= ntenants) return FRAMEFB_EINVAL;
   const int32_t N = seg_start[nseg];
-  // the segments of all matrices run as the matrices of one framefb_run call
+  for (int32_t j = 0; j < nmats; ++j)
+    if (!plan_header(mats[j].plan) || mats[j].N != N) return FRAMEFB_EINVAL;
+  // the segment table in the kernel parameters: units stay inside segments,
+  // one launch per chunk of matrices, where every chunk runs on a two-token
+  // kernel (FRAMEFB_SEG_KERNEL=0 takes the per-segment path below)
+  const char* env = std::getenv("FRAMEFB_SEG_KERNEL");
+  if (dtype == FRAMEFB_BF16 && nmats > 0 && nseg > 0 && nseg <= ffb::kTcMaxSeg && !(env && std::strcmp(env, "0") == 0)) {
+    std::vector<framefb_mat> grp, den;
+    framefb_status s = split_paths(mats, nmats, dtype, grp, den);
+    if (s != FRAMEFB_OK) return s;
+    if (den.empty()) {
+      const SegTable st{nseg, seg_start, seg_tenant};
+      size_t need = 0;
+      s = structured_check(grp.data(), static_cast<int32_t>(grp.size()), FRAMEFB_OP_FORWARD, dtype, &need, &st);
+      if (s == FRAMEFB_OK)
+        return structured_run(grp.data(), static_cast<int32_t>(grp.size()), FRAMEFB_OP_FORWARD, dtype, nullptr,
+                              static_cast<cudaStream_t>(stream), &st);
+      if (s != FRAMEFB_EUNSUPPORTED) return s;
+    }
+  }
+  // else the segments of all matrices run as the matrices of one framefb_run call
   if (static_cast<int64_t>(nmats) * nseg > INT32_MAX) return FRAMEFB_EINVAL;
   std::vector<framefb_mat> seg;
   try {

@@ -287,6 +287,7 @@ __device__ __forceinline__ void tc_load_chunk(Chunk<MODE, true, false>& ch, cons
 // swizzle, which lands one token row as the canonical SWIZZLE_64B K-major
 // UMMA operand (8-row atoms of 512 bytes).
 constexpr int kTcMaxMats = 64;
+constexpr int kTcMaxSeg = 256;  // segments of a mixed-tenant launch
 struct TcLaunchK {
   int32_t nmats, total_units, stride, S;
   float* partial;
@@ -298,6 +299,13 @@ struct TcLaunchK {
   int32_t tok_x, tok_u, vu, rzg, rzg_tok, pad2;
   MatK m[kTcMaxMats];
   alignas(64) CUtensorMap maps[2 * kTcMaxMats];
+  // mixed-tenant forward (two-token kernels): the tokens of every matrix
+  // fall in nseg segments, segment s = tokens [seg_tok[s], seg_tok[s + 1])
+  // of tenant seg_tenant[s], and a matrix's units are its segments' runs of
+  // units, unit seg_u0[s] + i holding tokens seg_tok[s] + T i .. of segment
+  // s only (nseg = 0: one run over all N tokens)
+  int32_t nseg, pad3;
+  int32_t seg_tok[kTcMaxSeg + 1], seg_u0[kTcMaxSeg + 1], seg_tenant[kTcMaxSeg];
 };
 
 __device__ __forceinline__ void tma_row3d(void* dst, const CUtensorMap* map, int32_t token, uint64_t* bar) {

@@ -24,6 +24,8 @@
 // Shapes: every group count a multiple of 8 and at most 128 (n, m <= 4096).
 // Waits are bounded as in tc_tile_kernel.
 #pragma once
+#include <type_traits>
+
 #include "framefb_tc.cuh"
 
 namespace ffb {
@@ -44,6 +46,42 @@ __device__ __forceinline__ bool spmm_bar_or(bool f) {
       : "memory");
   return out != 0;
 }
+
+// Matrix and segment of the units a role walks through in increasing order,
+// in a launch with a segment table (TcLaunchK::nseg > 0): every matrix's
+// units are its segments' runs of units, so a unit's tokens lie in one
+// segment and have one tenant.
+struct SegTrack {
+  int j, s;
+  int64_t end;  // first unit past matrix j
+  __device__ __forceinline__ void seek(const TcLaunchK& a, int64_t u) {
+    const int64_t lu = u - a.m[j].ubeg;
+    while (lu >= a.seg_u0[s + 1]) ++s;  // (empty segments have no units)
+  }
+  __device__ __forceinline__ void start(const TcLaunchK& a, int64_t u) {
+    j = matrix_of(a, 0, u);
+    end = a.m[j].ubeg + a.m[j].ntiles;
+    s = 0;
+    seek(a, u);
+  }
+  // returns true when the matrix changed
+  __device__ __forceinline__ bool advance(const TcLaunchK& a, int64_t u) {
+    bool moved = false;
+    while (u >= end) {
+      ++j;
+      end = a.m[j].ubeg + a.m[j].ntiles;
+      s = 0;
+      moved = true;
+    }
+    seek(a, u);
+    return moved;
+  }
+  // first token of unit u (u in matrix j, segment s) and the end of its segment
+  __device__ __forceinline__ int64_t tok0(const TcLaunchK& a, int64_t u) const {
+    return a.seg_tok[s] + static_cast<int64_t>(a.m[j].T) * (u - a.m[j].ubeg - a.seg_u0[s]);
+  }
+  __device__ __forceinline__ int32_t tend(const TcLaunchK& a) const { return a.seg_tok[s + 1]; }
+};
 
 // Register chunk of plan column `col` (its first KE entries): gather slots
 // in the float2 V / U layout, store targets in the canonical RZ / RG layout.
@@ -90,9 +128,26 @@ __device__ __forceinline__ void tc2_load_chunk(Chunk<MODE, true, false>& ch, con
   }
 }
 
-template <int MODE>
+// SEG: the launch carries a segment table (mixed-tenant forward): units
+// follow the segments and the coefficient values are the unit's tenant's.
+template <int MODE, bool SEG = false>
 __global__ void __launch_bounds__(kTcThreads, 1) tc2_tile_kernel(const __grid_constant__ TcLaunchK args) {
   constexpr bool F = MODE & MODE_F, D = MODE & MODE_D, C = MODE & MODE_C;
+  static_assert(!SEG || MODE == MODE_F, "segment tables serve the forward pass");
+  using Track = std::conditional_t<SEG, SegTrack, TileTrack>;
+  // first token of unit u (tracked by t), end of its tokens
+  auto tok0 = [&](const Track& t, int64_t u) -> int64_t {
+    if constexpr (SEG)
+      return t.tok0(args, u);
+    else
+      return 2 * (u - args.m[t.j].ubeg);
+  };
+  auto tend = [&](const Track& t) -> int64_t {
+    if constexpr (SEG)
+      return t.tend(args);
+    else
+      return args.m[t.j].N;
+  };
   constexpr bool NEED_V = F || C, NEED_U = D || C, SYN = F || D;
   constexpr int B = FFB_ENTRY_BLOCK;
   extern __shared__ __align__(1024) uint8_t smem[];
@@ -133,14 +188,14 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2_tile_kernel(const __grid_co
   // ---- copy issue (thread 32, at the start of its step, before it waits for
   // its own rows): both token rows of unit `issued`
   constexpr int kIssuer = 32;
-  TileTrack ti{};
+  Track ti{};
   int issued = 0;
   auto issue = [&]() {
     const int64_t u = u_begin + issued;
     ti.advance(args, u);
     const int jn = ti.j;
-    const int32_t t0 = static_cast<int32_t>(2 * (u - args.m[jn].ubeg));
-    const int Tc = min(2, args.m[jn].N - t0);
+    const int32_t t0 = static_cast<int32_t>(tok0(ti, u));
+    const int Tc = min(2, static_cast<int>(tend(ti) - t0));
     uint8_t* dst = stg0 + (issued % S) * args.stage;
     uint64_t* b = bar + (issued % S);
     mbar_arrive_expect_tx(b, static_cast<uint32_t>(Tc) * ((NEED_V ? 2u * args.m[jn].n : 0u) +
@@ -162,7 +217,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2_tile_kernel(const __grid_co
 
   if (warp < 4) {
     // ------------------------------------------------------------ tensor warps
-    TileTrack ta{}, ts{}, tr{};  // units of the analysis (s), the output rows (s-2), the synthesis issue (s-1)
+    Track ta{}, ts{}, tr{};  // units of the analysis (s), the output rows (s-2), the synthesis issue (s-1)
     ta.start(args, u_begin);
     ts.start(args, u_begin);
     tr.start(args, u_begin);
@@ -191,10 +246,10 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2_tile_kernel(const __grid_co
     const uint32_t lane_base = static_cast<uint32_t>(32 * warp) << 16;
     const int r0 = 32 * warp + lane;  // this thread's group (one 128-group tile)
     // synthesis matrix, in registers
-    int js = -1, N2 = 0, Gm2 = 0, Gn2 = 0;
+    int js = -1, Gm2 = 0, Gn2 = 0;
     bool on_y = false, on_x = false, wide_y = false, wide_x = false;
     __nv_bfloat16 *Y2 = nullptr, *X2 = nullptr;
-    int64_t ldy2 = 0, ldx2 = 0, ubeg2 = 0;
+    int64_t ldy2 = 0, ldx2 = 0;
     float seff2 = 0.f;
     auto load_syn = [&](int j) {
       js = j;
@@ -202,8 +257,6 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2_tile_kernel(const __grid_co
       X2 = static_cast<__nv_bfloat16*>(args.m[j].dX);
       ldy2 = args.m[j].ldy;
       ldx2 = args.m[j].ldx;
-      ubeg2 = args.m[j].ubeg;
-      N2 = args.m[j].N;
       Gm2 = args.m[j].m / FFB_GROUP;
       Gn2 = args.m[j].n / FFB_GROUP;
       seff2 = args.m[j].seff;
@@ -227,8 +280,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2_tile_kernel(const __grid_co
       if (epi) {
         ts.advance(args, u_begin + i2);
         if (ts.j != js) load_syn(ts.j);
-        t2 = 2 * (u_begin + i2 - ubeg2);
-        Tc2 = min(2, static_cast<int>(N2 - t2));
+        t2 = tok0(ts, u_begin + i2);
+        Tc2 = min(2, static_cast<int>(tend(ts) - t2));
       }
       // output rows of unit s-2 for this thread's group (read now, used after the wait)
       uint4 yp[2][2][4];
@@ -255,8 +308,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2_tile_kernel(const __grid_co
       if (ana && lane == 0 && warp < 2) {
         const int side = warp;
         ta.advance(args, u_begin + s);
-        const int64_t t0 = 2 * (u_begin + s - args.m[ta.j].ubeg);
-        const int Tc0 = min(2, static_cast<int>(args.m[ta.j].N - t0));
+        const int64_t t0 = tok0(ta, u_begin + s);
+        const int Tc0 = min(2, static_cast<int>(tend(ta) - t0));
         const bool landed = tc_wait_bounded(bar + (s % S), static_cast<uint32_t>((s / S) & 1));
         if (!landed) failed = true;
         if (landed && (side == 0 ? NEED_V : NEED_U)) {
@@ -316,8 +369,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2_tile_kernel(const __grid_co
       // half of the unit's parity
       if (iss && !failed && lane == 0) {
         tr.advance(args, u_begin + i1);
-        const int64_t t1 = 2 * (u_begin + i1 - args.m[tr.j].ubeg);
-        const int Tc1 = min(2, static_cast<int>(args.m[tr.j].N - t1));
+        const int64_t t1 = tok0(tr, u_begin + i1);
+        const int Tc1 = min(2, static_cast<int>(tend(tr) - t1));
         const int k = warp >> 1, side = warp & 1;
         const bool ok = tc_wait_bounded(rzg_bar, rzg_ph);
         if (ok)
@@ -358,9 +411,10 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2_tile_kernel(const __grid_co
     float dc[kEreg];
 #pragma unroll
     for (int e = 0; e < kEreg; ++e) dc[e] = 0.f;
-    TileTrack tp{}, tq{};
+    Track tp{}, tq{};
     tp.start(args, u_begin);
     tq.start(args, u_begin);
+    int tenant = -1;  // SEG: tenant of the loaded coefficient values
     uint32_t ana_ph = 0, syn_ph = 0;
     const int aside = (warp - 4) >> 2;  // analysis results written: warps 4-7 V (X), 8-11 U (dY)
     const uint32_t alane = static_cast<uint32_t>(32 * (warp & 3)) << 16;
@@ -378,6 +432,13 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2_tile_kernel(const __grid_co
       ana_open = ana;
       if (work) {
         tp.advance(args, u_begin + i1);
+        if constexpr (SEG) {
+          // another tenant of the same matrix: its coefficient values
+          if (tp.j == cur && args.seg_tenant[tp.s] != tenant) {
+            tenant = args.seg_tenant[tp.s];
+            tc2_load_chunk<MODE>(ch, splan, args.m[cur].c_val + static_cast<int64_t>(tenant) * hdr(splan).nnz, st);
+          }
+        }
         if (tp.j != cur) {
           if constexpr (C) {
             if (cur >= 0) {
@@ -389,7 +450,12 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2_tile_kernel(const __grid_co
           splan = args.m[cur].plan;
           mcur = args.m[cur].m;
           ncur = args.m[cur].n;
-          tc2_load_chunk<MODE>(ch, splan, args.m[cur].c_val, st);
+          if constexpr (SEG) {
+            tenant = args.seg_tenant[tp.s];
+            tc2_load_chunk<MODE>(ch, splan, args.m[cur].c_val + static_cast<int64_t>(tenant) * hdr(splan).nnz, st);
+          } else {
+            tc2_load_chunk<MODE>(ch, splan, args.m[cur].c_val, st);
+          }
 #pragma unroll
           for (int e = 0; e < kEreg; ++e) dc[e] = 0.f;
           zero_pending = true;
@@ -522,8 +588,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2_tile_kernel(const __grid_co
         if (ok && on) {
           tq.advance(args, u_begin + s);
           const int G = (aside == 0 ? args.m[tq.j].n : args.m[tq.j].m) / FFB_GROUP;
-          const int64_t t0 = 2 * (u_begin + s - args.m[tq.j].ubeg);
-          const bool two = args.m[tq.j].N - t0 >= 2;
+          const int64_t t0 = tok0(tq, u_begin + s);
+          const bool two = tend(tq) - t0 >= 2;
           float2* dst = aside == 0 ? V2 : U2;
 #pragma unroll
           for (int q8 = 0; q8 < 4; ++q8) {  // coefficients 8 q8 .. 8 q8 + 7: hi and lo in 16 columns

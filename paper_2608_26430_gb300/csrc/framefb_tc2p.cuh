@@ -28,9 +28,13 @@ namespace ffb {
 // the unpacked kernel).
 constexpr int kEregPack = 8;
 
-template <int MODE>
+// SEG: the launch carries a segment table (mixed-tenant forward): units
+// follow the segments and the coefficient values are the unit's tenant's.
+template <int MODE, bool SEG = false>
 __global__ void __launch_bounds__(kTcThreads, 1) tc2p_tile_kernel(const __grid_constant__ TcLaunchK args) {
   constexpr bool F = MODE & MODE_F, D = MODE & MODE_D, C = MODE & MODE_C;
+  static_assert(!SEG || MODE == MODE_F, "segment tables serve the forward pass");
+  using Track = std::conditional_t<SEG, SegTrack, TileTrack>;
   constexpr bool NEED_V = F || C, NEED_U = D || C, SYN = F || D;
   constexpr int B = FFB_ENTRY_BLOCK;
   constexpr int KE = kEregPack;  // register chunk entries
@@ -50,7 +54,20 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2p_tile_kernel(const __grid_c
   // token pairs per slot of matrix j (a unit is 2P tokens)
   auto pairs = [&](int j) { return args.m[j].T >> 1; };
   // slots of a unit starting at token t0 that hold tokens (1 or 2)
-  auto slots = [](int32_t N, int64_t t0, int P) { return N - t0 > P ? 2 : 1; };
+  auto slots = [](int64_t N, int64_t t0, int P) { return N - t0 > P ? 2 : 1; };
+  // first token of unit u (tracked by t), end of its tokens
+  auto tok0 = [&](const Track& t, int64_t u) -> int64_t {
+    if constexpr (SEG)
+      return t.tok0(args, u);
+    else
+      return 2 * static_cast<int64_t>(pairs(t.j)) * (u - args.m[t.j].ubeg);
+  };
+  auto tend = [&](const Track& t) -> int64_t {
+    if constexpr (SEG)
+      return t.tend(args);
+    else
+      return args.m[t.j].N;
+  };
 
   const int64_t units = args.total_units;
   const int64_t u_begin = (static_cast<int64_t>(blockIdx.x) * units) / gridDim.x;
@@ -76,18 +93,19 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2p_tile_kernel(const __grid_c
   // ---- copy issue (thread 32, at the start of its step, before it waits for
   // its own rows): both token rows of unit `issued`
   constexpr int kIssuer = 32;
-  TileTrack ti{};
+  Track ti{};
   int issued = 0;
   auto issue = [&]() {
     const int64_t u = u_begin + issued;
     ti.advance(args, u);
     const int jn = ti.j;
     const int P = pairs(jn);
-    const int32_t t0 = static_cast<int32_t>(2 * P * (u - args.m[jn].ubeg));
-    const int ns = slots(args.m[jn].N, t0, P);
+    const int32_t t0 = static_cast<int32_t>(tok0(ti, u));
+    const int ns = slots(tend(ti), t0, P);
     uint8_t* dst = stg0 + (issued % S) * args.stage;
     uint64_t* b = bar + (issued % S);
-    // whole boxes of P token rows: rows past N land as zeros and count
+    // whole boxes of P token rows: rows past N land as zeros and count;
+    // rows past the segment's end (of the next segment) are not used
     mbar_arrive_expect_tx(b, static_cast<uint32_t>(ns * P) * ((NEED_V ? 2u * args.m[jn].n : 0u) +
                                                              (NEED_U ? 2u * args.m[jn].m : 0u)));
     for (int k = 0; k < ns; ++k) {
@@ -107,7 +125,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2p_tile_kernel(const __grid_c
 
   if (warp < 4) {
     // ------------------------------------------------------------ tensor warps
-    TileTrack ta{}, ts{}, tr{};  // units of the analysis (s), the output rows (s-2), the synthesis issue (s-1)
+    Track ta{}, ts{}, tr{};  // units of the analysis (s), the output rows (s-2), the synthesis issue (s-1)
     ta.start(args, u_begin);
     ts.start(args, u_begin);
     tr.start(args, u_begin);
@@ -137,10 +155,10 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2p_tile_kernel(const __grid_c
     const int r0 = 32 * warp + lane;  // this thread's TMEM lane: (pair, group) p G + g
     // synthesis matrix, in registers: pairs, and this lane's pair and group
     // per side (Y: out groups, dX: in groups)
-    int js = -1, N2 = 0, P2 = 1, py = 0, gy = 0, px = 0, gx = 0;
+    int js = -1, P2 = 1, py = 0, gy = 0, px = 0, gx = 0;
     bool on_y = false, on_x = false, wide_y = false, wide_x = false;
     __nv_bfloat16 *Y2 = nullptr, *X2 = nullptr;
-    int64_t ldy2 = 0, ldx2 = 0, ubeg2 = 0;
+    int64_t ldy2 = 0, ldx2 = 0;
     float seff2 = 0.f;
     auto load_syn = [&](int j) {
       js = j;
@@ -148,8 +166,6 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2p_tile_kernel(const __grid_c
       X2 = static_cast<__nv_bfloat16*>(args.m[j].dX);
       ldy2 = args.m[j].ldy;
       ldx2 = args.m[j].ldx;
-      ubeg2 = args.m[j].ubeg;
-      N2 = args.m[j].N;
       P2 = pairs(j);
       const int Gm2 = args.m[j].m / FFB_GROUP, Gn2 = args.m[j].n / FFB_GROUP;
       py = r0 / Gm2;
@@ -174,10 +190,12 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2p_tile_kernel(const __grid_c
       if (tid == kIssuer && issued < count) issue();
       int64_t t2 = 0;
       int Tc2 = 0;
+      int64_t N2 = 0;  // end of the unit's tokens
       if (epi) {
         ts.advance(args, u_begin + i2);
         if (ts.j != js) load_syn(ts.j);
-        t2 = 2 * P2 * (u_begin + i2 - ubeg2);
+        t2 = tok0(ts, u_begin + i2);
+        N2 = tend(ts);
         Tc2 = slots(N2, t2, P2);
       }
       // token of slot k on this lane's side, and whether it is one
@@ -210,8 +228,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2p_tile_kernel(const __grid_c
         const int side = warp;
         ta.advance(args, u_begin + s);
         const int P0 = pairs(ta.j);
-        const int64_t t0 = 2 * P0 * (u_begin + s - args.m[ta.j].ubeg);
-        const int Tc0 = slots(args.m[ta.j].N, t0, P0);
+        const int64_t t0 = tok0(ta, u_begin + s);
+        const int Tc0 = slots(tend(ta), t0, P0);
         const bool landed = tc_wait_bounded(bar + (s % S), static_cast<uint32_t>((s / S) & 1));
         if (!landed) failed = true;
         if (landed && (side == 0 ? NEED_V : NEED_U)) {
@@ -272,8 +290,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2p_tile_kernel(const __grid_c
       if (iss && !failed && lane == 0) {
         tr.advance(args, u_begin + i1);
         const int P1 = pairs(tr.j);
-        const int64_t t1 = 2 * P1 * (u_begin + i1 - args.m[tr.j].ubeg);
-        const int Tc1 = slots(args.m[tr.j].N, t1, P1);
+        const int64_t t1 = tok0(tr, u_begin + i1);
+        const int Tc1 = slots(tend(tr), t1, P1);
         const int k = warp >> 1, side = warp & 1;
         const bool ok = tc_wait_bounded(rzg_bar, rzg_ph);
         if (ok)
@@ -314,9 +332,10 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2p_tile_kernel(const __grid_c
     float dc[kEreg];
 #pragma unroll
     for (int e = 0; e < KE; ++e) dc[e] = 0.f;
-    TileTrack tp{}, tq{};
+    Track tp{}, tq{};
     tp.start(args, u_begin);
     tq.start(args, u_begin);
+    int tenant = -1;  // SEG: tenant of the loaded coefficient values
     uint32_t ana_ph = 0, syn_ph = 0;
     const int aside = (warp - 4) >> 2;  // analysis results written: warps 4-7 V (X), 8-11 U (dY)
     const uint32_t alane = static_cast<uint32_t>(32 * (warp & 3)) << 16;
@@ -335,6 +354,13 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2p_tile_kernel(const __grid_c
       ana_open = ana;
       if (work) {
         tp.advance(args, u_begin + i1);
+        if constexpr (SEG) {
+          // another tenant of the same matrix: its coefficient values
+          if (tp.j == cur && args.seg_tenant[tp.s] != tenant) {
+            tenant = args.seg_tenant[tp.s];
+            tc2_load_chunk<MODE, KE>(ch, splan, args.m[cur].c_val + static_cast<int64_t>(tenant) * hdr(splan).nnz, st);
+          }
+        }
         if (tp.j != cur) {
           if constexpr (C) {
             if (cur >= 0) {
@@ -347,7 +373,12 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2p_tile_kernel(const __grid_c
           mcur = args.m[cur].m;
           ncur = args.m[cur].n;
           Pc = pairs(cur);
-          tc2_load_chunk<MODE, KE>(ch, splan, args.m[cur].c_val, st);
+          if constexpr (SEG) {
+            tenant = args.seg_tenant[tp.s];
+            tc2_load_chunk<MODE, KE>(ch, splan, args.m[cur].c_val + static_cast<int64_t>(tenant) * hdr(splan).nnz, st);
+          } else {
+            tc2_load_chunk<MODE, KE>(ch, splan, args.m[cur].c_val, st);
+          }
 #pragma unroll
           for (int e = 0; e < KE; ++e) dc[e] = 0.f;
           zero_pending = true;
@@ -378,8 +409,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2p_tile_kernel(const __grid_c
           }
         }
         // pairs of the unit that hold tokens
-        const int64_t t0s = 2 * static_cast<int64_t>(Pc) * (u_begin + i1 - args.m[cur].ubeg);
-        const int np = static_cast<int>(min(static_cast<int64_t>(Pc), args.m[cur].N - t0s));
+        const int64_t t0s = tok0(tp, u_begin + i1);
+        const int np = static_cast<int>(min(static_cast<int64_t>(Pc), tend(tp) - t0s));
         for (int p = 0; p < np; ++p) {
           const float2* V2p = V2 + p * (ncur + mcur);
           const float2* U2p = V2p + ncur;
@@ -504,8 +535,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2p_tile_kernel(const __grid_c
           // this lane's pair and group
           const int pp = ar / G;
           const int g = ar - pp * G;
-          const int64_t t0 = 2 * static_cast<int64_t>(P) * (u_begin + s - args.m[tq.j].ubeg);
-          const bool two = args.m[tq.j].N - t0 > P + pp;  // token t0 + P + pp (slot 1) exists
+          const int64_t t0 = tok0(tq, u_begin + s);
+          const bool two = tend(tq) - t0 > P + pp;  // token t0 + P + pp (slot 1) exists
           float2* dst = V2 + pp * (nq + mq) + (aside == 0 ? 0 : nq);
 #pragma unroll
           for (int q8 = 0; q8 < 4; ++q8) {  // coefficients 8 q8 .. 8 q8 + 7: hi and lo in 16 columns
