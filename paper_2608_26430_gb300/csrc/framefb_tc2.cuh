@@ -53,34 +53,60 @@ __device__ __forceinline__ bool spmm_bar_or(bool f) {
 // segment and have one tenant.
 struct SegTrack {
   int j, s;
-  int64_t end;  // first unit past matrix j
+  int64_t end;       // first unit past matrix j
+  int64_t ubeg;      // first unit of matrix j
+  int32_t T;         // tokens per unit of matrix j
+  int32_t u1;        // end of segment s in matrix-local units
+  int64_t base;      // first token of unit u = base + T u
+  int32_t tk1;       // end of segment s in tokens
+  bool seg_moved;    // the last advance entered another segment
+  __device__ __forceinline__ void load_mat(const TcLaunchK& a) {
+    ubeg = a.m[j].ubeg;
+    end = ubeg + a.m[j].ntiles;
+    T = a.m[j].T;
+  }
+  __device__ __forceinline__ void load_seg(const TcLaunchK& a) {
+    u1 = a.seg_u0[s + 1];
+    tk1 = a.seg_tok[s + 1];
+    base = a.seg_tok[s] - static_cast<int64_t>(T) * (ubeg + a.seg_u0[s]);
+  }
+  // segment of unit u of matrix j, from segment s on (empty segments have
+  // no units); the bounds of the current segment stay in registers
   __device__ __forceinline__ void seek(const TcLaunchK& a, int64_t u) {
-    const int64_t lu = u - a.m[j].ubeg;
-    while (lu >= a.seg_u0[s + 1]) ++s;  // (empty segments have no units)
+    seg_moved = false;
+    if (u - ubeg < u1) return;
+    do ++s;
+    while (u - ubeg >= a.seg_u0[s + 1]);
+    load_seg(a);
+    seg_moved = true;
   }
   __device__ __forceinline__ void start(const TcLaunchK& a, int64_t u) {
     j = matrix_of(a, 0, u);
-    end = a.m[j].ubeg + a.m[j].ntiles;
+    load_mat(a);
     s = 0;
+    load_seg(a);
     seek(a, u);
+    seg_moved = true;
   }
   // returns true when the matrix changed
   __device__ __forceinline__ bool advance(const TcLaunchK& a, int64_t u) {
     bool moved = false;
-    while (u >= end) {
-      ++j;
-      end = a.m[j].ubeg + a.m[j].ntiles;
+    if (u >= end) {
+      do {
+        ++j;
+        load_mat(a);
+      } while (u >= end);
       s = 0;
+      load_seg(a);
       moved = true;
     }
     seek(a, u);
+    seg_moved = seg_moved || moved;
     return moved;
   }
   // first token of unit u (u in matrix j, segment s) and the end of its segment
-  __device__ __forceinline__ int64_t tok0(const TcLaunchK& a, int64_t u) const {
-    return a.seg_tok[s] + static_cast<int64_t>(a.m[j].T) * (u - a.m[j].ubeg - a.seg_u0[s]);
-  }
-  __device__ __forceinline__ int32_t tend(const TcLaunchK& a) const { return a.seg_tok[s + 1]; }
+  __device__ __forceinline__ int64_t tok0(const TcLaunchK&, int64_t u) const { return base + T * u; }
+  __device__ __forceinline__ int32_t tend(const TcLaunchK&) const { return tk1; }
 };
 
 // Register chunk of plan column `col` (its first KE entries): gather slots
@@ -434,7 +460,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2_tile_kernel(const __grid_co
         tp.advance(args, u_begin + i1);
         if constexpr (SEG) {
           // another tenant of the same matrix: its coefficient values
-          if (tp.j == cur && args.seg_tenant[tp.s] != tenant) {
+          if (tp.seg_moved && tp.j == cur && args.seg_tenant[tp.s] != tenant) {
             tenant = args.seg_tenant[tp.s];
             tc2_load_chunk<MODE>(ch, splan, args.m[cur].c_val + static_cast<int64_t>(tenant) * hdr(splan).nnz, st);
           }

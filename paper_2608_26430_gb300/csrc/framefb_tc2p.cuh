@@ -356,7 +356,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc2p_tile_kernel(const __grid_c
         tp.advance(args, u_begin + i1);
         if constexpr (SEG) {
           // another tenant of the same matrix: its coefficient values
-          if (tp.j == cur && args.seg_tenant[tp.s] != tenant) {
+          if (tp.seg_moved && tp.j == cur && args.seg_tenant[tp.s] != tenant) {
             tenant = args.seg_tenant[tp.s];
             tc2_load_chunk<MODE, KE>(ch, splan, args.m[cur].c_val + static_cast<int64_t>(tenant) * hdr(splan).nnz, st);
           }
