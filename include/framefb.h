@@ -207,6 +207,34 @@ size_t framefb_plan_bytes(const framefb_plan* plan);
 const void* framefb_plan_data(const framefb_plan* plan);
 void framefb_plan_free(framefb_plan* plan);
 
+/*
+ * Parts of a structured plan that the fused tcgen05 kernels cannot take
+ * whole (more than 16 * FRAMEFB_THREADS entries, or an output frame of more
+ * than 128 groups of 32 features: the LLaMA-3 shapes), for plans whose input
+ * frame has at most 128 groups.  The support is cut into blocks of whole
+ * groups of the output side (at most 128 groups, a multiple of 8) and, per
+ * block, runs of at most 16 * FRAMEFB_THREADS entries in row-major order.
+ * (Blocks of the input side would give every part a partial sum of each
+ * row, and rounding the bf16 output once per part would exceed the bf16
+ * tolerance on heavy-tailed supports: such plans have no parts.)  Every part is a plan of its own over its two blocks,
+ * stored in the plan's device image after the whole plan, with the list of
+ * its entries' indices into the caller's C values and dC (int32).  framefb_run
+ * runs each part as a matrix of the fused kernels: ΔW is linear in C, so
+ * Y and dX take the sum of the parts' contributions, and each part writes
+ * its own entries of dC.  This restates the method exactly; it is the
+ * library's own execution plan, with no counterpart in the paper.
+ * framefb_plan_parts returns the number of parts (0 for plans the kernels
+ * take whole) and fills up to max_parts descriptors (parts may be NULL).
+ */
+typedef struct {
+  int64_t image_offset, image_bytes;  /* the part's plan image in the device image */
+  int64_t q_offset;                   /* its int32 entry indices (nnz of them) in the device image */
+  int32_t nnz;                        /* its entries */
+  int32_t n0, m0;                     /* first input / output feature of its blocks */
+  int32_t n, m;                       /* features of its blocks */
+} framefb_plan_part;
+int32_t framefb_plan_parts(const framefb_plan* plan, framefb_plan_part* parts, int32_t max_parts);
+
 /* ------------------------------------------------------------------------ */
 /* S3-S6  batched activation kernels (device)                                */
 /* ------------------------------------------------------------------------ */

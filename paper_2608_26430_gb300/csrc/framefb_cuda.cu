@@ -38,7 +38,7 @@ const FfbPlanHeader* plan_header(const framefb_plan* p) {
   if (!p || p->image.size() < sizeof(FfbPlanHeader)) return nullptr;
   const FfbPlanHeader* h = reinterpret_cast<const FfbPlanHeader*>(p->image.data());
   if (h->magic != FFB_PLAN_MAGIC || h->version != FFB_PLAN_VERSION || h->P != kThreads) return nullptr;
-  if (static_cast<size_t>(h->total_bytes) != p->image.size()) return nullptr;
+  if (static_cast<size_t>(h->total_bytes) > p->image.size()) return nullptr;  // (parts follow the plan)
   return h;
 }
 
@@ -350,7 +350,7 @@ framefb_status prepare(const framefb_mat* mats, int32_t nmats, int32_t ops, fram
     const FfbPlanHeader* h = groups_header(mats[j].plan);
     if (!h) return FRAMEFB_EINVAL;
     if (h->EZ > ffb::kEreg || h->EG > ffb::kEreg) reg = false;
-    nnz_max = std::max(nnz_max, h->nnz);
+    nnz_max = std::max({nnz_max, h->nnz, h->nnz_full});  // dC partial slots are indexed by q
   }
   int64_t units = 0;
   size_t smem = 0;
@@ -431,7 +431,8 @@ framefb_status prepare(const framefb_mat* mats, int32_t nmats, int32_t ops, fram
     const framefb_mat& M = mats[j];
     const FfbPlanHeader* h = plan_header(M.plan);
     if (M.N < 0 || M.n <= 0 || M.m <= 0) return FRAMEFB_EINVAL;
-    if (!frame_ok(M.fin, M.n) || !frame_ok(M.fout, M.m)) return FRAMEFB_EINVAL;
+    // (a plan's part covers blocks of the frames' features: n, m < d)
+    if (!frame_ok(M.fin, h->d_in) || !frame_ok(M.fout, h->d_out)) return FRAMEFB_EINVAL;
     if (h->n != M.n || h->m != M.m) return FRAMEFB_EINVAL;
     if (!M.plan_dev || !aligned16(M.plan_dev)) return FRAMEFB_EINVAL;
     if (!std::isfinite(M.scale)) return FRAMEFB_EINVAL;
@@ -484,6 +485,8 @@ framefb_status prepare(const framefb_mat* mats, int32_t nmats, int32_t ops, fram
     K.seff = M.scale / 16.f;
     ffb::ReduceMat& R = P.red->m[j];
     R.dC = M.dC;
+    R.qlist = h->off_qlist ? reinterpret_cast<const int32_t*>(static_cast<const uint8_t*>(M.plan_dev) + h->off_qlist)
+                           : nullptr;
     R.ubeg = K.ubeg;
     R.ntiles = ntiles;
     R.nnz = h->nnz;
@@ -714,21 +717,32 @@ bool fused_tc_ok(const FfbPlanHeader& h) {
          h.Gn <= 128 * ffb::kTcMaxTiles && h.Gm <= 128 * ffb::kTcMaxTiles;
 }
 
+bool parts_allowed() {
+  const char* e = std::getenv("FRAMEFB_PARTS");
+  return !(e && std::strcmp(e, "0") == 0);
+}
+
 // Matrices of a call split by path, each in call order: the fused kernels
-// (structured plans they take, fp32, or rows with padding), and the
-// contraction path of framefb_dense.cu (dense-layout plans, and bf16
-// structured plans the fused tcgen05 kernels do not take, with unpadded
-// rows).  FRAMEFB_KERNEL=tile keeps every structured plan on the warp-MMA
-// kernel.
+// (structured plans they take, fp32, or rows with padding), the plans' parts
+// on the fused tcgen05 kernels (bf16 structured plans the kernels do not
+// take whole, with parts, and tokens; FRAMEFB_PARTS=0 sends them to the
+// contraction path), and the contraction path of framefb_dense.cu
+// (dense-layout plans, and the other bf16 structured plans the fused
+// tcgen05 kernels do not take, with unpadded rows).  FRAMEFB_KERNEL=tile
+// keeps every structured plan on the warp-MMA kernel.
 framefb_status split_paths(const framefb_mat* mats, int32_t nmats, framefb_dtype dt, std::vector<framefb_mat>& grp,
-                           std::vector<framefb_mat>& den) {
+                           std::vector<framefb_mat>& den, std::vector<framefb_mat>* prt = nullptr) {
   try {
     for (int32_t j = 0; j < nmats; ++j) {
       const framefb_mat& M = mats[j];
       const FfbPlanHeader* h = plan_header(M.plan);
       if (!h) return FRAMEFB_EINVAL;
-      const bool split = h->layout == FFB_LAYOUT_GROUPS && dt == FRAMEFB_BF16 && tc_allowed() && !fused_tc_ok(*h) &&
-                         M.ldx == M.n && M.ldy == M.m;
+      const bool big = h->layout == FFB_LAYOUT_GROUPS && dt == FRAMEFB_BF16 && tc_allowed() && !fused_tc_ok(*h);
+      if (big && prt && parts_allowed() && !M.plan->subs.empty() && M.N > 0) {
+        prt->push_back(M);
+        continue;
+      }
+      const bool split = big && M.ldx == M.n && M.ldy == M.m;
       (h->layout == FFB_LAYOUT_DENSE || split ? den : grp).push_back(M);
     }
     // the two-token kernel's units carry P token pairs of a matrix (P = 1
@@ -744,6 +758,58 @@ framefb_status split_paths(const framefb_mat* mats, int32_t nmats, framefb_dtype
   return FRAMEFB_OK;
 }
 
+// The launch waves of the structured matrices: wave 0 holds the matrices
+// the fused kernels take whole; the matrices with parts run as their parts,
+// one matrix of the fused kernels per part (its blocks of X, dY, Y and dX,
+// the part's plan, the whole c_val and dC indexed by the part's entries).
+// ΔW is linear in C, so Y and dX take the sum of the parts' contributions;
+// parts of one matrix that write the same features of Y (forward) or dX
+// (backward dx) read-modify-write the same bytes and go to successive waves
+// (greedily), so that no launch holds both.
+framefb_status plan_waves(const framefb_mat* mats, int32_t nmats, int32_t ops, framefb_dtype dt,
+                          std::vector<std::vector<framefb_mat>>& waves, std::vector<framefb_mat>& den) {
+  std::vector<framefb_mat> grp, prt;
+  framefb_status s = split_paths(mats, nmats, dt, grp, den, &prt);
+  if (s != FRAMEFB_OK) return s;
+  const bool F = ops & FRAMEFB_OP_FORWARD, D = ops & FRAMEFB_OP_BACKWARD_DX;
+  const size_t esz = dt == FRAMEFB_BF16 ? 2 : 4;
+  try {
+    waves.assign(1, std::move(grp));
+    for (const framefb_mat& M : prt) {
+      const std::vector<FfbSubPlan>& sub = M.plan->subs;
+      std::vector<int32_t> wave(sub.size(), 0);
+      for (size_t i = 0; i < sub.size(); ++i) {
+        auto clash = [&](size_t k) {
+          return (F && sub[k].m0 == sub[i].m0) || (D && sub[k].n0 == sub[i].n0);
+        };
+        int32_t w = 0;
+        for (bool busy = true; busy; ) {
+          busy = false;
+          for (size_t k = 0; k < i && !busy; ++k) busy = wave[k] == w && clash(k);
+          if (busy) ++w;
+        }
+        wave[i] = w;
+        framefb_mat V = M;
+        const FfbPlanHeader* h = plan_header(sub[i].plan);
+        if (!h) return FRAMEFB_EINVAL;
+        V.n = h->n;
+        V.m = h->m;
+        V.X = M.X ? static_cast<const uint8_t*>(M.X) + esz * sub[i].n0 : nullptr;
+        V.dX = M.dX ? static_cast<uint8_t*>(M.dX) + esz * sub[i].n0 : nullptr;
+        V.dY = M.dY ? static_cast<const uint8_t*>(M.dY) + esz * sub[i].m0 : nullptr;
+        V.Y = M.Y ? static_cast<uint8_t*>(M.Y) + esz * sub[i].m0 : nullptr;
+        V.plan = sub[i].plan;
+        V.plan_dev = M.plan_dev ? static_cast<const uint8_t*>(M.plan_dev) + sub[i].dev_off : nullptr;
+        if (static_cast<size_t>(w) >= waves.size()) waves.resize(w + 1);
+        waves[w].push_back(V);
+      }
+    }
+  } catch (const std::bad_alloc&) {
+    return FRAMEFB_ENOMEM;
+  }
+  return FRAMEFB_OK;
+}
+
 }  // namespace
 
 extern "C" size_t framefb_workspace_size(const framefb_mat* mats, int32_t nmats, int32_t ops) {
@@ -751,13 +817,16 @@ extern "C" size_t framefb_workspace_size(const framefb_mat* mats, int32_t nmats,
   // the routing depends on the dtype: the larger need of the two
   size_t need = 0;
   for (const framefb_dtype dt : {FRAMEFB_BF16, FRAMEFB_F32}) {
-    std::vector<framefb_mat> grp, den;
-    if (split_paths(mats, nmats, dt, grp, den) != FRAMEFB_OK) return 0;
+    std::vector<std::vector<framefb_mat>> waves;
+    std::vector<framefb_mat> den;
+    if (plan_waves(mats, nmats, ops, dt, waves, den) != FRAMEFB_OK) return 0;
     size_t dneed = 0;
     if (!den.empty() &&
         ffb_host::dense_check(den.data(), static_cast<int32_t>(den.size()), ops, dt, &dneed) != FRAMEFB_OK)
       continue;
-    need = std::max({need, structured_workspace(grp.data(), static_cast<int32_t>(grp.size()), ops), dneed});
+    need = std::max(need, dneed);
+    for (const std::vector<framefb_mat>& w : waves)
+      need = std::max(need, structured_workspace(w.data(), static_cast<int32_t>(w.size()), ops));
   }
   return need;
 }
@@ -768,23 +837,31 @@ extern "C" framefb_status framefb_run(const framefb_mat* mats, int32_t nmats, in
   if (dtype != FRAMEFB_F32 && dtype != FRAMEFB_BF16) return FRAMEFB_EINVAL;
   if (nmats == 0) return FRAMEFB_OK;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  std::vector<framefb_mat> grp, den;
-  framefb_status s = split_paths(mats, nmats, dtype, grp, den);
+  std::vector<std::vector<framefb_mat>> waves;
+  std::vector<framefb_mat> den;
+  framefb_status s = plan_waves(mats, nmats, ops, dtype, waves, den);
   if (s != FRAMEFB_OK) return s;
-  // validate everything before queueing anything; the two paths run one
-  // after the other on the stream and share the workspace
-  size_t gneed = 0, dneed = 0;
-  s = structured_check(grp.data(), static_cast<int32_t>(grp.size()), ops, dtype, &gneed);
-  if (s != FRAMEFB_OK) return s;
+  // validate everything before queueing anything; the waves and the two
+  // paths run one after the other on the stream and share the workspace
+  size_t need = 0;
+  for (const std::vector<framefb_mat>& w : waves) {
+    size_t gneed = 0;
+    s = structured_check(w.data(), static_cast<int32_t>(w.size()), ops, dtype, &gneed);
+    if (s != FRAMEFB_OK) return s;
+    need = std::max(need, gneed);
+  }
+  size_t dneed = 0;
   s = ffb_host::dense_check(den.data(), static_cast<int32_t>(den.size()), ops, dtype, &dneed);
   if (s != FRAMEFB_OK) return s;
-  const size_t need = std::max(gneed, dneed);
+  need = std::max(need, dneed);
   if (need > 0) {
     if (!ws || ws_bytes < need) return FRAMEFB_EWORKSPACE;
     if (reinterpret_cast<uintptr_t>(ws) & 255u) return FRAMEFB_EINVAL;
   }
-  s = structured_run(grp.data(), static_cast<int32_t>(grp.size()), ops, dtype, ws, st);
-  if (s != FRAMEFB_OK) return s;
+  for (const std::vector<framefb_mat>& w : waves) {
+    s = structured_run(w.data(), static_cast<int32_t>(w.size()), ops, dtype, ws, st);
+    if (s != FRAMEFB_OK) return s;
+  }
   return ffb_host::dense_run(den.data(), static_cast<int32_t>(den.size()), ops, dtype, ws, ws_bytes, st);
 }
 
@@ -794,12 +871,15 @@ extern "C" framefb_status framefb_kernel_names(const framefb_mat* mats, int32_t 
   buf[0] = '\0';
   if (nmats < 0 || (nmats > 0 && !mats) || !ops_ok(ops)) return FRAMEFB_EINVAL;
   if (dtype != FRAMEFB_F32 && dtype != FRAMEFB_BF16) return FRAMEFB_EINVAL;
-  std::vector<framefb_mat> grp, den;
-  framefb_status s = split_paths(mats, nmats, dtype, grp, den);
+  std::vector<std::vector<framefb_mat>> waves;
+  std::vector<framefb_mat> den;
+  framefb_status s = plan_waves(mats, nmats, ops, dtype, waves, den);
   if (s != FRAMEFB_OK) return s;
   std::vector<std::string> names;
-  s = structured_names(grp.data(), static_cast<int32_t>(grp.size()), ops, dtype, names);
-  if (s != FRAMEFB_OK) return s;
+  for (const std::vector<framefb_mat>& w : waves) {
+    s = structured_names(w.data(), static_cast<int32_t>(w.size()), ops, dtype, names);
+    if (s != FRAMEFB_OK) return s;
+  }
   if (!den.empty()) {
     size_t need = 0;
     s = ffb_host::dense_check(den.data(), static_cast<int32_t>(den.size()), ops, dtype, &need);

@@ -66,7 +66,7 @@ const FfbPlanHeader* header_of(const framefb_plan* p) {
   if (!p || p->image.size() < sizeof(FfbPlanHeader)) return nullptr;
   const FfbPlanHeader* h = reinterpret_cast<const FfbPlanHeader*>(p->image.data());
   if (h->magic != FFB_PLAN_MAGIC || h->version != FFB_PLAN_VERSION || h->P != fd::kSpmmThreads) return nullptr;
-  if (static_cast<size_t>(h->total_bytes) != p->image.size()) return nullptr;
+  if (static_cast<size_t>(h->total_bytes) > p->image.size()) return nullptr;  // (parts follow the plan)
   return h;
 }
 

@@ -6,6 +6,8 @@
 #include "plan_internal.h"
 
 #include <algorithm>
+#include <atomic>
+#include <memory>
 #include <cmath>
 #include <cstdlib>
 #include <cstring>
@@ -405,7 +407,7 @@ struct PathBanks {
 // Outputs: pos[p * E + e] = entry index or -1 (padding), store[entry] = its
 // store target or FFB_NO_STORE.
 void pack_runs(const std::vector<Entry>& ent, int32_t P, int32_t E, int32_t base, int32_t nkeys,
-               const PathBanks& bk, bool search, std::vector<int32_t>& pos, std::vector<int32_t>& store,
+               const PathBanks& bk, int32_t moves, std::vector<int32_t>& pos, std::vector<int32_t>& store,
                std::vector<int32_t>& fix, int32_t& novf) {
   const int32_t nnz = static_cast<int32_t>(ent.size());
   pos.assign(static_cast<size_t>(P) * E, -1);
@@ -537,7 +539,7 @@ void pack_runs(const std::vector<Entry>& ent, int32_t P, int32_t E, int32_t base
     if (pl[k].len >= 2) multi.push_back(static_cast<int32_t>(k));
   }
   SplitMix64 rng{0x6A09E667F3BCC909ull ^ static_cast<uint64_t>(nnz)};
-  const int64_t iters = search ? std::min<int64_t>(static_cast<int64_t>(nnz) * 4000, 60000000) : 0;
+  const int64_t iters = std::min<int64_t>(static_cast<int64_t>(nnz) * moves, 60000000);
   std::vector<std::pair<int32_t, int32_t>> cells;
   std::vector<int32_t> groups, newcost;
   auto add_cell = [&](int32_t p, int32_t e) {
@@ -650,6 +652,204 @@ inline int32_t align16(size_t x) { return static_cast<int32_t>((x + 15) & ~size_
 
 }  // namespace
 
+namespace {
+
+// Plan image of the entries byrow (key0 = row a, key1 = column b, q = the
+// entry's index into the caller's C values and dC) and bycol (key0 = b,
+// key1 = a) over index spaces n (columns) and m (rows): chunks cut for
+// FRAMEFB_THREADS threads, store targets, fix-ups, group masks, merge block
+// lists.  nnz_full: the size of the q index space (the caller's nnz).
+// moves: moves per entry of the bank-placement search (0: none; the
+// default kernel's structured plans).
+framefb_status build_plan_image(int32_t n, int32_t m, bool structured, int32_t moves, int32_t d_in, int32_t d_out,
+                                std::vector<Entry>& byrow, std::vector<Entry>& bycol, int32_t nnz_full,
+                                std::vector<uint8_t>& image) {
+  const int32_t P = FRAMEFB_THREADS;
+  const int32_t nz = static_cast<int32_t>(byrow.size());
+  const int32_t Gn = (n + FFB_GROUP - 1) / FFB_GROUP, Gm = (m + FFB_GROUP - 1) / FFB_GROUP;
+  auto lt = [](const Entry& x, const Entry& y) { return x.key0 != y.key0 ? x.key0 < y.key0 : x.key1 < y.key1; };
+  std::sort(byrow.begin(), byrow.end(), lt);
+  std::sort(bycol.begin(), bycol.end(), lt);
+  const int32_t EZ = (nz + P - 1) / P, EG = EZ;
+
+  std::vector<int32_t> posZ, storeZ, fixZ, posG, storeG, fixG;
+  int32_t novfZ = 0, novfG = 0;
+  // banks of the default kernel's slots: row path gathers V[b] and stores
+  // Z[a]; column path gathers U[a], reloads V[b] where b changes and stores
+  // G[b]
+  PathBanks bkZ, bkG;
+  bkZ.gather.resize(nz);
+  bkZ.store.resize(nz);
+  for (int32_t q = 0; q < nz; ++q) {
+    bkZ.gather[q] = static_cast<int8_t>(gather_bank(byrow[q].key1));
+    bkZ.store[q] = static_cast<int8_t>(store_bank(byrow[q].key0, m));
+  }
+  bkG.gather.resize(nz);
+  bkG.key.resize(nz);
+  bkG.store.resize(nz);
+  for (int32_t q = 0; q < nz; ++q) {
+    bkG.gather[q] = static_cast<int8_t>(gather_bank(bycol[q].key1));
+    bkG.key[q] = static_cast<int8_t>(gather_bank(bycol[q].key0));
+    bkG.store[q] = static_cast<int8_t>(store_bank(bycol[q].key0, n));
+  }
+  // the two paths are independent searches: run them side by side (in
+  // sequence if no thread can be started); exceptions reach the caller's
+  // handler after the join
+  {
+    std::exception_ptr ez, eg;
+    auto run_z = [&]() {
+      try {
+        pack_runs(byrow, P, EZ, m, m, bkZ, moves, posZ, storeZ, fixZ, novfZ);
+      } catch (...) {
+        ez = std::current_exception();
+      }
+    };
+    std::thread tz;
+    try {
+      tz = std::thread(run_z);
+    } catch (const std::system_error&) {
+      run_z();
+    }
+    try {
+      pack_runs(bycol, P, EG, n, n, bkG, moves, posG, storeG, fixG, novfG);
+    } catch (...) {
+      eg = std::current_exception();
+    }
+    if (tz.joinable()) tz.join();
+    if (ez) std::rethrow_exception(ez);
+    if (eg) std::rethrow_exception(eg);
+  }
+
+  // store targets (own slots and overflow slots) are 16-bit fields
+  if (m + novfZ >= static_cast<int32_t>(FFB_NO_STORE) || n + novfG >= static_cast<int32_t>(FFB_NO_STORE))
+    return FRAMEFB_EUNSUPPORTED;
+  FfbPlanHeader h;
+  std::memset(&h, 0, sizeof(h));
+  h.layout = structured ? FFB_LAYOUT_GROUPS : FFB_LAYOUT_DENSE;
+  h.d_in = d_in;
+  h.d_out = d_out;
+  h.magic = FFB_PLAN_MAGIC;
+  h.version = FFB_PLAN_VERSION;
+  h.n = n;
+  h.m = m;
+  h.Gn = Gn;
+  h.Gm = Gm;
+  h.nnz = nz;
+  h.P = P;
+  h.EZ = EZ;
+  h.EG = EG;
+  h.ovfZ = (novfZ + 3) & ~3;
+  h.ovfG = (novfG + 3) & ~3;
+  h.nfixZ = static_cast<int32_t>(fixZ.size() / 4);
+  h.nfixG = static_cast<int32_t>(fixG.size() / 4);
+  h.nnz_full = nnz_full;
+
+  size_t off = align16(sizeof(FfbPlanHeader));
+  auto take = [&](size_t bytes) { const int32_t o = static_cast<int32_t>(off); off = align16(off + bytes); return o; };
+  const size_t ezp = static_cast<size_t>(EZ) * P, egp = static_cast<size_t>(EG) * P;
+  h.off_zb = take(ezp * 4);
+  h.off_zq = take(ezp * 4);
+  h.off_ga = take(egp * 4);
+  h.off_gb = take(egp * 4);
+  h.off_gq = take(egp * 4);
+  h.off_fixZ = take(fixZ.size() * 4);
+  h.off_fixG = take(fixG.size() * 4);
+  h.off_zmask = take(static_cast<size_t>(Gm) * 4);
+  h.off_gmask = take(static_cast<size_t>(Gn) * 4);
+  const size_t nblk = static_cast<size_t>(Gm) * Gn;
+  h.off_blkptr = take((nblk + 1) * 4);
+  h.off_blkent = take(static_cast<size_t>(nz) * 8);
+  if (off > static_cast<size_t>(INT32_MAX)) return FRAMEFB_EUNSUPPORTED;
+  h.total_bytes = static_cast<int32_t>(off);
+
+  image.assign(off, 0);
+  uint8_t* base = image.data();
+  auto arr = [&](int32_t o) { return reinterpret_cast<int32_t*>(base + o); };
+  std::memcpy(base, &h, sizeof(h));
+
+  // Per-thread chunk tables, entry-major ([e][p]) so that a warp reading
+  // entry e of its 32 threads touches 128 contiguous bytes.
+  int32_t* zb = arr(h.off_zb);
+  int32_t* zq = arr(h.off_zq);
+  int32_t* ga = arr(h.off_ga);
+  int32_t* gb = arr(h.off_gb);
+  int32_t* gq = arr(h.off_gq);
+  for (int32_t p = 0; p < P; ++p) {
+    for (int32_t e = 0; e < EZ; ++e) {
+      const int32_t idx = posZ[static_cast<size_t>(p) * EZ + e];
+      const size_t slot = static_cast<size_t>(e) * P + p;
+      if (idx >= 0) {
+        zb[slot] = byrow[idx].key1 | ((byrow[idx].key0 & 1) << 15) | (storeZ[idx] << 16);
+        zq[slot] = byrow[idx].q;
+      } else {
+        zb[slot] = (FFB_NO_STORE << 16);
+        zq[slot] = -1;
+      }
+    }
+    for (int32_t e = 0; e < EG; ++e) {
+      const int32_t idx = posG[static_cast<size_t>(p) * EG + e];
+      const size_t slot = static_cast<size_t>(e) * P + p;
+      if (idx >= 0) {
+        ga[slot] = bycol[idx].key1 | ((bycol[idx].key0 & 1) << 15) | (storeG[idx] << 16);
+        gb[slot] = bycol[idx].key0;
+        gq[slot] = bycol[idx].q;
+      } else {
+        ga[slot] = (FFB_NO_STORE << 16);
+        gb[slot] = 0;
+        gq[slot] = -1;
+      }
+    }
+  }
+  if (!fixZ.empty()) std::memcpy(arr(h.off_fixZ), fixZ.data(), fixZ.size() * 4);
+  if (!fixG.empty()) std::memcpy(arr(h.off_fixG), fixG.data(), fixG.size() * 4);
+  uint32_t* zmask = reinterpret_cast<uint32_t*>(arr(h.off_zmask));
+  uint32_t* gmask = reinterpret_cast<uint32_t*>(arr(h.off_gmask));
+  for (int32_t q = 0; q < nz; ++q) {
+    zmask[byrow[q].key0 >> 5] |= 1u << (byrow[q].key0 & 31);
+    gmask[bycol[q].key0 >> 5] |= 1u << (bycol[q].key0 & 31);
+  }
+  // Merge: entries grouped by 32 x 32 block (out group g, in group h).
+  int32_t* blkptr = arr(h.off_blkptr);
+  int32_t* blkent = arr(h.off_blkent);
+  std::vector<int32_t> cnt(nblk + 1, 0);
+  for (int32_t q = 0; q < nz; ++q) cnt[static_cast<size_t>(byrow[q].key0 >> 5) * Gn + (byrow[q].key1 >> 5) + 1]++;
+  for (size_t b = 0; b < nblk; ++b) cnt[b + 1] += cnt[b];
+  std::memcpy(blkptr, cnt.data(), (nblk + 1) * 4);
+  for (int32_t q = 0; q < nz; ++q) {  // byrow is sorted by (a, b): entries stay ordered inside a block
+    const size_t b = static_cast<size_t>(byrow[q].key0 >> 5) * Gn + (byrow[q].key1 >> 5);
+    const int32_t dst = cnt[b]++;
+    blkent[2 * dst] = (byrow[q].key0 & 31) | ((byrow[q].key1 & 31) << 8);
+    blkent[2 * dst + 1] = byrow[q].q;
+  }
+  return FRAMEFB_OK;
+}
+
+// Sub-plans of a structured plan beyond the fused tcgen05 kernels' limits
+// (more than kSubEntries entries, so longer chunks than the register chunk,
+// or an output side of more than kSubGroups groups): the output side cut
+// into blocks of whole groups (at most kSubGroups, a multiple of 8), and the
+// entries of a block, in row-major order, into runs of at most kSubEntries.  A
+// sub-plan is the plan of its run over its two blocks (group-major indices
+// less the blocks' first columns) and keeps the caller's entry indices q.
+constexpr int32_t kSubGroups = 128;
+constexpr int32_t kSubEntries = 16 * FRAMEFB_THREADS;
+// moves per entry of the bank-placement search: a whole plan, a part
+constexpr int32_t kMovesWhole = 4000, kMovesPart = 1500;
+
+struct Block { int32_t g0, g1; };  // groups [g0, g1)
+
+std::vector<Block> side_blocks(int32_t G) {
+  const int32_t nb = (G + kSubGroups - 1) / kSubGroups;
+  const int32_t w = ((G + nb - 1) / nb + 7) / 8 * 8;
+  std::vector<Block> out;
+  for (int32_t g0 = 0; g0 < G; g0 += w) out.push_back(Block{g0, std::min(G, g0 + w)});
+  return out;
+}
+
+inline size_t align256(size_t x) { return (x + 255) & ~size_t{255}; }
+
+}  // namespace
+
 extern "C" framefb_status framefb_plan_build(const framefb_frame* fin, const framefb_frame* fout,
                                              const int32_t* row, const int32_t* col, int64_t nnz,
                                              framefb_plan** out) {
@@ -676,8 +876,6 @@ extern "C" framefb_status framefb_plan_build(const framefb_frame* fin, const fra
     }
   }
   try {
-    const int32_t P = FRAMEFB_THREADS;
-    const int32_t Gn = (n + FFB_GROUP - 1) / FFB_GROUP, Gm = (m + FFB_GROUP - 1) / FFB_GROUP;
     std::vector<Entry> byrow(nz), bycol(nz);
     for (int32_t q = 0; q < nz; ++q) {
       const int32_t a = structured ? group_major(row[q], fout->rho) : row[q];
@@ -685,165 +883,139 @@ extern "C" framefb_status framefb_plan_build(const framefb_frame* fin, const fra
       byrow[q] = Entry{a, b, q};
       bycol[q] = Entry{b, a, q};
     }
-    auto lt = [](const Entry& x, const Entry& y) { return x.key0 != y.key0 ? x.key0 < y.key0 : x.key1 < y.key1; };
-    std::sort(byrow.begin(), byrow.end(), lt);
-    std::sort(bycol.begin(), bycol.end(), lt);
-    const int32_t EZ = (nz + P - 1) / P, EG = EZ;
-
-    std::vector<int32_t> posZ, storeZ, fixZ, posG, storeG, fixG;
-    int32_t novfZ = 0, novfG = 0;
-    // banks of the default kernel's slots: row path gathers V[b] and stores
-    // Z[a]; column path gathers U[a], reloads V[b] where b changes and stores
-    // G[b]
-    PathBanks bkZ, bkG;
-    bkZ.gather.resize(nz);
-    bkZ.store.resize(nz);
-    for (int32_t q = 0; q < nz; ++q) {
-      bkZ.gather[q] = static_cast<int8_t>(gather_bank(byrow[q].key1));
-      bkZ.store[q] = static_cast<int8_t>(store_bank(byrow[q].key0, m));
-    }
-    bkG.gather.resize(nz);
-    bkG.key.resize(nz);
-    bkG.store.resize(nz);
-    for (int32_t q = 0; q < nz; ++q) {
-      bkG.gather[q] = static_cast<int8_t>(gather_bank(bycol[q].key1));
-      bkG.key[q] = static_cast<int8_t>(gather_bank(bycol[q].key0));
-      bkG.store[q] = static_cast<int8_t>(store_bank(bycol[q].key0, n));
-    }
-    // the two paths are independent searches: run them side by side (in
-    // sequence if no thread can be started); exceptions reach the caller's
-    // handler after the join
-    {
-      std::exception_ptr ez, eg;
-      auto run_z = [&]() {
-        try {
-          pack_runs(byrow, P, EZ, m, m, bkZ, structured, posZ, storeZ, fixZ, novfZ);
-        } catch (...) {
-          ez = std::current_exception();
-        }
-      };
-      std::thread tz;
-      try {
-        tz = std::thread(run_z);
-      } catch (const std::system_error&) {
-        run_z();
-      }
-      try {
-        pack_runs(bycol, P, EG, n, n, bkG, structured, posG, storeG, fixG, novfG);
-      } catch (...) {
-        eg = std::current_exception();
-      }
-      if (tz.joinable()) tz.join();
-      if (ez) std::rethrow_exception(ez);
-      if (eg) std::rethrow_exception(eg);
-    }
-
-    // store targets (own slots and overflow slots) are 16-bit fields
-    if (m + novfZ >= static_cast<int32_t>(FFB_NO_STORE) || n + novfG >= static_cast<int32_t>(FFB_NO_STORE))
-      return FRAMEFB_EUNSUPPORTED;
-    FfbPlanHeader h;
-    std::memset(&h, 0, sizeof(h));
-    h.layout = structured ? FFB_LAYOUT_GROUPS : FFB_LAYOUT_DENSE;
-    h.d_in = fin->d;
-    h.d_out = fout->d;
-    h.magic = FFB_PLAN_MAGIC;
-    h.version = FFB_PLAN_VERSION;
-    h.n = n;
-    h.m = m;
-    h.Gn = Gn;
-    h.Gm = Gm;
-    h.nnz = nz;
-    h.P = P;
-    h.EZ = EZ;
-    h.EG = EG;
-    h.ovfZ = (novfZ + 3) & ~3;
-    h.ovfG = (novfG + 3) & ~3;
-    h.nfixZ = static_cast<int32_t>(fixZ.size() / 4);
-    h.nfixG = static_cast<int32_t>(fixG.size() / 4);
-
-    size_t off = align16(sizeof(FfbPlanHeader));
-    auto take = [&](size_t bytes) { const int32_t o = static_cast<int32_t>(off); off = align16(off + bytes); return o; };
-    const size_t ezp = static_cast<size_t>(EZ) * P, egp = static_cast<size_t>(EG) * P;
-    h.off_zb = take(ezp * 4);
-    h.off_zq = take(ezp * 4);
-    h.off_ga = take(egp * 4);
-    h.off_gb = take(egp * 4);
-    h.off_gq = take(egp * 4);
-    h.off_fixZ = take(fixZ.size() * 4);
-    h.off_fixG = take(fixG.size() * 4);
-    h.off_zmask = take(static_cast<size_t>(Gm) * 4);
-    h.off_gmask = take(static_cast<size_t>(Gn) * 4);
-    const size_t nblk = static_cast<size_t>(Gm) * Gn;
-    h.off_blkptr = take((nblk + 1) * 4);
-    h.off_blkent = take(static_cast<size_t>(nz) * 8);
-    if (off > static_cast<size_t>(INT32_MAX)) return FRAMEFB_EUNSUPPORTED;
-    h.total_bytes = static_cast<int32_t>(off);
-
+    const std::vector<Entry> ent = byrow;  // (a, b, q) in the caller's order
+    const int32_t Gn = (n + FFB_GROUP - 1) / FFB_GROUP, Gm = (m + FFB_GROUP - 1) / FFB_GROUP;
+    // the fused tcgen05 kernels take the plan whole, or run its parts (the
+    // whole plan then serves the other kernels only: no bank placement).
+    // Parts need the input side in one block: blocks of the input side would
+    // each hold a partial sum of every row's entries, and the bf16 output
+    // rounded once per part would then lose more than the tolerance of the
+    // bf16 path where a row's partial sums are larger than its sum
+    // (heavy-tailed supports); runs of entries keep a row together but for
+    // the row at a run boundary.
+    const bool parts = structured && nz > 0 && Gn <= kSubGroups && (nz > kSubEntries || Gm > kSubGroups);
+    std::vector<uint8_t> image;
+    framefb_status st =
+        build_plan_image(n, m, structured, structured && !parts ? kMovesWhole : 0, fin->d, fout->d, byrow, bycol, nz, image);
+    if (st != FRAMEFB_OK) return st;
     framefb_plan* plan = new framefb_plan;
-    plan->image.assign(off, 0);
-    uint8_t* base = plan->image.data();
-    auto arr = [&](int32_t o) { return reinterpret_cast<int32_t*>(base + o); };
-    std::memcpy(base, &h, sizeof(h));
-
-    // Per-thread chunk tables, entry-major ([e][p]) so that a warp reading
-    // entry e of its 32 threads touches 128 contiguous bytes.
-    int32_t* zb = arr(h.off_zb);
-    int32_t* zq = arr(h.off_zq);
-    int32_t* ga = arr(h.off_ga);
-    int32_t* gb = arr(h.off_gb);
-    int32_t* gq = arr(h.off_gq);
-    for (int32_t p = 0; p < P; ++p) {
-      for (int32_t e = 0; e < EZ; ++e) {
-        const int32_t idx = posZ[static_cast<size_t>(p) * EZ + e];
-        const size_t slot = static_cast<size_t>(e) * P + p;
-        if (idx >= 0) {
-          zb[slot] = byrow[idx].key1 | ((byrow[idx].key0 & 1) << 15) | (storeZ[idx] << 16);
-          zq[slot] = byrow[idx].q;
-        } else {
-          zb[slot] = (FFB_NO_STORE << 16);
-          zq[slot] = -1;
+    std::unique_ptr<framefb_plan> guard(plan);
+    plan->image = std::move(image);
+    if (parts) {
+      const std::vector<Block> bo = side_blocks(Gm), bi = side_blocks(Gn);
+      // the parts' entries first; their plans are built side by side
+      struct Job { std::vector<Entry> r, c, blk; int32_t n0, m0, nv, mv; std::vector<uint8_t> image; framefb_status st; };
+      std::vector<Job> jobs;
+      for (const Block& ob : bo) {
+        for (const Block& ib : bi) {
+          std::vector<Entry> blk;  // (a, b, q) of the block pair, block-local indices
+          for (const Entry& e : ent) {
+            const int32_t ga = e.key0 / FFB_GROUP, gb = e.key1 / FFB_GROUP;
+            if (ga >= ob.g0 && ga < ob.g1 && gb >= ib.g0 && gb < ib.g1)
+              blk.push_back(Entry{e.key0 - FFB_GROUP * ob.g0, e.key1 - FFB_GROUP * ib.g0, e.q});
+          }
+          if (blk.empty()) continue;
+          std::sort(blk.begin(), blk.end(), [](const Entry& x, const Entry& y) {
+            return x.key0 != y.key0 ? x.key0 < y.key0 : x.key1 < y.key1;
+          });
+          const int32_t cnt = static_cast<int32_t>(blk.size());
+          const int32_t runs = (cnt + kSubEntries - 1) / kSubEntries;
+          for (int32_t r = 0; r < runs; ++r) {
+            const int32_t e0 = static_cast<int32_t>(static_cast<int64_t>(cnt) * r / runs);
+            const int32_t e1 = static_cast<int32_t>(static_cast<int64_t>(cnt) * (r + 1) / runs);
+            Job jb;
+            jb.r.assign(blk.begin() + e0, blk.begin() + e1);
+            jb.c.resize(jb.r.size());
+            for (size_t i = 0; i < jb.r.size(); ++i) jb.c[i] = Entry{jb.r[i].key1, jb.r[i].key0, jb.r[i].q};
+            jb.blk = jb.r;  // (a, b, q) in row-major order: the part's entry list
+            jb.n0 = FFB_GROUP * ib.g0;
+            jb.m0 = FFB_GROUP * ob.g0;
+            jb.nv = FFB_GROUP * (ib.g1 - ib.g0);
+            jb.mv = FFB_GROUP * (ob.g1 - ob.g0);
+            jb.st = FRAMEFB_OK;
+            jobs.push_back(std::move(jb));
+          }
         }
       }
-      for (int32_t e = 0; e < EG; ++e) {
-        const int32_t idx = posG[static_cast<size_t>(p) * EG + e];
-        const size_t slot = static_cast<size_t>(e) * P + p;
-        if (idx >= 0) {
-          ga[slot] = bycol[idx].key1 | ((bycol[idx].key0 & 1) << 15) | (storeG[idx] << 16);
-          gb[slot] = bycol[idx].key0;
-          gq[slot] = bycol[idx].q;
-        } else {
-          ga[slot] = (FFB_NO_STORE << 16);
-          gb[slot] = 0;
-          gq[slot] = -1;
+      {
+        std::vector<std::exception_ptr> err(jobs.size());
+        auto work = [&](size_t i) {
+          try {
+            Job& jb = jobs[i];
+            jb.st = build_plan_image(jb.nv, jb.mv, true, kMovesPart, fin->d, fout->d, jb.r, jb.c, nz, jb.image);
+          } catch (...) {
+            err[i] = std::current_exception();
+          }
+        };
+        const size_t hw = std::max<size_t>(1, std::thread::hardware_concurrency() / 2);  // each build runs two threads
+        std::vector<std::thread> pool;
+        std::atomic<size_t> next{0};
+        auto loop = [&]() {
+          for (size_t i = next++; i < jobs.size(); i = next++) work(i);
+        };
+        for (size_t t = 0; t + 1 < std::min(hw, jobs.size()); ++t) {
+          try {
+            pool.emplace_back(loop);
+          } catch (const std::system_error&) {
+            break;
+          }
         }
+        loop();
+        for (std::thread& t : pool) t.join();
+        for (const std::exception_ptr& e : err)
+          if (e) std::rethrow_exception(e);
+      }
+      for (Job& jb : jobs) {
+        if (jb.st != FRAMEFB_OK) return jb.st;
+        FfbSubPlan sp{};
+        sp.plan = new framefb_plan;
+        std::unique_ptr<framefb_plan> sguard(sp.plan);
+        sp.plan->image = std::move(jb.image);
+        sp.n0 = jb.n0;
+        sp.m0 = jb.m0;
+        sp.nq = static_cast<int32_t>(jb.blk.size());
+        // the part's image ends with its entries' q; it sits in the device
+        // image after the whole plan, 256-byte aligned
+        std::vector<uint8_t>& pim = sp.plan->image;
+        const size_t qo = (pim.size() + 15) & ~size_t{15};
+        if (qo + 4 * static_cast<size_t>(sp.nq) > static_cast<size_t>(INT32_MAX)) return FRAMEFB_EUNSUPPORTED;
+        pim.resize(qo + 4 * static_cast<size_t>(sp.nq), 0);
+        int32_t* ql = reinterpret_cast<int32_t*>(pim.data() + qo);
+        for (int32_t i = 0; i < sp.nq; ++i) ql[i] = jb.blk[i].q;
+        FfbPlanHeader* ph = reinterpret_cast<FfbPlanHeader*>(pim.data());
+        ph->off_qlist = static_cast<int32_t>(qo);
+        ph->total_bytes = static_cast<int32_t>(pim.size());
+        sp.dev_off = align256(plan->image.size());
+        sp.q_off = sp.dev_off + qo;
+        plan->image.resize(sp.dev_off + pim.size(), 0);
+        std::memcpy(plan->image.data() + sp.dev_off, pim.data(), pim.size());
+        plan->subs.push_back(sp);
+        sguard.release();
       }
     }
-    if (!fixZ.empty()) std::memcpy(arr(h.off_fixZ), fixZ.data(), fixZ.size() * 4);
-    if (!fixG.empty()) std::memcpy(arr(h.off_fixG), fixG.data(), fixG.size() * 4);
-    uint32_t* zmask = reinterpret_cast<uint32_t*>(arr(h.off_zmask));
-    uint32_t* gmask = reinterpret_cast<uint32_t*>(arr(h.off_gmask));
-    for (int32_t q = 0; q < nz; ++q) {
-      zmask[byrow[q].key0 >> 5] |= 1u << (byrow[q].key0 & 31);
-      gmask[bycol[q].key0 >> 5] |= 1u << (bycol[q].key0 & 31);
-    }
-    // Merge: entries grouped by 32 x 32 block (out group g, in group h).
-    int32_t* blkptr = arr(h.off_blkptr);
-    int32_t* blkent = arr(h.off_blkent);
-    std::vector<int32_t> cnt(nblk + 1, 0);
-    for (int32_t q = 0; q < nz; ++q) cnt[static_cast<size_t>(byrow[q].key0 >> 5) * Gn + (byrow[q].key1 >> 5) + 1]++;
-    for (size_t b = 0; b < nblk; ++b) cnt[b + 1] += cnt[b];
-    std::memcpy(blkptr, cnt.data(), (nblk + 1) * 4);
-    for (int32_t q = 0; q < nz; ++q) {  // byrow is sorted by (a, b): entries stay ordered inside a block
-      const size_t b = static_cast<size_t>(byrow[q].key0 >> 5) * Gn + (byrow[q].key1 >> 5);
-      const int32_t dst = cnt[b]++;
-      blkent[2 * dst] = (byrow[q].key0 & 31) | ((byrow[q].key1 & 31) << 8);
-      blkent[2 * dst + 1] = byrow[q].q;
-    }
-    *out = plan;
+    *out = guard.release();
   } catch (const std::bad_alloc&) {
     return FRAMEFB_ENOMEM;
   }
   return FRAMEFB_OK;
+}
+
+extern "C" int32_t framefb_plan_parts(const framefb_plan* plan, framefb_plan_part* parts, int32_t max_parts) {
+  if (!plan) return 0;
+  const int32_t n = static_cast<int32_t>(plan->subs.size());
+  for (int32_t i = 0; i < n && i < max_parts && parts; ++i) {
+    const FfbSubPlan& sp = plan->subs[i];
+    const FfbPlanHeader* h = reinterpret_cast<const FfbPlanHeader*>(sp.plan->image.data());
+    parts[i].image_offset = static_cast<int64_t>(sp.dev_off);
+    parts[i].image_bytes = static_cast<int64_t>(sp.plan->image.size());
+    parts[i].q_offset = static_cast<int64_t>(sp.q_off);
+    parts[i].nnz = sp.nq;
+    parts[i].n0 = sp.n0;
+    parts[i].m0 = sp.m0;
+    parts[i].n = h->n;
+    parts[i].m = h->m;
+  }
+  return n;
 }
 
 extern "C" size_t framefb_plan_bytes(const framefb_plan* plan) { return plan ? plan->image.size() : 0; }

@@ -66,6 +66,7 @@ struct LaunchK {
 
 struct ReduceMat {
   float* dC;
+  const int32_t* qlist;  // a plan's part: the entries' indices into dC (nnz of them), else null
   int32_t ubeg, ntiles, nnz;
   float seff;
 };
@@ -730,12 +731,14 @@ __global__ void __launch_bounds__(kThreads, 1) fft_tile_kernel(const __grid_cons
   if (cur >= 0) ch.flush(plan, args.partial + static_cast<size_t>(blockIdx.x + cur) * args.stride, L, fsm, tid);
 }
 
-// dC_q = (s/16) * sum over the CTAs that visited the matrix, in CTA order.
+// dC_q = (s/16) * sum over the CTAs that visited the matrix, in CTA order
+// (a plan's part: q over its entries' indices).
 __global__ void __launch_bounds__(256) dc_reduce_kernel(const __grid_constant__ ReduceK r) {
   const int j = blockIdx.y;
   const ReduceMat& M = r.m[j];
-  const int q = blockIdx.x * blockDim.x + threadIdx.x;
-  if (q >= M.nnz) return;
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= M.nnz) return;
+  const int q = M.qlist ? __ldg(M.qlist + i) : i;
   float s = 0.f;
   if (M.ntiles > 0) {
     const int32_t c0 = cta_of_unit(M.ubeg, r.grid, r.total_units);

@@ -30,7 +30,7 @@
 #endif
 
 #define FFB_PLAN_MAGIC 0x50424646  /* "FFBP" */
-#define FFB_PLAN_VERSION 2
+#define FFB_PLAN_VERSION 3
 #define FFB_LAYOUT_GROUPS 0        /* structured kernels: group-major column index (k = 16, k*rho = d) */
 #define FFB_LAYOUT_DENSE 1         /* dense path: frame columns in the paper's order */
 #define FFB_GROUP 32               /* real coordinates (and frame columns) per group */
@@ -55,7 +55,9 @@ struct FfbPlanHeader {
   int32_t total_bytes;
   int32_t layout;          // FFB_LAYOUT_GROUPS or FFB_LAYOUT_DENSE (index space of the tables)
   int32_t d_in, d_out;     // features of the frames (= n, m for FFB_LAYOUT_GROUPS)
-  int32_t reserved[3];
+  int32_t nnz_full;        // size of the entry-index space q (the caller's nnz; > nnz for a part)
+  int32_t off_qlist;       // a part: its entries' q (int32 [nnz]), else 0
+  int32_t reserved;
 };
 
 // Slot of group-major index x (x < K) in a tile buffer.  Slots come in

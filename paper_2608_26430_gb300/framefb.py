@@ -25,6 +25,7 @@ THREADS = 256
 EXPORTED = [
     "framefb_status_string", "framefb_abi_version", "framefb_frame_build", "framefb_frame_free",
     "framefb_support_build", "framefb_plan_build", "framefb_plan_bytes", "framefb_plan_data", "framefb_plan_free",
+    "framefb_plan_parts",
     "framefb_workspace_size", "framefb_run", "framefb_forward", "framefb_backward_dx", "framefb_grad_coeff",
     "framefb_backward", "framefb_fused_fwd_bwd", "framefb_merge", "framefb_run_static_ws",
     "framefb_wait_timeouts", "framefb_adamw", "framefb_linear_warmup_lr", "framefb_forward_tenants",
@@ -104,6 +105,8 @@ def lib() -> ct.CDLL:
                                          ct.POINTER(vp)]
         L.framefb_plan_bytes.restype = sz
         L.framefb_plan_bytes.argtypes = [vp]
+        L.framefb_plan_parts.restype = i32
+        L.framefb_plan_parts.argtypes = [vp, ct.POINTER(framefb_plan_part), i32]
         L.framefb_plan_data.restype = vp
         L.framefb_plan_data.argtypes = [vp]
         L.framefb_plan_free.restype = None
@@ -243,6 +246,11 @@ def framefb_support_build(rows: int, cols: int, nnz: int, seed: int, mode: int =
     return row[:nnz], col[:nnz], rowptr, perm[:nnz]
 
 
+class framefb_plan_part(ct.Structure):
+    _fields_ = [("image_offset", ct.c_int64), ("image_bytes", ct.c_int64), ("q_offset", ct.c_int64),
+                ("nnz", ct.c_int32), ("n0", ct.c_int32), ("m0", ct.c_int32), ("n", ct.c_int32), ("m", ct.c_int32)]
+
+
 class Plan:
     """Host plan handle (framefb_plan_build) and its device image bytes."""
 
@@ -264,6 +272,14 @@ class Plan:
         n = lib().framefb_plan_bytes(self.handle)
         ptr = lib().framefb_plan_data(self.handle)
         return np.ctypeslib.as_array(ct.cast(ptr, ct.POINTER(ct.c_uint8)), (n,)).copy()
+
+    def parts(self) -> list:
+        """Descriptors of the plan's parts (framefb_plan_parts; [] when the
+        fused kernels take the plan whole)."""
+        n = lib().framefb_plan_parts(self.handle, None, 0)
+        arr = (framefb_plan_part * max(n, 1))()
+        lib().framefb_plan_parts(self.handle, arr, n)
+        return [{f: getattr(arr[i], f) for f, _ in framefb_plan_part._fields_} for i in range(n)]
 
     def to_device(self, device):
         import torch

@@ -118,9 +118,13 @@ def test_blockdiag_and_per_layer_supports(wname, kernel, monkeypatch):
     check_batch(b, ALL)
 
 
-def test_llama3_zipf_nonsquare():
-    # nnz = 8192 exceeds the register-resident chunk of the fused kernels:
-    # the split contraction path (X and dY shared by the layer's matrices)
+@pytest.mark.parametrize("parts", ["1", "0"])
+def test_llama3_zipf_nonsquare(parts, monkeypatch):
+    # nnz = 8192 exceeds the register-resident chunk of the fused kernels and
+    # d = 14336 their 128 groups: the plans' parts on the two-token tcgen05
+    # kernel (FRAMEFB_PARTS=0: the split contraction path); X and dY shared
+    # by the layer's matrices
+    monkeypatch.setenv("FRAMEFB_PARTS", parts)
     w = wl.WORKLOADS["llama3_8b_all"]
     b = AdapterBatch(w, DEV, N=9, indices=list(range(7)), alias_inputs=True, ops=ALL)
     run(b, ALL)
@@ -364,11 +368,39 @@ def test_merge_many_tenants_grid_stride():
 # ---------------------------------------------------------------------------
 # plans the fused tcgen05 kernels do not take: the split contraction path
 # ---------------------------------------------------------------------------
-def test_llama3_shapes_take_the_split_path():
+@pytest.mark.parametrize("ops", [ffb.OP_FORWARD, ffb.OP_BACKWARD_DX, ffb.OP_GRAD_COEFF,
+                                 ffb.OP_BACKWARD_DX | ffb.OP_GRAD_COEFF, ALL])
+def test_llama3_shapes_run_as_parts(ops):
     """LLaMA-3 shapes (Zipf support with 32 entries per plan column, d up to
-    14336 = 448 groups) run as grouped K = 32 contractions around the SpMM;
-    with FRAMEFB_KERNEL=tile the same call runs on the warp-MMA kernel, and
-    both agree with the oracle."""
+    14336 = 448 groups) run as their plans' parts on the two-token tcgen05
+    kernel, parts that write the same features in successive launches, for
+    every op mask; Y and dX accumulate the parts' contributions.  The down
+    projection (14336 inputs) has no parts and runs on the split path."""
+    w = wl.WORKLOADS["llama3_8b_all"]
+    b = AdapterBatch(w, DEV, N=45, indices=list(range(7)), ops=ops)
+    for k in set(b.keys):
+        assert bool(b.plans[k].parts()) == (k[1] <= 4096), k   # key (m, n)
+    names = ffb.framefb_kernel_names(b.mats, ops, b.dtype_code)
+    assert f"tc2_tile_kernel<{ops}>" in names and any(x.startswith("dense_") for x in names)
+    run(b, ops)
+    check_batch(b, ops)
+    if ops & (ffb.OP_FORWARD | ffb.OP_BACKWARD_DX):
+        y1 = [(x.Y.float().clone() if x.Y is not None else None, x.dX.float().clone() if x.dX is not None else None)
+              for x in b.bufs]
+        run(b, ops)
+        # doubled within the bf16 bar: the parts round once each
+        for (ya, xa), x in zip(y1, b.bufs):
+            for on, got, once in ((ops & ffb.OP_FORWARD, x.Y, ya), (ops & ffb.OP_BACKWARD_DX, x.dX, xa)):
+                if on:
+                    rms = float(once.pow(2).mean().sqrt())
+                    torch.testing.assert_close(got.float(), 2 * once, rtol=2e-2, atol=2e-2 * 2 * rms)
+
+
+def test_llama3_shapes_take_the_split_path(monkeypatch):
+    """With FRAMEFB_PARTS=0 the LLaMA-3 shapes run as grouped K = 32
+    contractions around the SpMM; with FRAMEFB_KERNEL=tile the same call runs
+    on the warp-MMA kernel, and both agree with the oracle."""
+    monkeypatch.setenv("FRAMEFB_PARTS", "0")
     w = wl.WORKLOADS["llama3_8b_all"]
     b = AdapterBatch(w, DEV, N=45, indices=list(range(7)), ops=ALL)
     names = ffb.framefb_kernel_names(b.mats, ALL, b.dtype_code)
@@ -386,9 +418,13 @@ def test_llama3_shapes_on_the_warp_mma_kernel(monkeypatch):
     check_batch(b, ALL)
 
 
-def test_padded_rows_keep_large_plans_on_the_warp_mma_kernel():
-    """The split path views rows as [tokens * groups][32]: padded rows (a
-    leading dimension above the features) stay on the fused warp-MMA kernel."""
+@pytest.mark.parametrize("parts", ["1", "0"])
+def test_padded_rows_of_large_plans(parts, monkeypatch):
+    """Padded rows (a leading dimension above the features) of a large plan:
+    its parts on the two-token tcgen05 kernel take strided rows; without parts
+    the split path (which views rows as [tokens * groups][32]) does not, and
+    the plan stays on the fused warp-MMA kernel."""
+    monkeypatch.setenv("FRAMEFB_PARTS", parts)
     w = wl.WORKLOADS["llama3_8b_all"]
     N, pad = 17, 64
     src = AdapterBatch(w, DEV, N=N, indices=[1], ops=ALL)   # k: 4096 -> 1024
@@ -404,7 +440,8 @@ def test_padded_rows_keep_large_plans_on_the_warp_mma_kernel():
     key = src.keys[0]
     mat = ffb.make_mat(src.dev_frames[n], src.dev_frames[m], src.plans[key], src.plan_dev[key], bb.c_val, bb.scale, N,
                        X=Xp, dX=dXp, dY=dYp, Y=Yp, dC=dC, ldx=n + pad, ldy=m + pad)
-    assert ffb.framefb_kernel_names([mat], ALL, ffb.FRAMEFB_BF16) == ["mma_tile_kernel<7>"]
+    assert ffb.framefb_kernel_names([mat], ALL, ffb.FRAMEFB_BF16) == (["tc2_tile_kernel<7>"] if parts == "1"
+                                                                       else ["mma_tile_kernel<7>"])
     ffb.framefb_run([mat], ALL, ffb.FRAMEFB_BF16, ffb.workspace([mat], ALL, DEV))
     torch.cuda.synchronize()
     e = Expect(src, 0)

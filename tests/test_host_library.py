@@ -104,7 +104,7 @@ def test_support_build_rejects():
 # ---------------------------------------------------------------------------
 HDR = ["magic", "version", "n", "m", "Gn", "Gm", "nnz", "P", "EZ", "EG", "ovfZ", "ovfG", "nfixZ", "nfixG",
        "off_zb", "off_zq", "off_ga", "off_gb", "off_gq", "off_fixZ", "off_fixG", "off_zmask", "off_gmask",
-       "off_blkptr", "off_blkent", "total_bytes", "layout", "d_in", "d_out"]
+       "off_blkptr", "off_blkent", "total_bytes", "layout", "d_in", "d_out", "nnz_full", "off_qlist"]
 
 
 def decode(img):
@@ -313,3 +313,51 @@ def test_dense_operand_image_matches_oracle_frame(d, k, rho):
     assert not hi[:, d:].any() and not lo[:, d:].any() and not sy[:, K:].any()
     bits = img[2 * an:2 * an + d * cp * 4].view(np.uint32)
     assert np.all(bits & 0x1FFF == 0)                                        # 10-bit mantissas
+
+
+# ---------------------------------------------------------------------------
+# parts: plans the fused tcgen05 kernels cannot take whole (LLaMA-3 shapes)
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("n,m,nnz,mode", [(4096, 14336, 8192, 1), (14336, 4096, 8192, 1), (4096, 4096, 8192, 1),
+                                          (4096, 1024, 8192, 1), (4096, 4096, 4096 * 2 + 5, 0),
+                                          (14336, 14336, 9000, 0), (4096, 4096, 4096, 1)])
+def test_plan_parts_cover_the_support_once(n, m, nnz, mode):
+    fin, fout = ffb.Frame(n, 16, n // 16), ffb.Frame(m, 16, m // 16)
+    row, col, _, _ = support.sample_support(m, n, nnz, 1, mode, 1.1, 16)
+    plan = ffb.Plan(fin, fout, row, col)
+    img = plan.image()
+    parts = plan.parts()
+    whole = decode(img)["h"]
+    if (whole["EZ"] <= 16 and whole["Gm"] <= 128) or whole["Gn"] > 128:
+        assert parts == []      # the fused kernels take it whole, or input blocks would be needed
+        return
+    assert all(pt["n0"] == 0 and pt["n"] == n for pt in parts)
+    assert parts and whole["total_bytes"] <= parts[0]["image_offset"]
+    a_gm, b_gm = group_major(row, m // 16), group_major(col, n // 16)
+    seen = np.zeros(nnz, np.int32)
+    for pt in parts:
+        off = pt["image_offset"]
+        assert off % 256 == 0 and off + pt["image_bytes"] <= img.size
+        t = decode(img[off:off + pt["image_bytes"]])
+        h = t["h"]
+        # a plan of its own within the kernels' limits, over whole groups
+        assert (h["n"], h["m"], h["nnz"]) == (pt["n"], pt["m"], pt["nnz"]) and h["nnz_full"] == nnz
+        assert h["EZ"] <= 16 and h["EG"] <= 16 and h["nnz"] <= 16 * ffb.THREADS
+        assert h["Gn"] <= 128 and h["Gm"] <= 128 and h["Gn"] % 8 == 0 and h["Gm"] % 8 == 0
+        assert pt["n0"] % 256 == 0 and pt["m0"] % 256 == 0 and pt["n0"] + pt["n"] <= n and pt["m0"] + pt["m"] <= m
+        assert (h["d_in"], h["d_out"]) == (n, m)
+        # its entry list, in its own image and at q_offset of the parent's
+        q = np.frombuffer(img[off + h["off_qlist"]:off + h["off_qlist"] + 4 * h["nnz"]].tobytes(), np.int32)
+        q2 = np.frombuffer(img[pt["q_offset"]:pt["q_offset"] + 4 * pt["nnz"]].tobytes(), np.int32)
+        assert np.array_equal(q, q2)
+        seen[q] += 1
+        assert sorted(t["zq"][t["zq"] >= 0].tolist()) == sorted(q.tolist())
+        assert sorted(t["gq"][t["gq"] >= 0].tolist()) == sorted(q.tolist())
+        # block lists: every entry's local (a, b) is its group-major index less the blocks' start
+        for blk in range(h["Gm"] * h["Gn"]):
+            g, hh = divmod(blk, h["Gn"])
+            for e in range(t["blkptr"][blk], t["blkptr"][blk + 1]):
+                x, qq = t["blkent"][e]
+                assert 32 * g + (x & 31) == a_gm[qq] - pt["m0"]
+                assert 32 * hh + ((x >> 8) & 31) == b_gm[qq] - pt["n0"]
+    assert np.all(seen == 1)     # every entry in exactly one part
