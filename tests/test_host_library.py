@@ -361,3 +361,56 @@ def test_plan_parts_cover_the_support_once(n, m, nnz, mode):
                 assert 32 * g + (x & 31) == a_gm[qq] - pt["m0"]
                 assert 32 * hh + ((x >> 8) & 31) == b_gm[qq] - pt["n0"]
     assert np.all(seen == 1)     # every entry in exactly one part
+
+
+@pytest.mark.parametrize("n,m", [(4096, 14336), (4096, 4096)])
+def test_plan_parts_replay_coefficient_products(n, m):
+    """Every part of a Zipf(1.1) LLaMA-3-shaped plan (8192 entries) replays
+    the kernels' sparse steps exactly: run sums by row and by column with the
+    overflow slots and fix-ups, and the dC products, against the part's
+    entries at their block-local indices."""
+    nnz = 8192
+    fin, fout = ffb.Frame(n, 16, n // 16), ffb.Frame(m, 16, m // 16)
+    row, col, _, _ = support.sample_support(m, n, nnz, 1, 1, 1.1, 16)
+    plan = ffb.Plan(fin, fout, row, col)
+    img, parts = plan.image(), plan.parts()
+    assert parts
+    a_gm, b_gm = group_major(row, m // 16), group_major(col, n // 16)
+    rng = np.random.default_rng(1)
+    c = rng.standard_normal(nnz)
+    for pt in parts:
+        off = pt["image_offset"]
+        t = decode(img[off:off + pt["image_bytes"]])
+        h = t["h"]
+        nv, mv = h["n"], h["m"]
+        V, U = rng.standard_normal((2, nv)), rng.standard_normal((2, mv))
+        RZ, RG = np.zeros((2, mv + h["ovfZ"])), np.zeros((2, nv + h["ovfG"]))
+        dC = np.zeros(nnz)
+        for p in range(h["P"]):
+            acc = np.zeros(2)
+            for e in range(h["EZ"]):
+                pk, q = int(t["zb"][e, p]), int(t["zq"][e, p])
+                acc += (c[q] if q >= 0 else 0.0) * V[:, pk & 0x7FFF]
+                if (pk >> 16) != 0xFFFF:
+                    RZ[:, pk >> 16] = acc
+                    acc = np.zeros(2)
+            acc = np.zeros(2)
+            for e in range(h["EG"]):
+                pa, pb, q = int(t["ga"][e, p]), int(t["gb"][e, p]), int(t["gq"][e, p])
+                acc += (c[q] if q >= 0 else 0.0) * U[:, pa & 0x7FFF]
+                if q >= 0:
+                    dC[q] += U[:, pa & 0x7FFF] @ V[:, pb]
+                if (pa >> 16) != 0xFFFF:
+                    RG[:, pa >> 16] = acc
+                    acc = np.zeros(2)
+        for dst, src, cnt, _ in t["fixZ"]:
+            RZ[:, dst] += RZ[:, src:src + cnt].sum(axis=1)
+        for dst, src, cnt, _ in t["fixG"]:
+            RG[:, dst] += RG[:, src:src + cnt].sum(axis=1)
+        q = np.frombuffer(img[pt["q_offset"]:pt["q_offset"] + 4 * pt["nnz"]].tobytes(), np.int32)
+        al, bl = a_gm[q] - pt["m0"], b_gm[q] - pt["n0"]
+        Cl = adapter.dense_C(mv, nv, al, bl, c[q])
+        np.testing.assert_allclose(RZ[:, :mv], V @ Cl.T, atol=1e-12)
+        np.testing.assert_allclose(RG[:, :nv], U @ Cl, atol=1e-12)
+        np.testing.assert_allclose(dC[q], np.einsum("ta,tb->ab", U, V)[al, bl], atol=1e-12)
+        assert not np.any(np.delete(dC, q))      # a part writes only its own entries
