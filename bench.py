@@ -278,10 +278,16 @@ def oracle_step_estimate(w, tokens: int, mats=(0,)):
 
 
 def config_of(w, nmats: int, world: int) -> dict:
-    """The workload description both arms print."""
+    """The workload description both arms print.  The timed steps do not flush
+    L2: the bytes of X, dY, Y and dX one step touches say whether they can stay
+    in it (the full evaluation workloads: no; the small profiling cases: yes)."""
+    esz = 4 if w.dtype == "f32" else 2
+    touched = 2 * esz * w.N * sum(s.n + s.m for s in w.mats[:nmats])
+    l2 = (f"inputs larger than L2 ({touched / 2 ** 30:.0f} GiB of X, dY, Y and dX per step)" if touched > 2 * L2_BYTES
+          else f"{touched / 2 ** 20:.0f} MiB of X, dY, Y and dX per step, L2 not flushed (a profiling case)")
     return {"workload": w.name, "matrices": nmats, "tokens": w.N, "nnz": w.nnz,
             "shape": f"{w.mats[0].m}x{w.mats[0].n}", "k": w.k, "parallelism": "replicas" if world > 1 else "single",
-            "l2": "inputs larger than L2 (32 GB per step)"}
+            "l2": l2}
 
 
 def max_over_ranks(ms: float, world: int, device) -> float:
